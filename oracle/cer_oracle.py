@@ -1,0 +1,213 @@
+"""CPU oracle for CE-Router's token-routed compacted block.
+
+TEST INFRASTRUCTURE ONLY.  Only ``tests/``, ``__graft_entry__.smoke()`` and the
+``cpu_baseline`` / ``--impl reference`` legs of ``bench.py`` may import or run
+anything under ``oracle/``.  The CUDA library never calls it and it calls nothing
+of the CUDA library: the two share no code.
+
+Plain, slow, obviously correct: numpy in fp64 (the paper fixes no precision),
+one step per paper passage, no blocking, fusion or reordering.  Data arrive as
+the same bf16 bit patterns (uint16) and fp32 arrays the GPU reads; they are
+widened exactly to fp64.  Library primitives used as steps: numpy matmul,
+numpy exp/cos/sin/floor, scipy.special.erf, Python's ``sorted``.
+
+Paper passages followed (CE-Router, "Core-Expansion Routing and Unified
+Computation Scheduling"):
+  * Sec. 3.2, Eq. 1 (core_expansion_formulation): logits l^U = c_l(h),
+    l^G = c_l(h) + e_{l,m(t)}(h); core and expansions are token-wise MLPs with a
+    scalar output; M segments of the denoising timesteps.
+  * Sec. 3.4, Eq. 4 (router_inference_outputs): p = sigmoid(l), R = TopK(p, K);
+    App. B.2: the sigmoid is monotonic, so ranking logits gives the same set.
+  * Sec. 3.4, task-adaptive token compaction: R is packed into a shorter
+    sequence for the FFN, D bypasses unchanged.
+  * Sec. 3.4 (2) FFN pruning and App. A.4: FFN restricted to the channels kept
+    by the static mask; the backbone is Qwen2.5 (App. A.5), a SwiGLU FFN.
+
+Readings where the paper is silent or leaves a choice open:
+  * scorer MLP form w2 . GELU(W1 h + b1) with exact-erf GELU; expansion adds
+    U . emb(t) before the GELU, emb a sinusoid [cos(1000 t f_j), sin(1000 t f_j)],
+    f_j = 10000^(-j/(E/2)), computed in fp64 and rounded to fp32;
+  * segment m(t) = min(M-1, floor(t*M)) in fp64 (equal-width progress segments);
+  * ranking on fp32 logits, larger first, ties to the lower token index,
+    -0.0 equal to +0.0, a NaN among the routable logits is an error;
+  * tokens outside the routable range [r0, r1) are always kept; the kept list is
+    in ascending token order;
+  * FFN without biases or norm, y = W_down[:, Cs] (SiLU(W_gate[Cs] x) * (W_up[Cs] x));
+    the update is not scaled by p;
+  * block output bf16(h + y) for kept rows: the fp64 sum rounded to fp32, then
+    to bf16 (round to nearest even at both steps); dropped rows bit-identical.
+
+Parity status: every function below is pinned by tests/test_oracle_pins.py
+(hand-computed example, brute-force top-k, closed forms, library special cases,
+invariants).  Agreement with what the paper's authors ran is unpinned: the paper
+prints no numerical value of the router, the FFN or the block.
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+from scipy.special import erf
+
+TASK_UND = 0
+TASK_GEN = 1
+
+
+class OracleNaN(ValueError):
+    """A routable logit is NaN: no top-K set is defined."""
+
+
+# ---------------------------------------------------------------- bf16 <-> fp64
+
+def bf16_to_f64(bits: np.ndarray) -> np.ndarray:
+    """Exact widening of bf16 bit patterns (uint16) to fp64."""
+    b = np.ascontiguousarray(bits, dtype=np.uint16).astype(np.uint32) << np.uint32(16)
+    return b.view(np.float32).astype(np.float64)
+
+
+def round_to_bf16(x: np.ndarray) -> np.ndarray:
+    """fp64 -> fp32 (nearest even) -> bf16 (nearest even); returns uint16 bits."""
+    f = np.asarray(x, dtype=np.float64).astype(np.float32)
+    u = f.view(np.uint32).astype(np.uint64)
+    lsb = (u >> np.uint64(16)) & np.uint64(1)
+    r = (u + np.uint64(0x7FFF) + lsb) >> np.uint64(16)
+    out = r.astype(np.uint16)
+    nan = np.isnan(f)
+    out[nan] = 0x7FC0
+    return out
+
+
+# ---------------------------------------------------------------- scorer pieces
+
+def gelu(x: np.ndarray) -> np.ndarray:
+    """GELU with the exact Gaussian CDF: x * Phi(x) = 0.5 x (1 + erf(x / sqrt 2))."""
+    return 0.5 * x * (1.0 + erf(x / math.sqrt(2.0)))
+
+
+def sinusoidal_embedding(t: float, E: int) -> np.ndarray:
+    """E-dim progress embedding of t (reading: cos half then sin half), fp32."""
+    half = E // 2
+    j = np.arange(half, dtype=np.float64)
+    freq = np.power(10000.0, -j / half)
+    arg = 1000.0 * float(t) * freq
+    return np.concatenate([np.cos(arg), np.sin(arg)]).astype(np.float32)
+
+
+def segment_index(t: float, n_segments: int) -> int:
+    """m(t): the denoising segment holding progress t (Sec. 3.2; equal widths)."""
+    return int(min(n_segments - 1, math.floor(float(t) * n_segments)))
+
+
+def mlp_score(x: np.ndarray, W1: np.ndarray, w2: np.ndarray, bias: np.ndarray) -> np.ndarray:
+    """Token-wise MLP with scalar output (Sec. 3.2): w2 . GELU(W1 x + bias), per row of x."""
+    a = x @ W1.T + bias[None, :]
+    return gelu(a) @ w2
+
+
+def score(h, W1, w2, b1, t, task, W1e=None, w2e=None, Ue=None, b1e=None) -> np.ndarray:
+    """Routing logits of Eq. 1 for every token; returns fp32 [B, N].
+
+    h: bf16 bits [B, N, d].  Core: W1 bf16 [Hc, d], w2 fp32 [Hc], b1 fp32 [Hc] or None.
+    Expansion (generation only): W1e bf16 [S, He, d], w2e fp32 [S, He],
+    Ue bf16 [S, He, E] or None, b1e fp32 [S, He] or None; segment m(t_b) per sequence.
+    """
+    B, N, d = h.shape
+    hf = bf16_to_f64(h)
+    W1f = bf16_to_f64(W1)
+    w2f = np.asarray(w2, dtype=np.float64)
+    bc = np.zeros(W1.shape[0]) if b1 is None else np.asarray(b1, dtype=np.float64)
+    out = np.empty((B, N), dtype=np.float32)
+    for b in range(B):
+        logit = mlp_score(hf[b], W1f, w2f, bc)                      # l^U = c_l(h)
+        if task == TASK_GEN:
+            S = W1e.shape[0]
+            m = segment_index(t[b], S)
+            bias = np.zeros(W1e.shape[1])
+            if Ue is not None:
+                emb = sinusoidal_embedding(t[b], Ue.shape[2]).astype(np.float64)
+                bias = bias + bf16_to_f64(Ue[m]) @ emb
+            if b1e is not None:
+                bias = bias + np.asarray(b1e[m], dtype=np.float64)
+            logit = logit + mlp_score(hf[b], bf16_to_f64(W1e[m]),
+                                      np.asarray(w2e[m], dtype=np.float64), bias)
+        out[b] = logit.astype(np.float32)                           # l^G = c_l + e_{l,m(t)}
+    return out
+
+
+def sigmoid(x: np.ndarray) -> np.ndarray:
+    """Bounded importance p = sigmoid(l) of Eq. 4, in fp64."""
+    return 1.0 / (1.0 + np.exp(-np.asarray(x, dtype=np.float64)))
+
+
+# ---------------------------------------------------------------- selection
+
+def select_topk(logits: np.ndarray, r0: int, r1: int, K: int):
+    """Per-sequence keep set R (Eq. 4): the K routable tokens of largest logit
+    (ties to the lower index, -0.0 == +0.0) plus every token outside [r0, r1).
+
+    Returns idx int32 [B, k_tot] (ascending token order) and mask uint8 [B, N].
+    """
+    logits = np.asarray(logits, dtype=np.float32)
+    B, N = logits.shape
+    if not (0 <= r0 <= r1 <= N) or not (0 <= K <= r1 - r0):
+        raise ValueError("bad routable range or K")
+    k_tot = K + N - (r1 - r0)
+    idx = np.empty((B, k_tot), dtype=np.int32)
+    mask = np.zeros((B, N), dtype=np.uint8)
+    for b in range(B):
+        vals = [float(v) for v in logits[b]]
+        if any(math.isnan(vals[i]) for i in range(r0, r1)):
+            raise OracleNaN(f"NaN logit in sequence {b}")
+        ranked = sorted(range(r0, r1), key=lambda i: (-vals[i], i))
+        keep = set(ranked[:K]) | set(range(0, r0)) | set(range(r1, N))
+        kept = sorted(keep)
+        idx[b] = kept
+        mask[b, kept] = 1
+    return idx, mask
+
+
+# ---------------------------------------------------------------- compaction
+
+def gather(h: np.ndarray, idx: np.ndarray) -> np.ndarray:
+    """Pack R (Sec. 3.4): X[b * k_tot + j] = h[b, idx[b, j]]; bf16 bits [B*k_tot, d]."""
+    B, k_tot = idx.shape
+    return np.concatenate([h[b, idx[b]] for b in range(B)], axis=0) if B else \
+        np.empty((0, h.shape[2]), dtype=np.uint16)
+
+
+def routed_ffn(X: np.ndarray, Wg: np.ndarray, Wu: np.ndarray, WdT: np.ndarray,
+               chan: np.ndarray) -> np.ndarray:
+    """SwiGLU FFN on the packed rows restricted to the kept channels Cs; fp64 [M, d].
+
+    y = sum_{c in Cs} WdT[c, :] * SiLU(Wg[c] . x) * (Wu[c] . x), with WdT the
+    down projection stored channel-major (row c is W_down[:, c], the vector whose
+    norm enters the saliency of Eq. 5).
+    """
+    cs = np.asarray(chan, dtype=np.int64)
+    x = bf16_to_f64(X)
+    g = x @ bf16_to_f64(Wg[cs]).T
+    u = x @ bf16_to_f64(Wu[cs]).T
+    with np.errstate(over="ignore"):
+        a = g / (1.0 + np.exp(-g)) * u          # SiLU(g) * u, SiLU(g) = g * sigmoid(g)
+    return a @ bf16_to_f64(WdT[cs])
+
+
+def scatter_add(h: np.ndarray, idx: np.ndarray, Y: np.ndarray) -> np.ndarray:
+    """Unpack (Sec. 3.4): kept rows become bf16(h + y), dropped rows stay bit-identical."""
+    out = h.copy()
+    B, k_tot = idx.shape
+    for b in range(B):
+        rows = Y[b * k_tot:(b + 1) * k_tot]
+        out[b, idx[b]] = round_to_bf16(bf16_to_f64(h[b, idx[b]]) + rows)
+    return out
+
+
+def routed_block(h, W1, w2, b1, t, task, r0, r1, K, Wg, Wu, WdT, chan,
+                 W1e=None, w2e=None, Ue=None, b1e=None) -> dict:
+    """Whole routed block: score -> TopK -> gather -> pruned FFN -> scatter-add."""
+    logits = score(h, W1, w2, b1, t, task, W1e, w2e, Ue, b1e)
+    idx, mask = select_topk(logits, r0, r1, K)
+    X = gather(h, idx)
+    Y = routed_ffn(X, Wg, Wu, WdT, chan)
+    out = scatter_add(h, idx, Y)
+    return {"logits": logits, "idx": idx, "mask": mask, "Y": Y, "out": out}
