@@ -1,0 +1,195 @@
+/*
+ * cer_api.h -- C ABI of the GB300 (sm_103a) token-routed compacted block of
+ * CE-Router (core-expansion routing): score every token, keep the top-K per
+ * sequence, pack the kept rows, run a channel-pruned SwiGLU FFN on them and add
+ * the result back into the residual stream; dropped tokens bypass unchanged.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * Memory.   Every tensor argument is DEVICE memory owned by the caller, dense
+ *           row-major, on the device current when the call is made.  bf16
+ *           tensors are passed as `const void*` (2-byte IEEE bfloat16), fp32 as
+ *           float*, indices as int32_t*, masks as uint8_t*.  The library never
+ *           allocates device memory: entry points that need scratch take a
+ *           caller-supplied `workspace` of at least the size reported by the
+ *           matching *_workspace_size() function (256-byte aligned).
+ * Alignment. Every tensor pointer must be 16-byte aligned (CER_ERR_ALIGN).
+ * Streams.  Work is enqueued asynchronously on `stream` (0 = legacy default
+ *           stream); a call returns before the GPU finishes.
+ * Errors.   Argument checks run on the host before any launch: on failure
+ *           nothing is enqueued, the status is returned and a message is
+ *           available from cer_get_error() (per host thread).  Errors found
+ *           by a kernel (a NaN routable logit, a bounded wait that gave up,
+ *           an out-of-range index) are recorded in a per-device status word
+ *           that cer_sync_status() reads and clears.  Nothing throws across
+ *           the ABI.
+ * Device.   The library holds sm_103a code only; a call on another device
+ *           returns CER_ERR_DEVICE.
+ *
+ * Notation: B sequences of N tokens with hidden size d; routable range
+ * [r0, r1) with N_r = r1 - r0 tokens (tokens outside it are always kept);
+ * K routable tokens kept per sequence; k_tot = K + N - N_r kept per sequence;
+ * M = B * k_tot packed rows; I full FFN intermediate width; C kept channels.
+ */
+#ifndef CER_API_H
+#define CER_API_H
+
+#include <stddef.h>
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum cer_status {
+  CER_OK = 0,
+  CER_ERR_NULL = 1,      /* a required pointer is NULL                                  */
+  CER_ERR_SHAPE = 2,     /* a size is out of range or not a supported multiple          */
+  CER_ERR_ALIGN = 3,     /* a tensor pointer is not 16-byte aligned                     */
+  CER_ERR_RANGE = 4,     /* a count or index is out of range (K > N_r, r0 > r1, ...)    */
+  CER_ERR_NAN = 5,       /* device: a routable logit was NaN                            */
+  CER_ERR_DEVICE = 6,    /* not an sm_103 device, or a CUDA runtime error               */
+  CER_ERR_TIMEOUT = 7,   /* device: a bounded wait inside a kernel gave up              */
+  CER_ERR_LAUNCH = 8,    /* a kernel launch failed                                      */
+  CER_ERR_WORKSPACE = 9, /* workspace NULL or smaller than *_workspace_size() reports   */
+  CER_ERR_INDEX = 10     /* device: an index list entry was out of range                */
+} cer_status;
+
+typedef enum cer_task { CER_TASK_UND = 0, CER_TASK_GEN = 1 } cer_task;
+
+/*
+ * One token-wise scorer MLP with a scalar output (Sec. 3.2: the core scorer
+ * c_l, or the M generation expansion scorers e_{l,m}, one per denoising
+ * segment).  Score of a token h:  w2[m] . GELU(W1[m] h + b1[m] + U[m] emb(t)),
+ * GELU with the exact Gaussian CDF; emb(t) the E-dim sinusoid
+ * [cos(1000 t f_j), sin(1000 t f_j)], f_j = 10000^(-j/(E/2)), j < E/2.
+ * Segment m(t) = min(n_segments-1, floor(t * n_segments)) (equal-width
+ * progress segments).  The core has n_segments == 1 and no U.
+ */
+typedef struct cer_scorer {
+  const void*  W1;        /* bf16 [n_segments][hidden][d]                                  */
+  const float* b1;        /* fp32 [n_segments][hidden], or NULL for no bias                */
+  const float* w2;        /* fp32 [n_segments][hidden]                                     */
+  const void*  U;         /* bf16 [n_segments][hidden][emb_dim], or NULL (no time input)   */
+  int hidden;             /* hidden width, a multiple of 64, <= 4096                       */
+  int emb_dim;            /* even, <= 1024; ignored when U is NULL                         */
+  int n_segments;         /* >= 1, <= 64                                                   */
+} cer_scorer;
+
+/* ------------------------------------------------------------------ S1 score
+ * Routing logits of Eq. 1 (Sec. 3.2): l^U = c(h) for understanding,
+ * l^G = c(h) + e_{m(t)}(h) for generation.
+ *   h        bf16 [B, N, d]; d a multiple of 64, <= 16384
+ *   core     the core scorer (n_segments must be 1, U must be NULL)
+ *   exp      the expansion scorers; read only when task == CER_TASK_GEN
+ *            (may be NULL for CER_TASK_UND); its hidden width may differ
+ *   t        fp32 [B] denoising progress per sequence (read for CER_TASK_GEN)
+ *   logits   fp32 [B, N] output
+ *   probs    fp32 [B, N] output p = sigmoid(l) of Eq. 4, or NULL
+ * Workspace: cer_score_workspace_size(B, N, core->hidden, exp hidden, task).
+ * The GEMM runs on tcgen05 tensor cores (bf16 operands, fp32 accumulation);
+ * bias, GELU and the w2 dot product are applied in fp32.                     */
+cer_status cer_score(const void* h, int B, int N, int d,
+                     const cer_scorer* core, const cer_scorer* exp,
+                     const float* t, int task,
+                     float* logits, float* probs,
+                     void* workspace, size_t workspace_bytes, cudaStream_t stream);
+size_t cer_score_workspace_size(int B, int N, int core_hidden, int exp_hidden, int task);
+
+/* ------------------------------------------------------------------ S2 select
+ * Keep set R of Eq. 4 (Sec. 3.4) per sequence: the K tokens of [r0, r1) with
+ * the largest logit (ranking logits equals ranking sigmoid(l), App. B.2), ties
+ * to the lower token index, -0.0 equal to +0.0, -inf allowed; plus every
+ * token outside [r0, r1).  Exact: integer radix select on order-preserving
+ * keys of the fp32 bits.
+ *   logits   fp32 [B, N]
+ *   idx      int32 [B, k_tot] output, kept token indices in ascending order
+ *   mask     uint8 [B, N] output (1 = kept), or NULL
+ * A NaN logit inside [r0, r1) sets CER_ERR_NAN in the device status word (the
+ * outputs are then unspecified).  N <= 49152.                                 */
+cer_status cer_select_topk(const float* logits, int B, int N, int r0, int r1, int K,
+                           int32_t* idx, uint8_t* mask, cudaStream_t stream);
+
+/* ------------------------------------------------------------------ S3 gather
+ * Token compaction (Sec. 3.4): X[b*k_tot + j, :] = h[b, idx[b, j], :].
+ *   h bf16 [B, N, d] (d a multiple of 8), idx int32 [B, k_tot], X bf16 [B*k_tot, d].
+ * An index outside [0, N) sets CER_ERR_INDEX and its row is left unwritten.   */
+cer_status cer_gather(const void* h, int B, int N, int d, const int32_t* idx, int k_tot,
+                      void* X, cudaStream_t stream);
+
+/* ------------------------------------------------------------------ S4 FFN
+ * Channel-pruned SwiGLU FFN on the packed rows (Sec. 3.4 FFN pruning; Qwen2.5
+ * backbone of App. A.5):
+ *   Y[m, :] = sum_{c in Cs} WdT[c, :] * SiLU(Wg[c] . X[m]) * (Wu[c] . X[m])
+ *   X     bf16 [M, d], d a multiple of 64
+ *   Wg,Wu bf16 [I, d]   gate and up projections, one row per channel
+ *   WdT   bf16 [I, d]   down projection stored channel-major (row c is
+ *                       W_down[:, c]), so that pruning is a row selection
+ *   chan  int32 [C] kept channel indices in [0, I), or NULL for all (C == I);
+ *         C a multiple of 64
+ *   Y     bf16 [M, d] output
+ * Two tcgen05 GEMMs (bf16 operands, fp32 accumulation in TMEM); the kept
+ * weight rows are fetched by TMA row gathers straight from the full weights.
+ * The SwiGLU activation passes through the workspace as bf16 [M, C].
+ * Workspace: cer_routed_ffn_workspace_size(M, C).                            */
+cer_status cer_routed_ffn(const void* X, int M, int d,
+                          const void* Wg, const void* Wu, const void* WdT, int I,
+                          const int32_t* chan, int C, void* Y,
+                          void* workspace, size_t workspace_bytes, cudaStream_t stream);
+size_t cer_routed_ffn_workspace_size(int M, int C);
+
+/* ------------------------------------------------------------------ S5 scatter
+ * Unpack (Sec. 3.4): h[b, idx[b, j], :] = bf16(h + Y[b*k_tot + j, :]) in place,
+ * fp32 sum rounded to nearest even; rows not in idx are not touched.
+ *   h bf16 [B, N, d] (d a multiple of 8), idx int32 [B, k_tot] without
+ *   duplicates within a sequence, Y bf16 [B*k_tot, d].                        */
+cer_status cer_scatter_add(void* h, int B, int N, int d, const int32_t* idx, int k_tot,
+                           const void* Y, cudaStream_t stream);
+
+/* ------------------------------------------------------------------ fused block
+ * The whole routed block S1..S5 in four kernels on one stream:
+ *   scorer GEMM -> top-K (also reduces the scorer's partial sums) ->
+ *   gate/up GEMM reading the kept rows of h by TMA row gather ->
+ *   down GEMM whose epilogue adds into the kept rows of the output.
+ *   h, out   bf16 [B, N, d]; out == h (or NULL) updates h in place and moves
+ *            no bytes for dropped rows; otherwise out must not overlap h and
+ *            dropped rows are copied (bypass)
+ *   core, exp, t, task   as for cer_score
+ *   r0, r1, K            as for cer_select_topk
+ *   Wg, Wu, WdT, I, chan, C   as for cer_routed_ffn
+ *   logits   fp32 [B, N] output, or NULL
+ *   idx      int32 [B, k_tot] output, or NULL
+ *   mask     uint8 [B, N] output, or NULL
+ *   stage_events  NULL, or n_stage_events == 5 caller-created CUDA events
+ *            recorded on `stream` before the scorer, after the scorer, after
+ *            the top-K, after the gate/up GEMM and after the down GEMM (for
+ *            per-stage timing).
+ * Workspace: cer_routed_block_workspace_size(...) with the same sizes.      */
+cer_status cer_routed_block(void* h, void* out, int B, int N, int d,
+                            const cer_scorer* core, const cer_scorer* exp,
+                            const float* t, int task, int r0, int r1, int K,
+                            const void* Wg, const void* Wu, const void* WdT, int I,
+                            const int32_t* chan, int C,
+                            float* logits, int32_t* idx, uint8_t* mask,
+                            void* workspace, size_t workspace_bytes,
+                            cudaEvent_t* stage_events, int n_stage_events,
+                            cudaStream_t stream);
+size_t cer_routed_block_workspace_size(int B, int N, int d, int core_hidden, int exp_hidden,
+                                       int task, int r0, int r1, int K, int C);
+
+/* ------------------------------------------------------------------ status
+ * cer_sync_status: synchronise `stream`, then return and clear the current
+ * device's status word (the first kernel-detected error since the last call),
+ * or CER_ERR_DEVICE if the synchronisation itself failed.
+ * cer_get_error: message of the last failing call on this host thread.
+ * cer_status_string: name of a status code.  cer_version: ABI version.     */
+cer_status  cer_sync_status(cudaStream_t stream);
+const char* cer_get_error(void);
+const char* cer_status_string(cer_status s);
+int         cer_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* CER_API_H */

@@ -1,0 +1,198 @@
+"""Python binding of libcer.so (include/cer_api.h): argument marshalling only.
+
+Every function named ``cer_*`` here calls the C entry point of the same name
+with the device pointers of torch tensors, the sizes read off their shapes and
+the current CUDA stream.  No computation happens in Python; there is no CPU or
+PyTorch fallback: if the library is missing or the device is not sm_103 the
+call raises.  PyTorch supplies device memory and streams only.
+"""
+from __future__ import annotations
+
+import ctypes
+import dataclasses
+import os
+from typing import Optional, Sequence
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libcer.so")
+
+TASK_UND = 0
+TASK_GEN = 1
+
+STATUS_NAMES = {0: "CER_OK", 1: "CER_ERR_NULL", 2: "CER_ERR_SHAPE", 3: "CER_ERR_ALIGN", 4: "CER_ERR_RANGE",
+                5: "CER_ERR_NAN", 6: "CER_ERR_DEVICE", 7: "CER_ERR_TIMEOUT", 8: "CER_ERR_LAUNCH",
+                9: "CER_ERR_WORKSPACE", 10: "CER_ERR_INDEX"}
+
+# Every symbol include/cer_api.h declares.
+EXPORTS = ("cer_score", "cer_score_workspace_size", "cer_select_topk", "cer_gather", "cer_routed_ffn",
+           "cer_routed_ffn_workspace_size", "cer_scatter_add", "cer_routed_block",
+           "cer_routed_block_workspace_size", "cer_sync_status", "cer_get_error", "cer_status_string",
+           "cer_version")
+
+
+class CerError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"{STATUS_NAMES.get(status, status)}: {message}")
+        self.status = status
+
+
+class CerScorerC(ctypes.Structure):
+    _fields_ = [("W1", ctypes.c_void_p), ("b1", ctypes.c_void_p), ("w2", ctypes.c_void_p),
+                ("U", ctypes.c_void_p), ("hidden", ctypes.c_int), ("emb_dim", ctypes.c_int),
+                ("n_segments", ctypes.c_int)]
+
+
+_lib = None
+
+_vp, _i, _sz, _f = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t, ctypes.c_float
+_SCP = ctypes.POINTER(CerScorerC)
+_SIGS = {
+    "cer_score": ([_vp, _i, _i, _i, _SCP, _SCP, _vp, _i, _vp, _vp, _vp, _sz, _vp], _i),
+    "cer_score_workspace_size": ([_i, _i, _i, _i, _i], _sz),
+    "cer_select_topk": ([_vp, _i, _i, _i, _i, _i, _vp, _vp, _vp], _i),
+    "cer_gather": ([_vp, _i, _i, _i, _vp, _i, _vp, _vp], _i),
+    "cer_routed_ffn": ([_vp, _i, _i, _vp, _vp, _vp, _i, _vp, _i, _vp, _vp, _sz, _vp], _i),
+    "cer_routed_ffn_workspace_size": ([_i, _i], _sz),
+    "cer_scatter_add": ([_vp, _i, _i, _i, _vp, _i, _vp, _vp], _i),
+    "cer_routed_block": ([_vp, _vp, _i, _i, _i, _SCP, _SCP, _vp, _i, _i, _i, _i, _vp, _vp, _vp, _i, _vp, _i,
+                          _vp, _vp, _vp, _vp, _sz, _vp, _i, _vp], _i),
+    "cer_routed_block_workspace_size": ([_i, _i, _i, _i, _i, _i, _i, _i, _i, _i], _sz),
+    "cer_sync_status": ([_vp], _i),
+    "cer_get_error": ([], ctypes.c_char_p),
+    "cer_status_string": ([_i], ctypes.c_char_p),
+    "cer_version": ([], _i),
+}
+
+
+def load(path: str = LIB_PATH) -> ctypes.CDLL:
+    """Load libcer.so (once).  Raises if it has not been built."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(path):
+            raise RuntimeError(f"{path} is missing: build it with __graft_entry__.build()")
+        lib = ctypes.CDLL(path)
+        for name, (args, res) in _SIGS.items():
+            fn = getattr(lib, name)
+            fn.argtypes = args
+            fn.restype = res
+        _lib = lib
+    return _lib
+
+
+def _check(status: int) -> None:
+    if status != 0:
+        raise CerError(status, load().cer_get_error().decode())
+
+
+def _p(t: Optional[torch.Tensor]):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+@dataclasses.dataclass
+class Scorer:
+    """One scorer MLP (core: W1 [H, d]; expansions: W1 [S, H, d]) on the device.
+
+    W1 and U are bf16, w2 and b1 fp32.  See ``cer_scorer`` in cer_api.h.
+    """
+    W1: torch.Tensor
+    w2: torch.Tensor
+    b1: Optional[torch.Tensor] = None
+    U: Optional[torch.Tensor] = None
+
+    def c_struct(self) -> CerScorerC:
+        S = 1 if self.W1.dim() == 2 else self.W1.shape[0]
+        return CerScorerC(_p(self.W1), _p(self.b1), _p(self.w2), _p(self.U), int(self.W1.shape[-2]),
+                          int(self.U.shape[-1]) if self.U is not None else 0, int(S))
+
+
+def _sref(s: Optional[Scorer]):
+    return None if s is None else ctypes.pointer(s.c_struct())
+
+
+def workspace(nbytes: int, device) -> torch.Tensor:
+    return torch.empty(max(int(nbytes), 256), dtype=torch.uint8, device=device)
+
+
+# ------------------------------------------------------------------ entry points
+
+def cer_score_workspace_size(B, N, core_hidden, exp_hidden, task) -> int:
+    return load().cer_score_workspace_size(B, N, core_hidden, exp_hidden, task)
+
+
+def cer_score(h, core: Scorer, exp: Optional[Scorer], t, task, logits, probs=None, ws=None, stream=None):
+    B, N, d = h.shape
+    need = cer_score_workspace_size(B, N, core.W1.shape[-2], exp.W1.shape[-2] if exp is not None else 0, task)
+    if ws is None:
+        ws = workspace(need, h.device)
+    _check(load().cer_score(_p(h), B, N, d, _sref(core), _sref(exp), _p(t), task, _p(logits), _p(probs),
+                            _p(ws), ws.numel(), _stream(stream)))
+
+
+def cer_select_topk(logits, r0, r1, K, idx, mask=None, stream=None):
+    B, N = logits.shape
+    _check(load().cer_select_topk(_p(logits), B, N, r0, r1, K, _p(idx), _p(mask), _stream(stream)))
+
+
+def cer_gather(h, idx, X, stream=None):
+    B, N, d = h.shape
+    _check(load().cer_gather(_p(h), B, N, d, _p(idx), idx.shape[1], _p(X), _stream(stream)))
+
+
+def cer_routed_ffn_workspace_size(M, C) -> int:
+    return load().cer_routed_ffn_workspace_size(M, C)
+
+
+def cer_routed_ffn(X, Wg, Wu, WdT, chan, Y, ws=None, stream=None):
+    M, d = X.shape
+    I = Wg.shape[0]
+    C = I if chan is None else chan.numel()
+    if ws is None:
+        ws = workspace(cer_routed_ffn_workspace_size(M, C), X.device)
+    _check(load().cer_routed_ffn(_p(X), M, d, _p(Wg), _p(Wu), _p(WdT), I, _p(chan), C, _p(Y), _p(ws), ws.numel(),
+                                 _stream(stream)))
+
+
+def cer_scatter_add(h, idx, Y, stream=None):
+    B, N, d = h.shape
+    _check(load().cer_scatter_add(_p(h), B, N, d, _p(idx), idx.shape[1], _p(Y), _stream(stream)))
+
+
+def cer_routed_block_workspace_size(B, N, d, core_hidden, exp_hidden, task, r0, r1, K, C) -> int:
+    return load().cer_routed_block_workspace_size(B, N, d, core_hidden, exp_hidden, task, r0, r1, K, C)
+
+
+def cer_routed_block(h, core: Scorer, exp: Optional[Scorer], t, task, r0, r1, K, Wg, Wu, WdT, chan,
+                     out=None, logits=None, idx=None, mask=None, ws=None,
+                     stage_events: Optional[Sequence[torch.cuda.Event]] = None, stream=None):
+    """The fused routed block; updates h in place when ``out`` is None or h."""
+    B, N, d = h.shape
+    I = Wg.shape[0]
+    C = I if chan is None else chan.numel()
+    eh = exp.W1.shape[-2] if exp is not None else 0
+    if ws is None:
+        ws = workspace(cer_routed_block_workspace_size(B, N, d, core.W1.shape[-2], eh, task, r0, r1, K, C),
+                       h.device)
+    ev_arr, n_ev = None, 0
+    if stage_events is not None:
+        handles = []
+        for ev in stage_events:
+            if ev.cuda_event == 0:     # torch creates the event lazily: force it
+                ev.record()
+            handles.append(ev.cuda_event)
+        ev_arr = (ctypes.c_void_p * len(handles))(*handles)
+        n_ev = len(handles)
+    _check(load().cer_routed_block(_p(h), _p(out), B, N, d, _sref(core), _sref(exp), _p(t), task, r0, r1, K,
+                                   _p(Wg), _p(Wu), _p(WdT), I, _p(chan), C, _p(logits), _p(idx), _p(mask),
+                                   _p(ws), ws.numel(), ev_arr, n_ev, _stream(stream)))
+
+
+def cer_sync_status(stream=None) -> None:
+    """Synchronise the stream and raise if a kernel recorded an error."""
+    _check(load().cer_sync_status(_stream(stream)))

@@ -1,0 +1,564 @@
+// cer_api.cu -- the C ABI declared in include/cer_api.h: host-side argument
+// checks, workspace carving, tensor-map encoding, per-device state (SM count,
+// architecture check, the device status word) and the launch sequences.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_runtime.h>
+
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <set>
+#include <string>
+#include <utility>
+
+#include "../../include/cer_api.h"
+#include "kernels.h"
+
+namespace {
+
+// ---------------------------------------------------------------- errors
+
+thread_local std::string g_error;
+
+cer_status fail(cer_status s, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_error = buf;
+  return s;
+}
+
+cer_status cuda_fail(cudaError_t e, const char* where) {
+  return fail(e == cudaErrorLaunchFailure || e == cudaErrorInvalidConfiguration ? CER_ERR_LAUNCH : CER_ERR_DEVICE,
+              "%s: %s", where, cudaGetErrorString(e));
+}
+
+// ---------------------------------------------------------------- per device
+
+__device__ int g_status_word;  // first kernel-detected error on this device
+
+constexpr int kMaxDevices = 64;
+
+struct DeviceInfo {
+  bool ready = false;
+  bool supported = false;
+  int n_sm = 0;
+  int* status = nullptr;  // device address of g_status_word
+};
+
+std::mutex g_dev_mu;
+DeviceInfo g_dev[kMaxDevices];
+
+cer_status device_info(DeviceInfo** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev < 0 || dev >= kMaxDevices) return fail(CER_ERR_DEVICE, "device index %d out of range", dev);
+  std::lock_guard<std::mutex> lk(g_dev_mu);
+  DeviceInfo& d = g_dev[dev];
+  if (!d.ready) {
+    int major = 0, minor = 0;
+    cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+    cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+    d.supported = (major == 10 && minor == 3);
+    cudaDeviceGetAttribute(&d.n_sm, cudaDevAttrMultiProcessorCount, dev);
+    if (d.supported) {
+      e = cudaGetSymbolAddress(reinterpret_cast<void**>(&d.status), g_status_word);
+      if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(status)");
+    }
+    d.ready = true;
+  }
+  if (!d.supported) return fail(CER_ERR_DEVICE, "device %d is not an sm_103 GPU; this library holds sm_103a code only", dev);
+  *out = &d;
+  return CER_OK;
+}
+
+// ---------------------------------------------------------------- checks
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+size_t round256(size_t x) { return (x + 255) & ~size_t(255); }
+
+#define CER_REQUIRE(cond, status, ...) \
+  do {                                 \
+    if (!(cond)) return fail(status, __VA_ARGS__); \
+  } while (0)
+
+#define CER_PTR(p) CER_REQUIRE((p) != nullptr, CER_ERR_NULL, "%s is NULL", #p)
+#define CER_ALIGN(p) CER_REQUIRE((p) == nullptr || aligned16(p), CER_ERR_ALIGN, "%s is not 16-byte aligned", #p)
+
+struct ScoreShape {
+  int Hc = 0, He = 0, gen = 0, n_chunks = 0, Ht = 0;
+};
+
+cer_status check_scorer(const cer_scorer* s, const char* name, bool is_core, int* hidden) {
+  if (s == nullptr) return fail(CER_ERR_NULL, "%s scorer is NULL", name);
+  if (s->W1 == nullptr || s->w2 == nullptr) return fail(CER_ERR_NULL, "%s scorer W1/w2 is NULL", name);
+  if (!aligned16(s->W1) || !aligned16(s->w2) || (s->b1 && !aligned16(s->b1)) || (s->U && !aligned16(s->U)))
+    return fail(CER_ERR_ALIGN, "%s scorer tensors must be 16-byte aligned", name);
+  if (s->hidden < 64 || s->hidden > 4096 || s->hidden % 64 != 0)
+    return fail(CER_ERR_SHAPE, "%s scorer hidden=%d must be a multiple of 64 in [64, 4096]", name, s->hidden);
+  if (s->n_segments < 1 || s->n_segments > 64)
+    return fail(CER_ERR_SHAPE, "%s scorer n_segments=%d must be in [1, 64]", name, s->n_segments);
+  if (is_core && (s->n_segments != 1 || s->U != nullptr))
+    return fail(CER_ERR_SHAPE, "the core scorer is shared by all tasks: n_segments must be 1 and U NULL");
+  if (s->U != nullptr && (s->emb_dim < 2 || s->emb_dim > 1024 || s->emb_dim % 2 != 0))
+    return fail(CER_ERR_SHAPE, "%s scorer emb_dim=%d must be even in [2, 1024]", name, s->emb_dim);
+  *hidden = s->hidden;
+  return CER_OK;
+}
+
+cer_status check_score_args(const void* h, int B, int N, int d, const cer_scorer* core, const cer_scorer* exp,
+                            const float* t, int task, ScoreShape* sh) {
+  CER_PTR(h);
+  CER_ALIGN(h);
+  CER_ALIGN(t);
+  CER_REQUIRE(task == CER_TASK_UND || task == CER_TASK_GEN, CER_ERR_RANGE, "task=%d is neither UND nor GEN", task);
+  CER_REQUIRE(B >= 0 && N >= 0, CER_ERR_SHAPE, "B=%d N=%d must be >= 0", B, N);
+  CER_REQUIRE(static_cast<long long>(B) * N < (1ll << 31), CER_ERR_SHAPE, "B*N too large");
+  CER_REQUIRE(d >= 64 && d <= 16384 && d % 64 == 0, CER_ERR_SHAPE, "d=%d must be a multiple of 64 in [64, 16384]", d);
+  cer_status s = check_scorer(core, "core", true, &sh->Hc);
+  if (s != CER_OK) return s;
+  sh->gen = (task == CER_TASK_GEN);
+  if (sh->gen) {
+    s = check_scorer(exp, "expansion", false, &sh->He);
+    if (s != CER_OK) return s;
+    CER_PTR(t);
+  }
+  const int bn = cer::score_chunk_width(sh->Hc, sh->He, sh->gen);
+  CER_REQUIRE(bn > 0, CER_ERR_SHAPE, "scorer hidden widths must be multiples of 64");
+  sh->Ht = sh->Hc + (sh->gen ? sh->He : 0);
+  sh->n_chunks = sh->Ht / bn;
+  return CER_OK;
+}
+
+size_t score_ws_bytes(int B, int N, const ScoreShape& sh) {
+  return 2 * round256(static_cast<size_t>(B) * sh.Ht * sizeof(float)) +
+         round256(static_cast<size_t>(sh.n_chunks) * B * N * sizeof(float));
+}
+
+cer::ScoreWorkspace carve_score_ws(void* ws, int B, int N, const ScoreShape& sh) {
+  char* p = static_cast<char*>(ws);
+  cer::ScoreWorkspace w;
+  const size_t tab = round256(static_cast<size_t>(B) * sh.Ht * sizeof(float));
+  w.bias_tab = reinterpret_cast<float*>(p);
+  w.w2_tab = reinterpret_cast<float*>(p + tab);
+  w.partial = reinterpret_cast<float*>(p + 2 * tab);
+  return w;
+}
+
+cer::ScoreArgs make_score_args(const void* h, int B, int N, int d, const cer_scorer* core, const cer_scorer* exp,
+                               const float* t, const ScoreShape& sh, int* status) {
+  cer::ScoreArgs a{};
+  a.h = static_cast<const __nv_bfloat16*>(h);
+  a.B = B;
+  a.N = N;
+  a.d = d;
+  a.W1 = static_cast<const __nv_bfloat16*>(core->W1);
+  a.b1 = core->b1;
+  a.w2 = core->w2;
+  a.Hc = sh.Hc;
+  a.gen = sh.gen;
+  a.t = t;
+  a.S = 1;
+  if (sh.gen) {
+    a.W1e = static_cast<const __nv_bfloat16*>(exp->W1);
+    a.b1e = exp->b1;
+    a.w2e = exp->w2;
+    a.U = static_cast<const __nv_bfloat16*>(exp->U);
+    a.He = sh.He;
+    a.E = exp->U ? exp->emb_dim : 0;
+    a.S = exp->n_segments;
+  }
+  a.status = status;
+  return a;
+}
+
+cer_status check_ffn_shape(int M, int d, int I, const int32_t* chan, int C) {
+  CER_REQUIRE(M >= 0, CER_ERR_SHAPE, "M=%d must be >= 0", M);
+  CER_REQUIRE(d >= 64 && d <= 16384 && d % 64 == 0, CER_ERR_SHAPE, "d=%d must be a multiple of 64 in [64, 16384]", d);
+  CER_REQUIRE(I >= 1, CER_ERR_SHAPE, "I=%d must be >= 1", I);
+  CER_REQUIRE(C >= 64 && C <= I && C % 64 == 0, CER_ERR_SHAPE, "C=%d must be a multiple of 64 in [64, I=%d]", C, I);
+  CER_REQUIRE(chan != nullptr || C == I, CER_ERR_SHAPE, "chan == NULL requires C == I (C=%d, I=%d)", C, I);
+  return CER_OK;
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------- internal helpers
+
+namespace cer {
+
+bool encode_bf16_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_cols,
+                    uint32_t box_rows) {
+  static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    cudaDriverEntryPointQueryResult q;
+    void* fn = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  });
+  if (encode == nullptr || rows == 0 || cols == 0) return false;
+  const cuuint64_t dims[2] = {cols, rows};
+  const cuuint64_t strides[1] = {cols * 2};
+  const cuuint32_t box[2] = {box_cols, box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  return encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+cudaError_t ensure_max_smem(const void* func, size_t bytes) {
+  static std::mutex mu;
+  static std::set<std::pair<int, const void*>> done;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> lk(mu);
+  if (done.count({dev, func})) return cudaSuccess;
+  e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes));
+  if (e == cudaSuccess) done.insert({dev, func});
+  return e;
+}
+
+}  // namespace cer
+
+// ---------------------------------------------------------------- the ABI
+
+extern "C" {
+
+int cer_version(void) { return 1; }
+
+const char* cer_get_error(void) { return g_error.c_str(); }
+
+const char* cer_status_string(cer_status s) {
+  switch (s) {
+    case CER_OK: return "CER_OK";
+    case CER_ERR_NULL: return "CER_ERR_NULL";
+    case CER_ERR_SHAPE: return "CER_ERR_SHAPE";
+    case CER_ERR_ALIGN: return "CER_ERR_ALIGN";
+    case CER_ERR_RANGE: return "CER_ERR_RANGE";
+    case CER_ERR_NAN: return "CER_ERR_NAN";
+    case CER_ERR_DEVICE: return "CER_ERR_DEVICE";
+    case CER_ERR_TIMEOUT: return "CER_ERR_TIMEOUT";
+    case CER_ERR_LAUNCH: return "CER_ERR_LAUNCH";
+    case CER_ERR_WORKSPACE: return "CER_ERR_WORKSPACE";
+    case CER_ERR_INDEX: return "CER_ERR_INDEX";
+  }
+  return "CER_UNKNOWN";
+}
+
+cer_status cer_sync_status(cudaStream_t stream) {
+  DeviceInfo* dev = nullptr;
+  cer_status s = device_info(&dev);
+  if (s != CER_OK) return s;
+  cudaError_t e = cudaStreamSynchronize(stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+  int v = 0;
+  e = cudaMemcpy(&v, dev->status, sizeof(int), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "reading the status word");
+  if (v != 0) {
+    const int zero = 0;
+    e = cudaMemcpy(dev->status, &zero, sizeof(int), cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return cuda_fail(e, "clearing the status word");
+    return fail(static_cast<cer_status>(v), "device reported %s", cer_status_string(static_cast<cer_status>(v)));
+  }
+  return CER_OK;
+}
+
+size_t cer_score_workspace_size(int B, int N, int core_hidden, int exp_hidden, int task) {
+  ScoreShape sh;
+  sh.Hc = core_hidden;
+  sh.He = exp_hidden;
+  sh.gen = (task == CER_TASK_GEN);
+  const int bn = cer::score_chunk_width(sh.Hc, sh.He, sh.gen);
+  if (bn == 0 || B < 0 || N < 0) return 0;
+  sh.Ht = sh.Hc + (sh.gen ? sh.He : 0);
+  sh.n_chunks = sh.Ht / bn;
+  return score_ws_bytes(B, N, sh);
+}
+
+cer_status cer_score(const void* h, int B, int N, int d, const cer_scorer* core, const cer_scorer* exp,
+                     const float* t, int task, float* logits, float* probs, void* workspace,
+                     size_t workspace_bytes, cudaStream_t stream) {
+  ScoreShape sh;
+  cer_status s = check_score_args(h, B, N, d, core, exp, t, task, &sh);
+  if (s != CER_OK) return s;
+  CER_PTR(logits);
+  CER_ALIGN(logits);
+  CER_ALIGN(probs);
+  CER_ALIGN(workspace);
+  const size_t need = score_ws_bytes(B, N, sh);
+  CER_REQUIRE(workspace != nullptr && workspace_bytes >= need, CER_ERR_WORKSPACE,
+              "workspace of %zu bytes needed, %zu given", need, workspace_bytes);
+  DeviceInfo* dev = nullptr;
+  if ((s = device_info(&dev)) != CER_OK) return s;
+  if (B == 0 || N == 0) return CER_OK;
+  cer::ScoreWorkspace ws = carve_score_ws(workspace, B, N, sh);
+  cer::ScoreArgs a = make_score_args(h, B, N, d, core, exp, t, sh, dev->status);
+  cudaError_t e = cer::launch_score(a, ws, dev->n_sm, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "scorer launch");
+  e = cer::launch_score_reduce(ws.partial, sh.n_chunks, static_cast<size_t>(B) * N, logits, probs, dev->n_sm,
+                               stream);
+  if (e != cudaSuccess) return cuda_fail(e, "score reduce launch");
+  return CER_OK;
+}
+
+cer_status cer_select_topk(const float* logits, int B, int N, int r0, int r1, int K, int32_t* idx, uint8_t* mask,
+                           cudaStream_t stream) {
+  CER_PTR(logits);
+  CER_PTR(idx);
+  CER_ALIGN(logits);
+  CER_ALIGN(idx);
+  CER_ALIGN(mask);
+  CER_REQUIRE(B >= 0 && N >= 0 && N <= cer::kTopkMaxN, CER_ERR_SHAPE, "B=%d N=%d (N <= %d)", B, N, cer::kTopkMaxN);
+  CER_REQUIRE(0 <= r0 && r0 <= r1 && r1 <= N, CER_ERR_RANGE, "routable range [%d, %d) not inside [0, %d]", r0, r1, N);
+  CER_REQUIRE(0 <= K && K <= r1 - r0, CER_ERR_RANGE, "K=%d not in [0, N_r=%d]", K, r1 - r0);
+  DeviceInfo* dev = nullptr;
+  cer_status s = device_info(&dev);
+  if (s != CER_OK) return s;
+  cer::TopkArgs a{};
+  a.src = logits;
+  a.n_chunks = 1;
+  a.chunk_stride = 0;
+  a.B = B;
+  a.N = N;
+  a.r0 = r0;
+  a.r1 = r1;
+  a.K = K;
+  a.idx = idx;
+  a.mask = mask;
+  a.status = dev->status;
+  cudaError_t e = cer::launch_topk(a, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "top-K launch");
+  return CER_OK;
+}
+
+cer_status cer_gather(const void* h, int B, int N, int d, const int32_t* idx, int k_tot, void* X,
+                      cudaStream_t stream) {
+  CER_PTR(h);
+  CER_PTR(idx);
+  CER_PTR(X);
+  CER_ALIGN(h);
+  CER_ALIGN(idx);
+  CER_ALIGN(X);
+  CER_REQUIRE(B >= 0 && N >= 0 && k_tot >= 0 && k_tot <= N, CER_ERR_SHAPE, "B=%d N=%d k_tot=%d", B, N, k_tot);
+  CER_REQUIRE(d > 0 && d % 8 == 0, CER_ERR_SHAPE, "d=%d must be a positive multiple of 8", d);
+  DeviceInfo* dev = nullptr;
+  cer_status s = device_info(&dev);
+  if (s != CER_OK) return s;
+  cudaError_t e = cer::launch_gather(static_cast<const __nv_bfloat16*>(h), B, N, d, idx, k_tot,
+                                     static_cast<__nv_bfloat16*>(X), dev->status, dev->n_sm, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "gather launch");
+  return CER_OK;
+}
+
+cer_status cer_scatter_add(void* h, int B, int N, int d, const int32_t* idx, int k_tot, const void* Y,
+                           cudaStream_t stream) {
+  CER_PTR(h);
+  CER_PTR(idx);
+  CER_PTR(Y);
+  CER_ALIGN(h);
+  CER_ALIGN(idx);
+  CER_ALIGN(Y);
+  CER_REQUIRE(B >= 0 && N >= 0 && k_tot >= 0 && k_tot <= N, CER_ERR_SHAPE, "B=%d N=%d k_tot=%d", B, N, k_tot);
+  CER_REQUIRE(d > 0 && d % 8 == 0, CER_ERR_SHAPE, "d=%d must be a positive multiple of 8", d);
+  DeviceInfo* dev = nullptr;
+  cer_status s = device_info(&dev);
+  if (s != CER_OK) return s;
+  cudaError_t e = cer::launch_scatter_add(static_cast<__nv_bfloat16*>(h), B, N, d, idx, k_tot,
+                                          static_cast<const __nv_bfloat16*>(Y), dev->status, dev->n_sm, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "scatter-add launch");
+  return CER_OK;
+}
+
+size_t cer_routed_ffn_workspace_size(int M, int C) {
+  if (M < 0 || C < 0) return 0;
+  return round256(static_cast<size_t>(M) * C * 2);
+}
+
+cer_status cer_routed_ffn(const void* X, int M, int d, const void* Wg, const void* Wu, const void* WdT, int I,
+                          const int32_t* chan, int C, void* Y, void* workspace, size_t workspace_bytes,
+                          cudaStream_t stream) {
+  CER_PTR(X);
+  CER_PTR(Wg);
+  CER_PTR(Wu);
+  CER_PTR(WdT);
+  CER_PTR(Y);
+  CER_ALIGN(X);
+  CER_ALIGN(Wg);
+  CER_ALIGN(Wu);
+  CER_ALIGN(WdT);
+  CER_ALIGN(chan);
+  CER_ALIGN(Y);
+  CER_ALIGN(workspace);
+  cer_status s = check_ffn_shape(M, d, I, chan, C);
+  if (s != CER_OK) return s;
+  const size_t need = cer_routed_ffn_workspace_size(M, C);
+  CER_REQUIRE(M == 0 || (workspace != nullptr && workspace_bytes >= need), CER_ERR_WORKSPACE,
+              "workspace of %zu bytes needed, %zu given", need, workspace_bytes);
+  DeviceInfo* dev = nullptr;
+  if ((s = device_info(&dev)) != CER_OK) return s;
+  if (M == 0) return CER_OK;
+  cer::FfnArgs a{};
+  a.X = static_cast<const __nv_bfloat16*>(X);
+  a.M = M;
+  a.d = d;
+  a.I = I;
+  a.C = C;
+  a.N = 0;
+  a.k_tot = 1;
+  a.Wg = static_cast<const __nv_bfloat16*>(Wg);
+  a.Wu = static_cast<const __nv_bfloat16*>(Wu);
+  a.WdT = static_cast<const __nv_bfloat16*>(WdT);
+  a.chan = chan;
+  a.act = static_cast<__nv_bfloat16*>(workspace);
+  a.Y = static_cast<__nv_bfloat16*>(Y);
+  a.scatter = 0;
+  a.status = dev->status;
+  cudaError_t e = cer::launch_ffn_gateup(a, dev->n_sm, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "gate/up GEMM launch");
+  e = cer::launch_ffn_down(a, dev->n_sm, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "down GEMM launch");
+  return CER_OK;
+}
+
+size_t cer_routed_block_workspace_size(int B, int N, int d, int core_hidden, int exp_hidden, int task, int r0,
+                                       int r1, int K, int C) {
+  (void)d;
+  const size_t sc = cer_score_workspace_size(B, N, core_hidden, exp_hidden, task);
+  if (sc == 0 && B > 0 && N > 0) return 0;
+  if (B < 0 || N < 0 || r0 < 0 || r1 < r0 || r1 > N || K < 0 || K > r1 - r0 || C < 0) return 0;
+  const size_t k_tot = static_cast<size_t>(K) + (N - (r1 - r0));
+  const size_t M = static_cast<size_t>(B) * k_tot;
+  return sc + round256(M * sizeof(int32_t)) + round256(M * C * 2);
+}
+
+cer_status cer_routed_block(void* h, void* out, int B, int N, int d, const cer_scorer* core, const cer_scorer* exp,
+                            const float* t, int task, int r0, int r1, int K, const void* Wg, const void* Wu,
+                            const void* WdT, int I, const int32_t* chan, int C, float* logits, int32_t* idx,
+                            uint8_t* mask, void* workspace, size_t workspace_bytes, cudaEvent_t* stage_events,
+                            int n_stage_events, cudaStream_t stream) {
+  ScoreShape sh;
+  cer_status s = check_score_args(h, B, N, d, core, exp, t, task, &sh);
+  if (s != CER_OK) return s;
+  CER_PTR(Wg);
+  CER_PTR(Wu);
+  CER_PTR(WdT);
+  CER_ALIGN(out);
+  CER_ALIGN(Wg);
+  CER_ALIGN(Wu);
+  CER_ALIGN(WdT);
+  CER_ALIGN(chan);
+  CER_ALIGN(logits);
+  CER_ALIGN(idx);
+  CER_ALIGN(mask);
+  CER_ALIGN(workspace);
+  CER_REQUIRE(N <= cer::kTopkMaxN, CER_ERR_SHAPE, "N=%d exceeds %d", N, cer::kTopkMaxN);
+  CER_REQUIRE(0 <= r0 && r0 <= r1 && r1 <= N, CER_ERR_RANGE, "routable range [%d, %d) not inside [0, %d]", r0, r1, N);
+  CER_REQUIRE(0 <= K && K <= r1 - r0, CER_ERR_RANGE, "K=%d not in [0, N_r=%d]", K, r1 - r0);
+  const int k_tot = K + N - (r1 - r0);
+  const long long M64 = static_cast<long long>(B) * k_tot;
+  s = check_ffn_shape(static_cast<int>(M64), d, I, chan, C);
+  if (s != CER_OK) return s;
+  CER_REQUIRE(stage_events == nullptr || n_stage_events == 5, CER_ERR_RANGE,
+              "stage_events needs exactly 5 events (got %d)", n_stage_events);
+  const size_t need = cer_routed_block_workspace_size(B, N, d, sh.Hc, sh.He, task, r0, r1, K, C);
+  CER_REQUIRE(workspace != nullptr && workspace_bytes >= need, CER_ERR_WORKSPACE,
+              "workspace of %zu bytes needed, %zu given", need, workspace_bytes);
+  const bool in_place = (out == nullptr || out == h);
+  const size_t hbytes = static_cast<size_t>(B) * N * d * 2;
+  if (!in_place) {
+    const char* a0 = static_cast<const char*>(h);
+    const char* b0 = static_cast<const char*>(out);
+    CER_REQUIRE(b0 + hbytes <= a0 || a0 + hbytes <= b0, CER_ERR_RANGE, "out overlaps h without being equal to it");
+  }
+  DeviceInfo* dev = nullptr;
+  if ((s = device_info(&dev)) != CER_OK) return s;
+
+  auto mark = [&](int i) -> cudaError_t {
+    return stage_events ? cudaEventRecord(stage_events[i], stream) : cudaSuccess;
+  };
+  cudaError_t e = mark(0);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+  void* dst = in_place ? h : out;
+  if (!in_place && hbytes) {
+    e = cudaMemcpyAsync(out, h, hbytes, cudaMemcpyDeviceToDevice, stream);  // bypass rows
+    if (e != cudaSuccess) return cuda_fail(e, "bypass copy");
+  }
+  if (B == 0 || N == 0) {
+    for (int i = 1; i < 5; ++i) mark(i);
+    return CER_OK;
+  }
+  char* ws = static_cast<char*>(workspace);
+  cer::ScoreWorkspace sws = carve_score_ws(ws, B, N, sh);
+  ws += score_ws_bytes(B, N, sh);
+  int32_t* idx_buf = idx ? idx : reinterpret_cast<int32_t*>(ws);
+  ws += round256(static_cast<size_t>(M64) * sizeof(int32_t));
+  __nv_bfloat16* act = reinterpret_cast<__nv_bfloat16*>(ws);
+
+  // S1: scorer GEMM -> partial sums
+  cer::ScoreArgs sa = make_score_args(h, B, N, d, core, exp, t, sh, dev->status);
+  e = cer::launch_score(sa, sws, dev->n_sm, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "scorer launch");
+  if ((e = mark(1)) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+
+  // S2: reduce partial sums + top-K keep list
+  cer::TopkArgs ta{};
+  ta.src = sws.partial;
+  ta.n_chunks = sh.n_chunks;
+  ta.chunk_stride = static_cast<size_t>(B) * N;
+  ta.B = B;
+  ta.N = N;
+  ta.r0 = r0;
+  ta.r1 = r1;
+  ta.K = K;
+  ta.logits_out = logits;
+  ta.idx = idx_buf;
+  ta.mask = mask;
+  ta.status = dev->status;
+  e = cer::launch_topk(ta, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "top-K launch");
+  if ((e = mark(2)) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+
+  // S3+S4: gate/up GEMM on the kept rows of h (row gathers)
+  cer::FfnArgs fa{};
+  fa.h = static_cast<const __nv_bfloat16*>(h);
+  fa.idx = idx_buf;
+  fa.N = N;
+  fa.k_tot = k_tot;
+  fa.M = static_cast<int>(M64);
+  fa.d = d;
+  fa.I = I;
+  fa.C = C;
+  fa.Wg = static_cast<const __nv_bfloat16*>(Wg);
+  fa.Wu = static_cast<const __nv_bfloat16*>(Wu);
+  fa.WdT = static_cast<const __nv_bfloat16*>(WdT);
+  fa.chan = chan;
+  fa.act = act;
+  fa.out = static_cast<__nv_bfloat16*>(dst);
+  fa.scatter = 1;
+  fa.status = dev->status;
+  if (M64 > 0) {
+    e = cer::launch_ffn_gateup(fa, dev->n_sm, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "gate/up GEMM launch");
+  }
+  if ((e = mark(3)) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+
+  // S4+S5: down GEMM with the unpack fused into its epilogue
+  if (M64 > 0) {
+    e = cer::launch_ffn_down(fa, dev->n_sm, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "down GEMM launch");
+  }
+  if ((e = mark(4)) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+  return CER_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,94 @@
+// kernels.h -- internal launch interface between the C ABI (cer_api.cu) and
+// the kernel translation units.  Not part of the public ABI.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <cstddef>
+#include <cstdint>
+
+namespace cer {
+
+// Encode a 2-D bf16 tensor map (rows x cols, row pitch cols*2 bytes) with a
+// box of box_cols x box_rows elements, 128-byte swizzle, zero fill.
+bool encode_bf16_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_cols,
+                    uint32_t box_rows);
+
+// Raise a kernel's dynamic shared-memory limit once per device.
+cudaError_t ensure_max_smem(const void* func, size_t bytes);
+
+// ------------------------------------------------------------------ S1 score
+struct ScoreArgs {
+  const __nv_bfloat16* h;
+  int B, N, d;
+  const __nv_bfloat16* W1;
+  const float* b1;
+  const float* w2;
+  int Hc;
+  const __nv_bfloat16* W1e;
+  const float* b1e;
+  const float* w2e;
+  const __nv_bfloat16* U;
+  int He, E, S;
+  const float* t;
+  int gen;
+  int* status;
+};
+
+struct ScoreWorkspace {
+  float* bias_tab;  // [B][Hc + He]
+  float* w2_tab;    // [B][Hc + He]
+  float* partial;   // [n_chunks][B*N]
+};
+
+int score_chunk_width(int Hc, int He, int gen);
+cudaError_t launch_score(const ScoreArgs& a, const ScoreWorkspace& ws, int n_sm, cudaStream_t stream);
+cudaError_t launch_score_reduce(const float* partial, int n_chunks, size_t total, float* logits, float* probs,
+                                int n_sm, cudaStream_t stream);
+
+// ------------------------------------------------------------------ S2 select
+struct TopkArgs {
+  const float* src;      // logits [B*N] (n_chunks == 1) or scorer partial sums [n_chunks][B*N]
+  int n_chunks;
+  size_t chunk_stride;
+  int B, N, r0, r1, K;
+  float* logits_out;     // nullable
+  float* probs_out;      // nullable
+  int32_t* idx;          // [B][k_tot]
+  uint8_t* mask;         // nullable
+  int* status;
+};
+constexpr int kTopkMaxN = 49152;
+cudaError_t launch_topk(const TopkArgs& a, cudaStream_t stream);
+
+// ------------------------------------------------------------------ S3 / S5 rows
+cudaError_t launch_gather(const __nv_bfloat16* h, int B, int N, int d, const int32_t* idx, int k_tot,
+                          __nv_bfloat16* X, int* status, int n_sm, cudaStream_t stream);
+cudaError_t launch_scatter_add(__nv_bfloat16* h, int B, int N, int d, const int32_t* idx, int k_tot,
+                               const __nv_bfloat16* Y, int* status, int n_sm, cudaStream_t stream);
+
+// ------------------------------------------------------------------ S4 FFN
+struct FfnArgs {
+  // A operand of the gate/up GEMM: either packed rows X [M, d] (idx == nullptr)
+  // or the kept rows of h [B, N, d] selected by idx [B][k_tot].
+  const __nv_bfloat16* X;
+  const __nv_bfloat16* h;
+  const int32_t* idx;
+  int N, k_tot;
+  int M, d, I, C;
+  const __nv_bfloat16* Wg;
+  const __nv_bfloat16* Wu;
+  const __nv_bfloat16* WdT;
+  const int32_t* chan;   // nullable: all channels
+  __nv_bfloat16* act;    // workspace [M, C]
+  // Output: Y [M, d] (scatter == 0) or out[b, idx] = bf16(h + y) (scatter == 1).
+  __nv_bfloat16* Y;
+  __nv_bfloat16* out;
+  int scatter;
+  int* status;
+};
+cudaError_t launch_ffn_gateup(const FfnArgs& a, int n_sm, cudaStream_t stream);
+cudaError_t launch_ffn_down(const FfnArgs& a, int n_sm, cudaStream_t stream);
+
+}  // namespace cer

@@ -1,0 +1,105 @@
+// rows_kernel.cu -- S3 gather (token compaction) and S5 scatter-add (unpack
+// with bypass), Sec. 3.4.  Pure HBM streams: one warp per packed row, 16-byte
+// vector loads and stores, four vectors in flight per lane; a persistent grid
+// of 16 warps per SM.  Dropped rows are never touched.
+#include <cuda_bf16.h>
+
+#include "kernels.h"
+#include "status.cuh"
+
+namespace cer {
+
+constexpr int kRowThreads = 512;
+
+__global__ void __launch_bounds__(kRowThreads) gather_rows_kernel(const uint4* __restrict__ h, int N, int d16,
+                                                                  const int32_t* __restrict__ idx, int k_tot,
+                                                                  int M, uint4* __restrict__ X, int* status) {
+  const int lane = threadIdx.x & 31;
+  const int wpb = blockDim.x >> 5;
+  for (int m = blockIdx.x * wpb + (threadIdx.x >> 5); m < M; m += gridDim.x * wpb) {
+    const int b = m / k_tot;
+    const int i = __ldg(idx + m);
+    if (i < 0 || i >= N) {
+      if (lane == 0) record_status(status, CER_DEV_INDEX);
+      continue;
+    }
+    const uint4* src = h + (static_cast<size_t>(b) * N + i) * d16;
+    uint4* dst = X + static_cast<size_t>(m) * d16;
+    int c = lane;
+    for (; c + 96 < d16; c += 128) {
+      const uint4 v0 = __ldg(src + c), v1 = __ldg(src + c + 32), v2 = __ldg(src + c + 64), v3 = __ldg(src + c + 96);
+      dst[c] = v0;
+      dst[c + 32] = v1;
+      dst[c + 64] = v2;
+      dst[c + 96] = v3;
+    }
+    for (; c < d16; c += 32) dst[c] = __ldg(src + c);
+  }
+}
+
+__device__ __forceinline__ uint32_t add_bf16x2(uint32_t hv, uint32_t yv) {
+  __nv_bfloat162 a = *reinterpret_cast<__nv_bfloat162*>(&hv);
+  __nv_bfloat162 b = *reinterpret_cast<__nv_bfloat162*>(&yv);
+  const float2 fa = __bfloat1622float2(a), fb = __bfloat1622float2(b);
+  __nv_bfloat162 r = __floats2bfloat162_rn(fa.x + fb.x, fa.y + fb.y);
+  return *reinterpret_cast<uint32_t*>(&r);
+}
+
+__device__ __forceinline__ uint4 add_row_vec(uint4 hv, uint4 yv) {
+  return make_uint4(add_bf16x2(hv.x, yv.x), add_bf16x2(hv.y, yv.y), add_bf16x2(hv.z, yv.z), add_bf16x2(hv.w, yv.w));
+}
+
+__global__ void __launch_bounds__(kRowThreads) scatter_add_kernel(uint4* __restrict__ h, int N, int d16,
+                                                                  const int32_t* __restrict__ idx, int k_tot,
+                                                                  int M, const uint4* __restrict__ Y,
+                                                                  int* status) {
+  const int lane = threadIdx.x & 31;
+  const int wpb = blockDim.x >> 5;
+  for (int m = blockIdx.x * wpb + (threadIdx.x >> 5); m < M; m += gridDim.x * wpb) {
+    const int b = m / k_tot;
+    const int i = __ldg(idx + m);
+    if (i < 0 || i >= N) {
+      if (lane == 0) record_status(status, CER_DEV_INDEX);
+      continue;
+    }
+    uint4* row = h + (static_cast<size_t>(b) * N + i) * d16;
+    const uint4* y = Y + static_cast<size_t>(m) * d16;
+    int c = lane;
+    for (; c + 32 < d16; c += 64) {
+      const uint4 h0 = row[c], h1 = row[c + 32];
+      const uint4 y0 = __ldg(y + c), y1 = __ldg(y + c + 32);
+      row[c] = add_row_vec(h0, y0);
+      row[c + 32] = add_row_vec(h1, y1);
+    }
+    for (; c < d16; c += 32) row[c] = add_row_vec(row[c], __ldg(y + c));
+  }
+}
+
+static int row_grid(int M, int n_sm) {
+  const int wpb = kRowThreads / 32;
+  int blocks = (M + wpb - 1) / wpb;
+  const int cap = n_sm * 4;  // 4 blocks x 16 warps per SM
+  return blocks < cap ? blocks : cap;
+}
+
+cudaError_t launch_gather(const __nv_bfloat16* h, int B, int N, int d, const int32_t* idx, int k_tot,
+                          __nv_bfloat16* X, int* status, int n_sm, cudaStream_t stream) {
+  const int M = B * k_tot;
+  if (M == 0 || d == 0) return cudaSuccess;
+  gather_rows_kernel<<<row_grid(M, n_sm), kRowThreads, 0, stream>>>(reinterpret_cast<const uint4*>(h), N, d / 8,
+                                                                    idx, k_tot, M, reinterpret_cast<uint4*>(X),
+                                                                    status);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_scatter_add(__nv_bfloat16* h, int B, int N, int d, const int32_t* idx, int k_tot,
+                               const __nv_bfloat16* Y, int* status, int n_sm, cudaStream_t stream) {
+  const int M = B * k_tot;
+  if (M == 0 || d == 0) return cudaSuccess;
+  scatter_add_kernel<<<row_grid(M, n_sm), kRowThreads, 0, stream>>>(reinterpret_cast<uint4*>(h), N, d / 8, idx,
+                                                                    k_tot, M, reinterpret_cast<const uint4*>(Y),
+                                                                    status);
+  return cudaGetLastError();
+}
+
+}  // namespace cer

@@ -1,0 +1,196 @@
+// topk_kernel.cu -- S2: the per-sequence keep set R = TopK(sigmoid(l), K) of
+// Eq. 4 (Sec. 3.4), computed exactly on the fp32 logits (the sigmoid is
+// monotonic, App. B.2).
+//
+// One 1024-thread CTA per sequence keeps the N order-preserving 32-bit keys in
+// shared memory.  A four-pass MSB-first radix select (8-bit digits, shared
+// histograms) finds the K-th largest routable key T and how many tokens equal
+// to T must be taken; two block-wide scans in token order then give every
+// tie its rank (lowest index first) and every kept token its output slot, so
+// the kept list comes out in ascending token order with no sort.  When fed
+// the scorer's partial sums it also reduces them (in chunk order) into the
+// logits.
+#include <cuda_runtime.h>
+
+#include "kernels.h"
+#include "status.cuh"
+
+namespace cer {
+
+constexpr int kTopkThreads = 1024;
+
+// Monotone map from fp32 to uint32: a > b (as floats) iff key(a) > key(b);
+// -0.0 is mapped like +0.0.
+__device__ __forceinline__ uint32_t order_key(float v) {
+  uint32_t u = __float_as_uint(v);
+  if (u == 0x80000000u) u = 0u;
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+// Exclusive prefix sum over the block (all threads must call).
+__device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t* warp_tot) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  uint32_t incl = v;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const uint32_t o = __shfl_up_sync(0xffffffffu, incl, off);
+    if (lane >= off) incl += o;
+  }
+  if (lane == 31) warp_tot[warp] = incl;
+  __syncthreads();
+  if (warp == 0) {
+    const int nw = blockDim.x >> 5;
+    uint32_t t = lane < nw ? warp_tot[lane] : 0u;
+    uint32_t ti = t;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const uint32_t o = __shfl_up_sync(0xffffffffu, ti, off);
+      if (lane >= off) ti += o;
+    }
+    if (lane < nw) warp_tot[lane] = ti - t;  // exclusive over warps
+  }
+  __syncthreads();
+  const uint32_t r = warp_tot[warp] + incl - v;
+  __syncthreads();
+  return r;
+}
+
+__global__ void __launch_bounds__(kTopkThreads) topk_kernel(TopkArgs a) {
+  extern __shared__ uint32_t keys[];
+  __shared__ uint32_t hist[256];
+  __shared__ uint32_t warp_tot[32];
+  __shared__ uint32_t s_prefix, s_remaining;
+  __shared__ int s_nan;
+
+  const int tid = threadIdx.x;
+  const int b = blockIdx.x;
+  const int N = a.N;
+  const size_t base = static_cast<size_t>(b) * N;
+  if (tid == 0) s_nan = 0;
+  __syncthreads();
+
+  // 1. logits (reduced from partial sums in chunk order) -> keys
+  for (int i = tid; i < N; i += blockDim.x) {
+    float v = a.src[base + i];
+    for (int c = 1; c < a.n_chunks; ++c) v += a.src[static_cast<size_t>(c) * a.chunk_stride + base + i];
+    if (a.logits_out) a.logits_out[base + i] = v;
+    if (a.probs_out) a.probs_out[base + i] = 1.0f / (1.0f + expf(-v));
+    if (i >= a.r0 && i < a.r1 && v != v) s_nan = 1;
+    keys[i] = order_key(v);
+  }
+  __syncthreads();
+
+  const int Nr = a.r1 - a.r0;
+  const int K = a.K;
+  const bool keep_all = (K == Nr);
+  const bool keep_none = (K == 0);
+  uint32_t thr = 0, need_eq = 0;
+
+  // 2. radix select of the K-th largest routable key
+  if (!keep_all && !keep_none) {
+    uint32_t prefix = 0, pmask = 0, remaining = static_cast<uint32_t>(K);
+    for (int shift = 24; shift >= 0; shift -= 8) {
+      for (int i = tid; i < 256; i += blockDim.x) hist[i] = 0;
+      __syncthreads();
+      for (int i = a.r0 + tid; i < a.r1; i += blockDim.x) {
+        const uint32_t k = keys[i];
+        if ((k & pmask) == prefix) atomicAdd(&hist[(k >> shift) & 255u], 1u);
+      }
+      __syncthreads();
+      if (tid < 32) {
+        const int lane = tid;
+        uint32_t local[8];
+        uint32_t tot = 0;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          local[j] = hist[8 * lane + j];
+          tot += local[j];
+        }
+        uint32_t incl = tot;  // sum over lanes >= lane
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+          const uint32_t o = __shfl_down_sync(0xffffffffu, incl, off);
+          if (lane + off < 32) incl += o;
+        }
+        uint32_t cum = incl - tot;  // keys in higher digits than this lane's bins
+#pragma unroll
+        for (int j = 7; j >= 0; --j) {
+          if (cum < remaining && cum + local[j] >= remaining) {
+            s_prefix = prefix | (static_cast<uint32_t>(8 * lane + j) << shift);
+            s_remaining = remaining - cum;
+          }
+          cum += local[j];
+        }
+      }
+      __syncthreads();
+      prefix = s_prefix;
+      remaining = s_remaining;
+      pmask |= 255u << shift;
+      __syncthreads();
+    }
+    thr = prefix;
+    need_eq = remaining;
+  }
+
+  // 3. keep decisions in token order; ties to T ranked by index
+  const int seg = (N + blockDim.x - 1) / blockDim.x;
+  const int s0 = min(tid * seg, N);
+  const int s1 = min(s0 + seg, N);
+  uint32_t eq_cnt = 0;
+  if (!keep_all && !keep_none) {
+    for (int i = s0; i < s1; ++i)
+      if (i >= a.r0 && i < a.r1 && keys[i] == thr) ++eq_cnt;
+  }
+  const uint32_t eq_before = block_exclusive_scan(eq_cnt, warp_tot);
+
+  uint32_t keep_cnt = 0;
+  {
+    uint32_t er = eq_before;
+    for (int i = s0; i < s1; ++i) {
+      bool keep;
+      if (i < a.r0 || i >= a.r1 || keep_all) {
+        keep = true;
+      } else if (keep_none) {
+        keep = false;
+      } else {
+        const uint32_t k = keys[i];
+        if (k > thr) keep = true;
+        else if (k == thr) keep = (er++ < need_eq);
+        else keep = false;
+      }
+      keep_cnt += keep ? 1u : 0u;
+    }
+  }
+  const uint32_t pos0 = block_exclusive_scan(keep_cnt, warp_tot);
+
+  const int k_tot = K + N - Nr;
+  int32_t* idx = a.idx + static_cast<size_t>(b) * k_tot;
+  uint32_t er = eq_before, pos = pos0;
+  for (int i = s0; i < s1; ++i) {
+    bool keep;
+    if (i < a.r0 || i >= a.r1 || keep_all) {
+      keep = true;
+    } else if (keep_none) {
+      keep = false;
+    } else {
+      const uint32_t k = keys[i];
+      if (k > thr) keep = true;
+      else if (k == thr) keep = (er++ < need_eq);
+      else keep = false;
+    }
+    if (keep && pos < static_cast<uint32_t>(k_tot)) idx[pos++] = i;
+    if (a.mask) a.mask[base + i] = keep ? 1 : 0;
+  }
+  if (tid == 0 && s_nan) record_status(a.status, CER_DEV_NAN);
+}
+
+cudaError_t launch_topk(const TopkArgs& a, cudaStream_t stream) {
+  if (a.B == 0 || a.N == 0) return cudaSuccess;
+  const size_t smem = static_cast<size_t>(a.N) * sizeof(uint32_t);
+  cudaError_t e = ensure_max_smem(reinterpret_cast<const void*>(topk_kernel), smem);
+  if (e != cudaSuccess) return e;
+  topk_kernel<<<a.B, kTopkThreads, smem, stream>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace cer

@@ -1,0 +1,217 @@
+// umma_gemm.cuh -- persistent, warp-specialised tcgen05 GEMM skeleton for
+// sm_103a, shared by the scorer and the two FFN contractions.
+//
+// One CTA per SM (192 threads, ~193 KB shared memory, 2*BN TMEM columns):
+//   warp 0     producer: TMA loads (tiled or 4-row gathers) of the A tile
+//              (128 rows x 64 bf16) and the B tile (BN rows x 64 bf16, or
+//              64 K-rows x BN for an MN-major B) into a STAGES-deep ring;
+//   warp 1     allocates TMEM, one elected lane issues tcgen05.mma
+//              (M=128, N=BN, K=16) four times per 64-wide K block and
+//              commits the ring slot back to the producer;
+//   warps 2-5  epilogue: read the fp32 accumulator out of TMEM (lane = tile
+//              row) and apply the problem's fused epilogue.
+// The accumulator is double-buffered in TMEM so the epilogue of tile i
+// overlaps the MMAs of tile i+1.  Tiles are visited with a stride of
+// gridDim.x.  Every wait is bounded (ptx.cuh); on a timeout the CTA unwinds,
+// waits briefly for its own copies and MMAs, frees TMEM and exits.
+//
+// A problem class P supplies:
+//   BN, STAGES, B_MN_MAJOR, kBStepBytes, Params (with `int* status`),
+//   num_tiles(p), num_kb(p), prod_tile(p, tile, lane, state),
+//   prod_kb(p, state, tile, kb, lane, a_smem, b_smem, bar),
+//   stage_bytes(p, tile, kb), bdesc(saddr), epilogue(p, tile, row, taddr).
+#pragma once
+
+#include "ptx.cuh"
+
+namespace cer {
+
+constexpr int kGemmThreads = 192;
+constexpr uint32_t kATileBytes = 128 * 128;  // 128 rows x 64 bf16
+
+template <int BN>
+struct TmemCols {
+  static constexpr uint32_t need = 2 * BN;
+  static constexpr uint32_t value = need <= 32 ? 32 : need <= 64 ? 64 : need <= 128 ? 128 : need <= 256 ? 256 : 512;
+};
+
+template <class P>
+constexpr size_t gemm_smem_bytes() {
+  return 1024 + static_cast<size_t>(P::STAGES) * (kATileBytes + P::BN * 128) + 256;
+}
+
+// A short, abort-independent wait used only while unwinding.
+__device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
+  const uint64_t t0 = globaltimer_ns();
+  while (!mbar_try_wait(bar, parity)) {
+    if (globaltimer_ns() - t0 > 100000000ull) return;
+  }
+}
+
+// Lane 0 waits, the whole warp takes its verdict: keeps every branch after a
+// wait warp-uniform, which the .sync.aligned tcgen05 instructions require.
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int* status) {
+  int ok = 1;
+  if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, abort_flag, status) ? 1 : 0;
+  ok = __shfl_sync(0xffffffffu, ok, 0);
+  __syncwarp();
+  return ok != 0;
+}
+
+template <class P>
+__global__ void __launch_bounds__(kGemmThreads, 1) umma_gemm_kernel(const __grid_constant__ typename P::Params p) {
+  constexpr int BN = P::BN;
+  constexpr int STAGES = P::STAGES;
+  constexpr uint32_t B_BYTES = BN * 128;
+  constexpr uint32_t TMEM_COLS = TmemCols<BN>::value;
+  constexpr uint32_t IDESC = idesc_bf16(128, BN, P::B_MN_MAJOR);
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* a_ring = smem;
+  uint8_t* b_ring = smem + STAGES * kATileBytes;
+  uint64_t* full = reinterpret_cast<uint64_t*>(b_ring + STAGES * B_BYTES);
+  uint64_t* empty = full + STAGES;
+  uint64_t* tfull = empty + STAGES;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* drain = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&tfull[a], 1);
+      mbar_init(&tempty[a], 128);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int ntiles = P::num_tiles(p);
+  const int nkb = P::num_kb(p);
+
+  if (warp == 0) {
+    // ---------------------------------------------------------------- producer
+    typename P::ProdState st;
+    int stage = 0;
+    uint32_t phase = 0;
+    long issued = 0;
+    bool ok = true;
+    for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
+      P::prod_tile(p, tile, lane, st);
+      for (int kb = 0; kb < nkb; ++kb) {
+        if (!warp_wait(&empty[stage], phase ^ 1, abort_flag, p.status)) {
+          ok = false;
+          break;
+        }
+        const uint32_t bytes = P::stage_bytes(p, tile, kb);
+        if (lane == 0) mbar_arrive_expect_tx(&full[stage], bytes);
+        __syncwarp();
+        P::prod_kb(p, st, tile, kb, lane, a_ring + stage * kATileBytes, b_ring + stage * B_BYTES, &full[stage]);
+        ++issued;
+        if (++stage == STAGES) {
+          stage = 0;
+          phase ^= 1;
+        }
+      }
+    }
+    if (!ok && lane == 0) {
+      // Let the copies already issued land before the CTA's memory goes away.
+      for (long n = issued - 1; n >= 0 && n >= issued - STAGES; --n)
+        drain_wait(&full[n % STAGES], static_cast<uint32_t>((n / STAGES) & 1));
+    }
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA issuer
+    int stage = 0;
+    uint32_t phase = 0;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    bool ok = true;
+    bool issued_any = false;
+    for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
+      if (!warp_wait(&tempty[acc], acc_phase ^ 1, abort_flag, p.status)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
+      for (int kb = 0; kb < nkb; ++kb) {
+        if (!warp_wait(&full[stage], phase, abort_flag, p.status)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        if (lane == 0) {
+          const uint32_t a_base = smem_u32(a_ring + stage * kATileBytes);
+          const uint32_t b_base = smem_u32(b_ring + stage * B_BYTES);
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            umma_bf16(d_tmem, sdesc_kmajor_sw128(a_base + k * 32), P::bdesc(b_base + k * P::kBStepBytes), IDESC,
+                      (kb | k) != 0 ? 1u : 0u);
+          }
+          umma_commit(&empty[stage]);
+          issued_any = true;
+        }
+        __syncwarp();
+        if (++stage == STAGES) {
+          stage = 0;
+          phase ^= 1;
+        }
+      }
+      if (!ok) break;
+      if (lane == 0) umma_commit(&tfull[acc]);
+      __syncwarp();
+      if (++acc == 2) {
+        acc = 0;
+        acc_phase ^= 1;
+      }
+    }
+    if (!ok && lane == 0 && issued_any) {
+      umma_commit(drain);
+      drain_wait(drain, 0);
+    }
+  } else {
+    // ---------------------------------------------------------------- epilogue
+    const int q = warp & 3;            // TMEM lane quadrant this warp may access
+    const int row = q * 32 + lane;     // accumulator row = TMEM lane
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+      if (!warp_wait(&tfull[acc], acc_phase, abort_flag, p.status)) break;
+      tc_fence_after();
+      const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BN);
+      P::epilogue(p, tile, row, taddr);
+      tc_fence_before();
+      mbar_arrive(&tempty[acc]);
+      if (++acc == 2) {
+        acc = 0;
+        acc_phase ^= 1;
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, TMEM_COLS);
+  }
+}
+
+}  // namespace cer

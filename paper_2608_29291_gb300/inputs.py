@@ -29,13 +29,16 @@ _CHUNK = 1 << 22
 
 
 def _mix64(z: np.ndarray) -> np.ndarray:
-    """SplitMix64 output function on a uint64 array (wrapping arithmetic)."""
-    z = z.copy()
-    z ^= z >> np.uint64(30)
+    """SplitMix64 output function on a uint64 array (wrapping arithmetic), in place."""
+    t = np.empty_like(z)
+    np.right_shift(z, np.uint64(30), out=t)
+    z ^= t
     z *= _M1
-    z ^= z >> np.uint64(27)
+    np.right_shift(z, np.uint64(27), out=t)
+    z ^= t
     z *= _M2
-    z ^= z >> np.uint64(31)
+    np.right_shift(z, np.uint64(31), out=t)
+    z ^= t
     return z
 
 
@@ -57,8 +60,10 @@ def substream_seed(seed: int, name: str) -> int:
 def raw_u64(seed: int, start: int, count: int) -> np.ndarray:
     """Counter-based SplitMix64 words for counters start .. start+count-1."""
     with np.errstate(over="ignore"):
-        ctr = np.arange(start + 1, start + count + 1, dtype=np.uint64)
-        return _mix64(np.uint64(seed) + ctr * _GAMMA)
+        z = np.arange(start + 1, start + count + 1, dtype=np.uint64)
+        z *= _GAMMA
+        z += np.uint64(seed)
+        return _mix64(z)
 
 
 def uniform01(seed: int, count: int, start: int = 0) -> np.ndarray:
@@ -89,14 +94,20 @@ def f32_to_bf16_bits(x: np.ndarray) -> np.ndarray:
 
 
 def bf16_normal(seed: int, name: str, shape, std: float) -> np.ndarray:
-    """bf16 bit patterns of N(0, std^2) draws, uint16 array of the given shape."""
+    """bf16 bit patterns of N(0, std^2) draws, uint16 array of the given shape.
+
+    One SplitMix64 word per element: its top 24 bits and its low 24 bits give
+    the two Box-Muller uniforms ((k + 0.5) * 2^-24), enough for a bf16 result.
+    """
     count = int(np.prod(shape))
     out = np.empty(count, dtype=np.uint16)
     ss = substream_seed(seed, name)
     for s in range(0, count, _CHUNK):
         n = min(_CHUNK, count - s)
-        u = uniform01(ss, 2 * n, start=2 * s)
-        z = np.sqrt(-2.0 * np.log(u[0::2])) * np.cos(2.0 * math.pi * u[1::2])
+        w = raw_u64(ss, s, n)
+        u1 = ((w >> np.uint64(40)).astype(np.float64) + 0.5) * (2.0 ** -24)
+        u2 = ((w & np.uint64(0xFFFFFF)).astype(np.float64) + 0.5) * (2.0 ** -24)
+        z = np.sqrt(-2.0 * np.log(u1)) * np.cos(2.0 * math.pi * u2)
         out[s:s + n] = f32_to_bf16_bits((z * std).astype(np.float32))
     return out.reshape(shape)
 
@@ -200,12 +211,13 @@ def sweep(n: int, token_ratio: float, ffn_ratio: float) -> Workload:
 WORKLOADS = {"tiny": tiny, "und_1p5b": und_1p5b, "gen_1p5b": gen_1p5b, "long_7b": long_7b}
 
 
-def make_inputs(w: Workload) -> dict:
+def make_inputs(w: Workload, ffn_weights: Optional[tuple] = None) -> dict:
     """All tensors of one workload as host numpy arrays (bf16 as uint16 bits).
 
     Recipe: h ~ N(0,1) (routable rows times lognormal(0, 0.5) per row when
     ``visual_lognormal``); every weight ~ N(0, 1/fan_in); scorer output vectors
     w2 fp32; t_b fixed or ~ U[0,1); channel keep set by Fisher-Yates.
+    ``ffn_weights`` may pass (Wg, Wu, WdT) drawn earlier for the same (seed, I, d).
     """
     s = w.seed
     h_shape = (w.B, w.N, w.d)
@@ -222,9 +234,9 @@ def make_inputs(w: Workload) -> dict:
         "W1": bf16_normal(s, "W1", (w.Hc, w.d), 1.0 / math.sqrt(w.d)),
         "w2": f32_normal(s, "w2", (w.Hc,), 1.0 / math.sqrt(w.Hc)),
         "b1": f32_normal(s, "b1", (w.Hc,), 0.1) if w.core_bias else None,
-        "Wg": bf16_normal(s, "Wg", (w.I, w.d), 1.0 / math.sqrt(w.d)),
-        "Wu": bf16_normal(s, "Wu", (w.I, w.d), 1.0 / math.sqrt(w.d)),
-        "WdT": bf16_normal(s, "WdT", (w.I, w.d), 1.0 / math.sqrt(w.I)),
+        "Wg": ffn_weights[0] if ffn_weights else bf16_normal(s, "Wg", (w.I, w.d), 1.0 / math.sqrt(w.d)),
+        "Wu": ffn_weights[1] if ffn_weights else bf16_normal(s, "Wu", (w.I, w.d), 1.0 / math.sqrt(w.d)),
+        "WdT": ffn_weights[2] if ffn_weights else bf16_normal(s, "WdT", (w.I, w.d), 1.0 / math.sqrt(w.I)),
         "chan": channel_keep_set(s, "chan", w.I, w.C),
     }
     if w.t_fixed is not None:

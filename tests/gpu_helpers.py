@@ -1,0 +1,45 @@
+"""Move seeded host inputs onto the GPU as torch tensors, and back."""
+import numpy as np
+import torch
+
+from paper_2608_29291_gb300 import cer
+
+
+def bf16_dev(bits: np.ndarray, dev="cuda") -> torch.Tensor:
+    return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).to(dev)
+
+
+def bits_host(t: torch.Tensor) -> np.ndarray:
+    return t.detach().contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+
+
+def f32_dev(a, dev="cuda"):
+    return None if a is None else torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(dev)
+
+
+def i32_dev(a, dev="cuda"):
+    return None if a is None else torch.from_numpy(np.ascontiguousarray(a, dtype=np.int32)).to(dev)
+
+
+def scorers(inp: dict, dev="cuda"):
+    core = cer.Scorer(W1=bf16_dev(inp["W1"], dev), w2=f32_dev(inp["w2"], dev), b1=f32_dev(inp.get("b1"), dev))
+    exp = None
+    if inp.get("W1e") is not None:
+        exp = cer.Scorer(W1=bf16_dev(inp["W1e"], dev), w2=f32_dev(inp["w2e"], dev), b1=f32_dev(inp.get("b1e"), dev),
+                         U=bf16_dev(inp["Ue"], dev) if inp.get("Ue") is not None else None)
+    return core, exp
+
+
+def rel_err(got: np.ndarray, want: np.ndarray, floor_frac: float = 1e-2) -> float:
+    """max |got - want| / max(|want|, floor_frac * RMS(want)), elementwise."""
+    want = np.asarray(want, dtype=np.float64)
+    got = np.asarray(got, dtype=np.float64)
+    rms = float(np.sqrt(np.mean(want ** 2))) if want.size else 0.0
+    den = np.maximum(np.abs(want), floor_frac * rms)
+    den = np.where(den == 0, 1.0, den)
+    return float(np.max(np.abs(got - want) / den)) if want.size else 0.0
+
+
+def rms(x) -> float:
+    x = np.asarray(x, dtype=np.float64)
+    return float(np.sqrt(np.mean(x ** 2))) if x.size else 0.0

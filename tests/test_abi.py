@@ -1,0 +1,100 @@
+"""Host-side checks of the C ABI that need no GPU: the library builds and loads,
+exports every entry point include/cer_api.h declares, sizes workspaces, and
+rejects bad arguments before touching a device.  A well-formed call on a
+machine without an sm_103 GPU must fail loudly (CER_ERR_DEVICE), never fall
+back to anything."""
+import ctypes
+import os
+import re
+
+import pytest
+import torch
+
+from paper_2608_29291_gb300 import cer
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "cer_api.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if not os.path.exists(cer.LIB_PATH):
+        from paper_2608_29291_gb300 import build_lib
+        build_lib.build()
+    return cer.load()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"^\s*(?:cer_status|size_t|const char\*|int)\s+(cer_\w+)\s*\(", text, re.M)))
+
+
+def test_header_declares_the_expected_entry_points():
+    assert declared_functions() == sorted(cer.EXPORTS)
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+    assert lib.cer_version() == 1
+    for code, name in cer.STATUS_NAMES.items():
+        assert lib.cer_status_string(code).decode() == name
+
+
+def test_workspace_sizes(lib):
+    # scorer: bias + w2 tables [B][Ht] and partial sums [chunks][B*N], 256-byte rounded
+    assert lib.cer_score_workspace_size(4, 1024, 256, 0, 0) == 2 * 4096 + 1 * 4 * 1024 * 4
+    assert lib.cer_score_workspace_size(2, 4096, 512, 512, 1) == 2 * 8192 + 4 * 2 * 4096 * 4
+    assert lib.cer_score_workspace_size(1, 256, 64, 64, 1) == 2 * 512 + 2 * 256 * 4
+    assert lib.cer_score_workspace_size(1, 10, 100, 0, 0) == 0          # hidden not a multiple of 64
+    assert lib.cer_routed_ffn_workspace_size(2348, 6720) == (2348 * 6720 * 2 + 255) // 256 * 256
+    ws = lib.cer_routed_block_workspace_size(4, 1024, 1536, 256, 0, 0, 0, 729, 292, 6720)
+    M = 4 * (292 + 1024 - 729)
+    assert ws == lib.cer_score_workspace_size(4, 1024, 256, 0, 0) + (M * 4 + 255) // 256 * 256 + \
+        (M * 6720 * 2 + 255) // 256 * 256
+
+
+FAKE = ctypes.c_void_p(1 << 20)      # 16-byte aligned, never dereferenced: checks fail first
+
+
+def _err(lib):
+    return lib.cer_get_error().decode()
+
+
+def test_select_argument_checks(lib):
+    assert lib.cer_select_topk(None, 1, 8, 0, 8, 4, FAKE, None, None) == 1          # NULL logits
+    assert lib.cer_select_topk(FAKE, 1, 8, 0, 8, 9, FAKE, None, None) == 4          # K > N_r
+    assert "K=9" in _err(lib)
+    assert lib.cer_select_topk(FAKE, 1, 8, 5, 3, 0, FAKE, None, None) == 4          # r0 > r1
+    assert lib.cer_select_topk(FAKE, 1, 8, 0, 9, 1, FAKE, None, None) == 4          # r1 > N
+    assert lib.cer_select_topk(FAKE, 1, 60000, 0, 8, 1, FAKE, None, None) == 2      # N too large
+    assert lib.cer_select_topk(ctypes.c_void_p((1 << 20) + 4), 1, 8, 0, 8, 1, FAKE, None, None) == 3
+
+
+def test_ffn_argument_checks(lib):
+    f = lib.cer_routed_ffn
+    assert f(FAKE, 10, 100, FAKE, FAKE, FAKE, 512, None, 512, FAKE, FAKE, 1 << 20, None) == 2   # d % 64
+    assert f(FAKE, 10, 128, FAKE, FAKE, FAKE, 512, None, 256, FAKE, FAKE, 1 << 20, None) == 2   # NULL chan, C != I
+    assert f(FAKE, 10, 128, FAKE, FAKE, FAKE, 512, FAKE, 100, FAKE, FAKE, 1 << 20, None) == 2   # C % 64
+    assert f(FAKE, 10, 128, FAKE, FAKE, FAKE, 512, FAKE, 576, FAKE, FAKE, 1 << 20, None) == 2   # C > I
+    assert f(FAKE, 1000, 128, FAKE, FAKE, FAKE, 512, FAKE, 256, FAKE, FAKE, 16, None) == 9      # workspace
+    assert f(FAKE, 10, 128, None, FAKE, FAKE, 512, FAKE, 256, FAKE, FAKE, 1 << 20, None) == 1   # NULL Wg
+
+
+def test_score_argument_checks(lib):
+    core = cer.CerScorerC(FAKE.value, None, FAKE.value, None, 256, 0, 1)
+    bad_core = cer.CerScorerC(FAKE.value, None, FAKE.value, FAKE.value, 256, 64, 1)   # core with U
+    s = lib.cer_score
+    assert s(FAKE, 1, 16, 1536, ctypes.pointer(core), None, None, 1, FAKE, None, FAKE, 1 << 30, None) == 1  # GEN, no exp
+    assert s(FAKE, 1, 16, 1500, ctypes.pointer(core), None, None, 0, FAKE, None, FAKE, 1 << 30, None) == 2  # d % 64
+    assert s(FAKE, 1, 16, 1536, ctypes.pointer(bad_core), None, None, 0, FAKE, None, FAKE, 1 << 30, None) == 2
+    assert s(FAKE, 1, 16, 1536, ctypes.pointer(core), None, None, 7, FAKE, None, FAKE, 1 << 30, None) == 4  # task
+    assert s(FAKE, 1, 16, 1536, ctypes.pointer(core), None, None, 0, FAKE, None, FAKE, 8, None) == 9        # workspace
+
+
+@pytest.mark.skipif(torch.cuda.is_available(), reason="checks the behaviour without a GPU")
+def test_well_formed_call_without_gpu_fails_loudly(lib):
+    st = lib.cer_select_topk(FAKE, 1, 8, 0, 8, 4, FAKE, None, None)
+    assert st == 6, (st, _err(lib))   # CER_ERR_DEVICE: no device, no fallback
+    with pytest.raises(cer.CerError):
+        cer._check(st)

@@ -1,0 +1,336 @@
+"""GPU parity: every C-ABI entry point against the CPU oracle on the same seeded
+inputs.  Bars: keep lists and masks bit-exact given the same fp32 logits;
+gather and scatter bit-exact; logits within 1e-4 relative (floor 1e-2 RMS);
+FFN and block outputs within 2e-2 x RMS of the oracle's output."""
+import zlib
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import cer_oracle as ora
+from paper_2608_29291_gb300 import cer
+from paper_2608_29291_gb300 import inputs as gen
+from tests.gpu_helpers import bf16_dev, bits_host, f32_dev, i32_dev, rel_err, rms, scorers
+
+pytestmark = pytest.mark.gpu
+
+SCORE_TOL = 1e-4
+OUT_TOL = 2e-2
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _device():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    cer.load()
+    yield
+    cer.cer_sync_status()
+
+
+def test_device_is_sm103():
+    assert torch.cuda.get_device_capability() == (10, 3)
+
+
+# ------------------------------------------------------------------ S2 select
+
+def _logit_cases():
+    rng = np.random.default_rng(11)
+    cases = []
+    ties = np.array([0.0, -0.0, 1.5, -2.0, -np.inf], np.float32)
+    cases.append(("n1_k0", np.array([[0.3]], np.float32), 0, 1, 0))
+    cases.append(("n1_k1", np.array([[0.3]], np.float32), 0, 1, 1))
+    v = np.array([[0.0, -0.0, 0.0, -1.0, -np.inf, 3.0]], np.float32)
+    for r0, r1, K in [(0, 6, 0), (0, 6, 1), (0, 6, 3), (0, 6, 5), (0, 6, 6), (1, 5, 2), (2, 4, 1), (3, 3, 0)]:
+        cases.append((f"golden_{r0}_{r1}_{K}", v, r0, r1, K))
+    cases.append(("heavy_ties", ties[rng.integers(0, 5, (3, 1000))], 17, 990, 411))
+    cases.append(("all_equal", np.full((2, 1000), 0.25, np.float32), 0, 1000, 300))
+    n16 = rng.normal(0, 1, (1, 16384)).astype(np.float32)
+    for K in (0, 1, 1638, 8192, 16383, 16384):
+        cases.append((f"n16384_k{K}", n16, 0, 16384, K))
+    cases.append(("n49152_max", rng.normal(0, 2, (1, 49152)).astype(np.float32), 0, 49152, 12345))
+    cases.append(("gen_layout", rng.normal(0, 1, (8, 1088)).astype(np.float32), 64, 1088, 512))
+    cases.append(("und_layout", rng.normal(0, 1, (4, 1024)).astype(np.float32), 0, 729, 292))
+    q = np.round(rng.normal(0, 1, (4, 3000)) * 4).astype(np.float32) / 4      # quantised: many ties
+    cases.append(("quantised", q, 100, 2900, 1399))
+    return cases
+
+
+@pytest.mark.parametrize("case", _logit_cases(), ids=lambda c: c[0])
+def test_select_topk_bit_exact(case):
+    _, logits, r0, r1, K = case
+    B, N = logits.shape
+    k_tot = K + N - (r1 - r0)
+    lg = f32_dev(logits)
+    idx = torch.full((B, k_tot), -1, dtype=torch.int32, device="cuda")
+    mask = torch.full((B, N), 7, dtype=torch.uint8, device="cuda")
+    cer.cer_select_topk(lg, r0, r1, K, idx, mask)
+    cer.cer_sync_status()
+    want_idx, want_mask = ora.select_topk(logits, r0, r1, K)
+    assert np.array_equal(idx.cpu().numpy(), want_idx)
+    assert np.array_equal(mask.cpu().numpy(), want_mask)
+
+
+def test_select_nan_reports_status_then_clears():
+    lg = f32_dev(np.array([[0.1, np.nan, 0.3, 0.2]], np.float32))
+    idx = torch.empty((1, 2), dtype=torch.int32, device="cuda")
+    cer.cer_select_topk(lg, 0, 4, 2, idx)
+    with pytest.raises(cer.CerError) as e:
+        cer.cer_sync_status()
+    assert e.value.status == 5
+    cer.cer_sync_status()   # cleared
+    # a NaN outside the routable range is not an error
+    cer.cer_select_topk(lg, 2, 4, 1, torch.empty((1, 3), dtype=torch.int32, device="cuda"))
+    cer.cer_sync_status()
+
+
+# ------------------------------------------------------------------ S3 / S5 rows
+
+def _rows_case(B, N, d, K, seed):
+    rng = np.random.default_rng(seed)
+    h = gen.f32_to_bf16_bits(rng.normal(0, 1, (B, N, d)).astype(np.float32))
+    idx, _ = ora.select_topk(rng.normal(0, 1, (B, N)).astype(np.float32), 0, N, K)
+    Y = gen.f32_to_bf16_bits(rng.normal(0, 1, (B * K, d)).astype(np.float32))
+    return h, idx, Y
+
+
+@pytest.mark.parametrize("B,N,d,K", [(1, 1, 8, 1), (3, 100, 264, 37), (2, 4096, 3584, 1229), (4, 1024, 1536, 0)])
+def test_gather_bit_exact(B, N, d, K):
+    h, idx, _ = _rows_case(B, N, d, K, 1)
+    X = torch.zeros((B * K, d), dtype=torch.bfloat16, device="cuda")
+    cer.cer_gather(bf16_dev(h), i32_dev(idx), X)
+    cer.cer_sync_status()
+    assert np.array_equal(bits_host(X), ora.gather(h, idx))
+
+
+@pytest.mark.parametrize("B,N,d,K", [(1, 1, 8, 1), (3, 100, 264, 37), (2, 4096, 3584, 1229)])
+def test_scatter_add_bit_exact(B, N, d, K):
+    h, idx, Y = _rows_case(B, N, d, K, 2)
+    hd = bf16_dev(h)
+    cer.cer_scatter_add(hd, i32_dev(idx), bf16_dev(Y))
+    cer.cer_sync_status()
+    want = ora.scatter_add(h, idx, ora.bf16_to_f64(Y))
+    assert np.array_equal(bits_host(hd), want)
+
+
+def test_out_of_range_index_is_reported_not_followed():
+    h, idx, _ = _rows_case(1, 50, 64, 10, 3)
+    idx = idx.copy()
+    idx[0, 4] = 50 + 7
+    X = torch.zeros((10, 64), dtype=torch.bfloat16, device="cuda")
+    cer.cer_gather(bf16_dev(h), i32_dev(idx), X)
+    with pytest.raises(cer.CerError) as e:
+        cer.cer_sync_status()
+    assert e.value.status == 10
+    got = bits_host(X)
+    good = [j for j in range(10) if j != 4]
+    assert np.array_equal(got[good], h[0, idx[0, good]])
+    assert not got[4].any()
+
+
+# ------------------------------------------------------------------ S1 score
+
+def _score_case(name):
+    rng = np.random.default_rng(zlib.crc32(name.encode()))
+
+    def bf(shape, s):
+        return gen.f32_to_bf16_bits(rng.normal(0, s, shape).astype(np.float32))
+    if name == "tiny":
+        w = gen.tiny()
+        inp = gen.make_inputs(w)
+        return inp, w.task
+    if name == "und_ragged_bias":
+        B, N, d, Hc = 3, 300, 512, 256
+        inp = dict(h=bf((B, N, d), 1), W1=bf((Hc, d), d ** -.5), w2=rng.normal(0, Hc ** -.5, Hc).astype(np.float32),
+                   b1=rng.normal(0, .1, Hc).astype(np.float32), t=np.zeros(B, np.float32))
+        return inp, 0
+    if name in ("gen_segments", "gen_segments_noU"):
+        B, N, d, Hc, He, E, S = 4, 130, 384, 192, 128, 32, 4
+        inp = dict(h=bf((B, N, d), 1), W1=bf((Hc, d), d ** -.5), w2=rng.normal(0, Hc ** -.5, Hc).astype(np.float32),
+                   b1=None, W1e=bf((S, He, d), d ** -.5), w2e=rng.normal(0, He ** -.5, (S, He)).astype(np.float32),
+                   Ue=bf((S, He, E), E ** -.5) if name == "gen_segments" else None,
+                   b1e=rng.normal(0, .1, (S, He)).astype(np.float32),
+                   t=np.array([0.05, 0.3, 0.6, 0.999], np.float32))
+        return inp, 1
+    raise KeyError(name)
+
+
+def _oracle_logits(inp, task):
+    return ora.score(inp["h"], inp["W1"], inp["w2"], inp.get("b1"), inp["t"], task, inp.get("W1e"),
+                     inp.get("w2e"), inp.get("Ue"), inp.get("b1e"))
+
+
+@pytest.mark.parametrize("name", ["tiny", "und_ragged_bias", "gen_segments", "gen_segments_noU"])
+def test_score_matches_oracle(name):
+    inp, task = _score_case(name)
+    B, N, d = inp["h"].shape
+    core, exp = scorers(inp)
+    logits = torch.empty((B, N), dtype=torch.float32, device="cuda")
+    probs = torch.empty((B, N), dtype=torch.float32, device="cuda")
+    cer.cer_score(bf16_dev(inp["h"]), core, exp, f32_dev(inp["t"]), task, logits, probs)
+    cer.cer_sync_status()
+    want = _oracle_logits(inp, task)
+    assert rel_err(logits.cpu().numpy(), want) <= SCORE_TOL
+    assert np.max(np.abs(probs.cpu().numpy() - ora.sigmoid(want))) <= 1e-5
+
+
+# ------------------------------------------------------------------ S4 FFN
+
+@pytest.mark.parametrize("M,d,I,C,pruned", [(1, 256, 1024, 512, True), (127, 256, 1024, 512, True),
+                                            (300, 512, 640, 640, False), (129, 1536, 8960, 6720, True)])
+def test_routed_ffn_matches_oracle(M, d, I, C, pruned):
+    rng = np.random.default_rng(M + d)
+    X = gen.f32_to_bf16_bits(rng.normal(0, 1, (M, d)).astype(np.float32))
+    Wg, Wu = (gen.bf16_normal(M, n, (I, d), d ** -.5) for n in ("g", "u"))
+    WdT = gen.bf16_normal(M, "dn", (I, d), I ** -.5)
+    chan = gen.channel_keep_set(M, "c", I, C) if pruned else None
+    Y = torch.empty((M, d), dtype=torch.bfloat16, device="cuda")
+    cer.cer_routed_ffn(bf16_dev(X), bf16_dev(Wg), bf16_dev(Wu), bf16_dev(WdT), i32_dev(chan), Y)
+    cer.cer_sync_status()
+    want = ora.routed_ffn(X, Wg, Wu, WdT, chan if pruned else np.arange(I))
+    got = ora.bf16_to_f64(bits_host(Y))
+    assert np.max(np.abs(got - want)) <= OUT_TOL * rms(want)
+
+
+# ------------------------------------------------------------------ fused block
+
+_WEIGHTS = {}
+
+
+def _inputs(w):
+    """Inputs of a full-size workload; FFN weights drawn once per (seed, I, d)."""
+    key = (w.seed, w.I, w.d)
+    if key not in _WEIGHTS:
+        _WEIGHTS.clear()
+        inp = gen.make_inputs(w)
+        _WEIGHTS[key] = (inp["Wg"], inp["Wu"], inp["WdT"])
+        return inp
+    return gen.make_inputs(w, ffn_weights=_WEIGHTS[key])
+
+
+def _run_block(w, inp, out_of_place=False):
+    core, exp = scorers(inp)
+    h = bf16_dev(inp["h"])
+    out = torch.empty_like(h) if out_of_place else None
+    logits = torch.empty((w.B, w.N), dtype=torch.float32, device="cuda")
+    idx = torch.empty((w.B, w.k_tot), dtype=torch.int32, device="cuda")
+    mask = torch.empty((w.B, w.N), dtype=torch.uint8, device="cuda")
+    chan = i32_dev(inp["chan"]) if w.C < w.I else None
+    cer.cer_routed_block(h, core, exp if w.task == 1 else None, f32_dev(inp["t"]), w.task, w.r0, w.r1, w.K,
+                         bf16_dev(inp["Wg"]), bf16_dev(inp["Wu"]), bf16_dev(inp["WdT"]), chan,
+                         out=out, logits=logits, idx=idx, mask=mask)
+    cer.cer_sync_status()
+    res = dict(out=bits_host(out if out_of_place else h), logits=logits.cpu().numpy(), idx=idx.cpu().numpy(),
+               mask=mask.cpu().numpy())
+    if out_of_place:
+        res["h_after"] = bits_host(h)
+    return res
+
+
+def _check_block(w, inp, res, sample_rows=None, seed=0):
+    h = inp["h"]
+    # S1: logits against the oracle's
+    want_logits = _oracle_logits(inp, w.task)
+    assert rel_err(res["logits"], want_logits) <= SCORE_TOL
+    # S2: the GPU keep list is exactly the oracle's selection on the GPU's logits ...
+    idx_o, mask_o = ora.select_topk(res["logits"], w.r0, w.r1, w.K)
+    assert np.array_equal(res["idx"], idx_o)
+    assert np.array_equal(res["mask"], mask_o)
+    # ... and any difference from the oracle's own selection is a near-tie at the K-th boundary
+    idx_ref, _ = ora.select_topk(want_logits, w.r0, w.r1, w.K)
+    rms_l = rms(want_logits)
+    for b in range(w.B):
+        diff = set(idx_ref[b].tolist()) ^ set(res["idx"][b].tolist())
+        if diff and w.K > 0:
+            routable = want_logits[b, w.r0:w.r1].astype(np.float64)
+            kth = np.sort(routable)[::-1][w.K - 1]
+            for i in diff:
+                assert abs(float(want_logits[b, i]) - kth) <= 4 * SCORE_TOL * max(abs(kth), 1e-2 * rms_l)
+    # S5 bypass: dropped rows bit-identical
+    dropped = res["mask"] == 0
+    assert np.array_equal(res["out"][dropped], h[dropped])
+    # S3-S5 kept rows against the oracle FFN evaluated on the GPU's keep list
+    rows = np.arange(w.M)
+    if sample_rows is not None and sample_rows < w.M:
+        rows = np.sort(np.random.default_rng(seed).choice(w.M, sample_rows, replace=False))
+    b_of = rows // w.k_tot
+    tok = res["idx"].reshape(-1)[rows]
+    X = h[b_of, tok]
+    y = ora.routed_ffn(X, inp["Wg"], inp["Wu"], inp["WdT"], inp["chan"])
+    want = ora.bf16_to_f64(ora.round_to_bf16(ora.bf16_to_f64(X) + y))
+    got = ora.bf16_to_f64(res["out"][b_of, tok])
+    assert np.max(np.abs(got - want)) <= OUT_TOL * rms(want)
+
+
+def _small(name):
+    base = dict(B=2, N=300, d=256, I=1024, C=512, r0=20, r1=290, K=100, Hc=128, He=64, E=64, task=1)
+    variants = {
+        "ragged_gen": {},
+        "und_text_tail": dict(task=0, He=0, E=0, r0=0, r1=200, K=77, B=3),
+        "k0": dict(K=0),
+        "dense_all_kept": dict(r0=0, r1=300, K=300, C=1024),
+        "segments": dict(n_segments=4, B=4, N=130, r0=0, r1=130, K=65),
+        "one_token": dict(B=1, N=1, r0=0, r1=1, K=1),
+        "d3584": dict(B=1, N=200, d=3584, I=2048, C=1024, r0=0, r1=200, K=60),
+    }
+    kw = dict(base)
+    kw.update(variants[name])
+    return gen.Workload(name=name, **kw)
+
+
+@pytest.mark.parametrize("name", ["ragged_gen", "und_text_tail", "k0", "dense_all_kept", "segments", "one_token",
+                                  "d3584"])
+def test_routed_block_small(name):
+    w = _small(name)
+    inp = gen.make_inputs(w)
+    res = _run_block(w, inp)
+    _check_block(w, inp, res)
+
+
+def test_routed_block_tiny_config_full_compare():
+    w = gen.tiny()
+    inp = gen.make_inputs(w)
+    res = _run_block(w, inp)
+    _check_block(w, inp, res)
+    full = ora.routed_block(inp["h"], inp["W1"], inp["w2"], None, inp["t"], w.task, w.r0, w.r1, w.K, inp["Wg"],
+                            inp["Wu"], inp["WdT"], inp["chan"], inp["W1e"], inp["w2e"], inp["Ue"], None)
+    if np.array_equal(full["idx"], res["idx"]):
+        diff = np.abs(ora.bf16_to_f64(res["out"]) - ora.bf16_to_f64(full["out"]))
+        assert diff.max() <= OUT_TOL * rms(ora.bf16_to_f64(full["out"]))
+
+
+def test_routed_block_out_of_place_leaves_h():
+    w = _small("ragged_gen")
+    inp = gen.make_inputs(w)
+    res = _run_block(w, inp, out_of_place=True)
+    assert np.array_equal(res["h_after"], inp["h"])
+    _check_block(w, inp, res)
+
+
+def test_stage_events_are_recorded():
+    w = _small("ragged_gen")
+    inp = gen.make_inputs(w)
+    core, exp = scorers(inp)
+    h = bf16_dev(inp["h"])
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
+    cer.cer_routed_block(h, core, exp, f32_dev(inp["t"]), 1, w.r0, w.r1, w.K, bf16_dev(inp["Wg"]),
+                         bf16_dev(inp["Wu"]), bf16_dev(inp["WdT"]), i32_dev(inp["chan"]), stage_events=evs)
+    cer.cer_sync_status()
+    times = [evs[i].elapsed_time(evs[i + 1]) for i in range(4)]
+    assert all(t >= 0 for t in times) and sum(times) > 0
+
+
+@pytest.mark.parametrize("wname", ["und_1p5b", "gen_1p5b", "long_7b"])
+def test_routed_block_full_size_sampled(wname):
+    w = gen.WORKLOADS[wname]()
+    inp = _inputs(w)
+    res = _run_block(w, inp)
+    _check_block(w, inp, res, sample_rows=48, seed=1)
+
+
+@pytest.mark.parametrize("n,tr,fr", [(1024, 0.1, 0.25), (16384, 0.9, 1.0), (4096, 0.5, 0.5)])
+def test_routed_block_sweep_points_sampled(n, tr, fr):
+    w = gen.sweep(n, tr, fr)
+    inp = _inputs(w)
+    res = _run_block(w, inp)
+    _check_block(w, inp, res, sample_rows=32, seed=2)
