@@ -1,0 +1,355 @@
+#!/usr/bin/env python
+"""Benchmark of the routed block (score -> top-K -> gather -> pruned SwiGLU FFN
+-> scatter-add) on GB300, one JSON line on stdout (rank 0).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--config und_1p5b]
+  python bench.py --impl reference ...      # the CPU oracle on the same workload
+
+A step is one cer_routed_block call (in place on the residual stream h) over
+the whole synthetic batch of the workload, inputs resident in HBM.  Between
+timed steps, outside the timed interval, h is restored from a pristine copy
+and L2 is flushed (a 256 MiB write); each step is timed with CUDA events on
+the launching stream.  For N > 1 each
+rank runs its own replica batch (weak scaling, no data-path collective); the
+slowest rank's time is reported.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import re
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+from paper_2608_29291_gb300 import inputs as gen  # noqa: E402
+from paper_2608_29291_gb300 import runtime  # noqa: E402
+
+METRIC = "routed block tokens/s; FFN TFLOP/s & gather/scatter GB/s vs GB300 peak"
+UNIT = "tokens/s"
+KERNELS_PER_STEP = 5      # time-bias table, scorer GEMM, top-K, gate/up GEMM, down GEMM
+FLUSH_BYTES = 256 << 20   # > 129 MB L2
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+GEMM_SOURCES = ("ffn_kernel.cu", "umma_gemm.cuh", "ptx.cuh")
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            return json.load(f), "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+def gemm_source_hash() -> str:
+    h = hashlib.sha256()
+    for name in GEMM_SOURCES:
+        with open(os.path.join(ROOT, "paper_2608_29291_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(workload: str):
+    """DRAM bytes per gate/up launch from the committed ncu summary, if it was
+    taken on this workload with the current kernel sources; else None."""
+    path = os.path.join(ROOT, "profiles", "ffn_gateup_traffic.md")
+    if not os.path.exists(path):
+        return None
+    text = open(path).read()
+    m_src = re.search(r"kernel_source_hash:\s*([0-9a-f]+)", text)
+    m_wl = re.search(r"workload:\s*(\S+)", text)
+    m_b = re.search(r"dram_bytes_per_launch:\s*([0-9]+)", text)
+    if not (m_src and m_wl and m_b) or m_src.group(1) != gemm_source_hash() or m_wl.group(1) != workload:
+        return None
+    return int(m_b.group(1))
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling around the timed region."""
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.QUERY}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        self.t0 = time.time()
+
+    def stop(self):
+        if self.proc is None:
+            return
+        time.sleep(0.05)
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        self.lines = [ln for ln in out.splitlines() if ln.strip()]
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for name, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def smi_index(local_rank: int) -> str:
+    """nvidia-smi's name for this rank's GPU (honours CUDA_VISIBLE_DEVICES)."""
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+    if vis:
+        ids = [x.strip() for x in vis.split(",") if x.strip()]
+        if local_rank < len(ids):
+            return ids[local_rank]
+    return str(local_rank)
+
+
+def workload_config(w: gen.Workload, flush: bool) -> dict:
+    return {"workload": w.name, "B": w.B, "N": w.N, "d": w.d, "intermediate": w.I, "kept_channels": w.C,
+            "routable": [w.r0, w.r1], "K": w.K, "kept_rows": w.M, "core_hidden": w.Hc, "exp_hidden": w.He,
+            "task": "generation" if w.task == 1 else "understanding",
+            "l2": "flushed between timed steps (256 MiB write)" if flush else "not flushed",
+            "inputs": "seeded synthetic (SplitMix64 normals), resident in HBM"}
+
+
+# ------------------------------------------------------------------ CPU oracle timing
+
+def time_oracle(w: gen.Workload, inp: dict, min_seconds: float, max_reps: int = 50):
+    """The oracle as it stands on one sequence of the workload, repeated until
+    min_seconds; returns (tokens/s, seconds, reps)."""
+    from oracle import cer_oracle as ora
+    b = 0
+    sl = slice(b, b + 1)
+    args = (inp["h"][sl], inp["W1"], inp["w2"], inp.get("b1"), inp["t"][sl], w.task, w.r0, w.r1, w.K,
+            inp["Wg"], inp["Wu"], inp["WdT"], inp["chan"], inp.get("W1e"), inp.get("w2e"), inp.get("Ue"),
+            inp.get("b1e"))
+    t0 = time.perf_counter()
+    reps = 0
+    while True:
+        ora.routed_block(*args)
+        reps += 1
+        el = time.perf_counter() - t0
+        if el >= min_seconds or reps >= max_reps:
+            break
+    return w.N * reps / el, el, reps
+
+
+def blas_threads() -> int:
+    for var in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS", "MKL_NUM_THREADS"):
+        v = os.environ.get(var)
+        if v and v.isdigit():
+            return int(v)
+    return os.cpu_count() or 1
+
+
+def run_reference(args, info):
+    """--impl reference: the CPU oracle, timed on the host cores, same workload."""
+    if not info.is_root:
+        return 0
+    w = gen.WORKLOADS[args.config]()
+    inp = gen.make_inputs(w)
+    for _ in range(args.warmup):
+        time_oracle(w, inp, 0.0, max_reps=1)
+    times = []
+    for _ in range(args.steps):
+        _, el, _ = time_oracle(w, inp, 0.0, max_reps=1)
+        times.append(el)
+    t = float(np.mean(times))
+    value = w.N / t
+    sample = f"one sequence ({w.N} tokens) of {w.name} per step, full routed block in fp64 numpy"
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": t * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": workload_config(w, False),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": blas_threads(), "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ------------------------------------------------------------------ GPU arm
+
+def run_gpu(args, info):
+    import torch
+    from paper_2608_29291_gb300 import cer
+
+    torch.cuda.set_device(info.local_rank)
+    dev = torch.device("cuda", info.local_rank)
+    dist = runtime.init_group(info, "nccl")
+    cer.load()
+
+    base = gen.WORKLOADS[args.config]()
+    w = gen.Workload(**{**base.__dict__, "seed": runtime.replica_seed(base.seed, info.rank)})
+    inp = gen.make_inputs(w)
+
+    def bf(bits):
+        return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).to(dev)
+
+    def f32(a):
+        return None if a is None else torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(dev)
+
+    core = cer.Scorer(W1=bf(inp["W1"]), w2=f32(inp["w2"]), b1=f32(inp.get("b1")))
+    exp = None
+    if w.task == 1:
+        exp = cer.Scorer(W1=bf(inp["W1e"]), w2=f32(inp["w2e"]), U=bf(inp["Ue"]) if inp.get("Ue") is not None else None)
+    h = bf(inp["h"])
+    h0 = h.clone()          # pristine residual stream, restored before every step
+    t = f32(inp["t"])
+    Wg, Wu, WdT = bf(inp["Wg"]), bf(inp["Wu"]), bf(inp["WdT"])
+    chan = torch.from_numpy(inp["chan"]).to(dev) if w.C < w.I else None
+    ws = cer.workspace(cer.cer_routed_block_workspace_size(w.B, w.N, w.d, w.Hc, w.He if w.task else 0, w.task,
+                                                           w.r0, w.r1, w.K, w.C), dev)
+    flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step(stage_events=None):
+        cer.cer_routed_block(h, core, exp, t, w.task, w.r0, w.r1, w.K, Wg, Wu, WdT, chan, ws=ws,
+                             stage_events=stage_events, stream=stream)
+
+    def prepare(i):
+        """Outside the timed interval: restore h (the block updates it in place),
+        then evict L2 with a 256 MiB write so the step reads its inputs from HBM."""
+        h.copy_(h0)
+        flush.fill_(float(i))
+
+    for i in range(args.warmup):
+        prepare(i)
+        step()
+    cer.cer_sync_status(stream)
+
+    # ---- device-timed region: K steps, L2 flushed between steps
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(args.steps)]
+    clocks = ClockSampler(smi_index(info.local_rank))
+    clocks.start()
+    time.sleep(0.3)
+    runtime.barrier(dist)
+    torch.cuda.synchronize(dev)
+    for i in range(args.steps):
+        prepare(i)
+        step(evs[i])
+    torch.cuda.synchronize(dev)
+    runtime.barrier(dist)
+    clocks.stop()
+    cer.cer_sync_status(stream)
+    stage = np.array([[e[j].elapsed_time(e[j + 1]) for j in range(4)] for e in evs])   # ms
+    step_ms = stage.sum(axis=1)
+    mean_ms = float(step_ms.mean())
+    slow_ms = runtime.max_over_ranks(dist, mean_ms, device=dev)
+    tokens = w.B * w.N * info.world
+    value = tokens / (slow_ms * 1e-3)
+
+    # ---- end to end through the public API: pinned host h in, h out
+    h_host = torch.from_numpy(np.ascontiguousarray(inp["h"]).view(np.int16)).view(torch.bfloat16).pin_memory()
+    t_host = torch.from_numpy(np.ascontiguousarray(inp["t"], dtype=np.float32)).pin_memory()
+    out_host = torch.empty_like(h_host).pin_memory()
+    e2e_steps = max(3, min(args.steps, 50))
+    e_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(e2e_steps)]
+    for i in range(e2e_steps):
+        flush.fill_(float(i))
+        e_ev[i][0].record(stream)
+        h.copy_(h_host, non_blocking=True)
+        t.copy_(t_host, non_blocking=True)
+        step()
+        out_host.copy_(h, non_blocking=True)
+        e_ev[i][1].record(stream)
+    torch.cuda.synchronize(dev)
+    cer.cer_sync_status(stream)
+    e2e_ms = runtime.max_over_ranks(dist, float(np.mean([a.elapsed_time(b) for a, b in e_ev])), device=dev)
+    h2d = h_host.numel() * 2 + t_host.numel() * 4
+    d2h = out_host.numel() * 2
+
+    if not info.is_root:
+        return 0
+
+    peaks, peak_kind = load_peaks()
+    gateup_ms = float(stage[:, 2].mean())
+    gateup_flops = 4.0 * w.M * w.d * w.C
+    achieved = gateup_flops / (gateup_ms * 1e-3) / 1e12
+    peak = float(peaks["bf16_tflops"])
+    down_ms = float(stage[:, 3].mean())
+    down_flops = 2.0 * w.M * w.d * w.C
+    score_ms = float(stage[:, 0].mean())
+    topk_ms = float(stage[:, 1].mean())
+
+    cpu = None
+    if info.world == 1 and not args.no_cpu_baseline:
+        cps, el, reps = time_oracle(w, inp, args.cpu_seconds)
+        cpu = {"value": cps, "unit": UNIT, "cores": blas_threads(), "kind": "oracle",
+               "sample": f"{reps} x one sequence ({w.N} tokens) of {w.name}, full routed block, fp64 numpy, "
+                         f"{el:.1f} s"}
+
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": info.world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": slow_ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": workload_config(w, True),
+        "roofline": {"kernel": "ffn gate/up GEMM (tcgen05, fused row gather + SwiGLU)", "bound": "tensor",
+                     "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
+                     "peak_source": f"bf16_tflops (burst) of {peak_kind}",
+                     "algorithmic_flops_per_launch": gateup_flops,
+                     "traffic": profiled_traffic(w.name)},
+        "stages_ms": {"score": score_ms, "topk": topk_ms, "ffn_gateup": gateup_ms, "ffn_down_scatter": down_ms},
+        "ffn_tflops": (gateup_flops + down_flops) / ((gateup_ms + down_ms) * 1e-3) / 1e12,
+        "score_tflops": w.score_flops() / (score_ms * 1e-3) / 1e12,
+        "cpu_baseline": cpu,
+        "e2e": {"value": tokens / (e2e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
+        "gpu_launches": KERNELS_PER_STEP * args.steps,
+        "clocks": clocks.summary(),
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=("cer", "reference"), default="cer")
+    ap.add_argument("--config", choices=sorted(gen.WORKLOADS), default="und_1p5b")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    info = runtime.rank_info()
+    if args.impl == "reference":
+        return run_reference(args, info)
+    return run_gpu(args, info)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

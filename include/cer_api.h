@@ -14,6 +14,7 @@
  *           caller-supplied `workspace` of at least the size reported by the
  *           matching *_workspace_size() function (256-byte aligned).
  * Alignment. Every tensor pointer must be 16-byte aligned (CER_ERR_ALIGN).
+ *           A pointer to a tensor with no elements may be NULL.
  * Streams.  Work is enqueued asynchronously on `stream` (0 = legacy default
  *           stream); a call returns before the GPU finishes.
  * Errors.   Argument checks run on the host before any launch: on failure

@@ -89,6 +89,8 @@ size_t round256(size_t x) { return (x + 255) & ~size_t(255); }
   } while (0)
 
 #define CER_PTR(p) CER_REQUIRE((p) != nullptr, CER_ERR_NULL, "%s is NULL", #p)
+// A pointer that may be NULL only when the tensor it stands for is empty.
+#define CER_PTR_IF(p, nonempty) CER_REQUIRE(!(nonempty) || (p) != nullptr, CER_ERR_NULL, "%s is NULL", #p)
 #define CER_ALIGN(p) CER_REQUIRE((p) == nullptr || aligned16(p), CER_ERR_ALIGN, "%s is not 16-byte aligned", #p)
 
 struct ScoreShape {
@@ -114,7 +116,7 @@ cer_status check_scorer(const cer_scorer* s, const char* name, bool is_core, int
 
 cer_status check_score_args(const void* h, int B, int N, int d, const cer_scorer* core, const cer_scorer* exp,
                             const float* t, int task, ScoreShape* sh) {
-  CER_PTR(h);
+  CER_PTR_IF(h, static_cast<long long>(B) * N > 0);
   CER_ALIGN(h);
   CER_ALIGN(t);
   CER_REQUIRE(task == CER_TASK_UND || task == CER_TASK_GEN, CER_ERR_RANGE, "task=%d is neither UND nor GEN", task);
@@ -127,7 +129,7 @@ cer_status check_score_args(const void* h, int B, int N, int d, const cer_scorer
   if (sh->gen) {
     s = check_scorer(exp, "expansion", false, &sh->He);
     if (s != CER_OK) return s;
-    CER_PTR(t);
+    CER_PTR_IF(t, B > 0);
   }
   const int bn = cer::score_chunk_width(sh->Hc, sh->He, sh->gen);
   CER_REQUIRE(bn > 0, CER_ERR_SHAPE, "scorer hidden widths must be multiples of 64");
@@ -291,7 +293,7 @@ cer_status cer_score(const void* h, int B, int N, int d, const cer_scorer* core,
   ScoreShape sh;
   cer_status s = check_score_args(h, B, N, d, core, exp, t, task, &sh);
   if (s != CER_OK) return s;
-  CER_PTR(logits);
+  CER_PTR_IF(logits, static_cast<long long>(B) * N > 0);
   CER_ALIGN(logits);
   CER_ALIGN(probs);
   CER_ALIGN(workspace);
@@ -313,8 +315,8 @@ cer_status cer_score(const void* h, int B, int N, int d, const cer_scorer* core,
 
 cer_status cer_select_topk(const float* logits, int B, int N, int r0, int r1, int K, int32_t* idx, uint8_t* mask,
                            cudaStream_t stream) {
-  CER_PTR(logits);
-  CER_PTR(idx);
+  CER_PTR_IF(logits, static_cast<long long>(B) * N > 0);
+  CER_PTR_IF(idx, static_cast<long long>(B) * (K + N - (r1 - r0)) > 0);
   CER_ALIGN(logits);
   CER_ALIGN(idx);
   CER_ALIGN(mask);
@@ -343,9 +345,9 @@ cer_status cer_select_topk(const float* logits, int B, int N, int r0, int r1, in
 
 cer_status cer_gather(const void* h, int B, int N, int d, const int32_t* idx, int k_tot, void* X,
                       cudaStream_t stream) {
-  CER_PTR(h);
-  CER_PTR(idx);
-  CER_PTR(X);
+  CER_PTR_IF(h, static_cast<long long>(B) * N > 0);
+  CER_PTR_IF(idx, static_cast<long long>(B) * k_tot > 0);
+  CER_PTR_IF(X, static_cast<long long>(B) * k_tot > 0);
   CER_ALIGN(h);
   CER_ALIGN(idx);
   CER_ALIGN(X);
@@ -362,9 +364,9 @@ cer_status cer_gather(const void* h, int B, int N, int d, const int32_t* idx, in
 
 cer_status cer_scatter_add(void* h, int B, int N, int d, const int32_t* idx, int k_tot, const void* Y,
                            cudaStream_t stream) {
-  CER_PTR(h);
-  CER_PTR(idx);
-  CER_PTR(Y);
+  CER_PTR_IF(h, static_cast<long long>(B) * N > 0);
+  CER_PTR_IF(idx, static_cast<long long>(B) * k_tot > 0);
+  CER_PTR_IF(Y, static_cast<long long>(B) * k_tot > 0);
   CER_ALIGN(h);
   CER_ALIGN(idx);
   CER_ALIGN(Y);
@@ -387,11 +389,11 @@ size_t cer_routed_ffn_workspace_size(int M, int C) {
 cer_status cer_routed_ffn(const void* X, int M, int d, const void* Wg, const void* Wu, const void* WdT, int I,
                           const int32_t* chan, int C, void* Y, void* workspace, size_t workspace_bytes,
                           cudaStream_t stream) {
-  CER_PTR(X);
+  CER_PTR_IF(X, M > 0);
   CER_PTR(Wg);
   CER_PTR(Wu);
   CER_PTR(WdT);
-  CER_PTR(Y);
+  CER_PTR_IF(Y, M > 0);
   CER_ALIGN(X);
   CER_ALIGN(Wg);
   CER_ALIGN(Wu);

@@ -15,7 +15,8 @@ namespace cer {
 bool encode_bf16_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_cols,
                     uint32_t box_rows);
 
-// Raise a kernel's dynamic shared-memory limit once per device.
+// Raise a kernel's dynamic shared-memory limit to `bytes` (its largest
+// launch) once per device.
 cudaError_t ensure_max_smem(const void* func, size_t bytes);
 
 // ------------------------------------------------------------------ S1 score

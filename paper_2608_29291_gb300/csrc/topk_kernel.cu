@@ -187,7 +187,8 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(TopkArgs a) {
 cudaError_t launch_topk(const TopkArgs& a, cudaStream_t stream) {
   if (a.B == 0 || a.N == 0) return cudaSuccess;
   const size_t smem = static_cast<size_t>(a.N) * sizeof(uint32_t);
-  cudaError_t e = ensure_max_smem(reinterpret_cast<const void*>(topk_kernel), smem);
+  // The limit is raised once per device to the largest N ever accepted.
+  cudaError_t e = ensure_max_smem(reinterpret_cast<const void*>(topk_kernel), kTopkMaxN * sizeof(uint32_t));
   if (e != cudaSuccess) return e;
   topk_kernel<<<a.B, kTopkThreads, smem, stream>>>(a);
   return cudaGetLastError();

@@ -30,14 +30,36 @@ def scorers(inp: dict, dev="cuda"):
     return core, exp
 
 
-def rel_err(got: np.ndarray, want: np.ndarray, floor_frac: float = 1e-2) -> float:
-    """max |got - want| / max(|want|, floor_frac * RMS(want)), elementwise."""
+def rel_err(got: np.ndarray, want: np.ndarray, floor_frac: float = 1.0) -> float:
+    """max |got - want| / max(|want|, floor_frac * RMS(want)), elementwise.
+
+    The RMS floor puts near-zero scores on the scale of the score array: fp32
+    accumulation over d products leaves an absolute error of order
+    sqrt(d) * 2^-24 * RMS, independent of a score's own size."""
     want = np.asarray(want, dtype=np.float64)
     got = np.asarray(got, dtype=np.float64)
     rms = float(np.sqrt(np.mean(want ** 2))) if want.size else 0.0
     den = np.maximum(np.abs(want), floor_frac * rms)
     den = np.where(den == 0, 1.0, den)
     return float(np.max(np.abs(got - want) / den)) if want.size else 0.0
+
+
+def ulp_bf16(x) -> np.ndarray:
+    """Spacing of bf16 values at |x| (8 significant bits); 2^-133 below the normal range."""
+    a = np.abs(np.asarray(x, dtype=np.float64))
+    e = np.floor(np.log2(np.maximum(a, 2.0 ** -126)))
+    return np.exp2(e - 7)
+
+
+def out_err_ok(got_bf16: np.ndarray, exact: np.ndarray, tol_frac: float):
+    """A bf16 output against the oracle's unrounded fp64 value: the error must
+    stay within tol_frac * RMS(exact) plus half a bf16 ulp (the final rounding,
+    which may land either side of a rounding boundary).  Returns (ok, worst excess)."""
+    got = np.asarray(got_bf16, dtype=np.float64)
+    exact = np.asarray(exact, dtype=np.float64)
+    bound = tol_frac * rms(exact) + 0.5 * ulp_bf16(np.maximum(np.abs(exact), np.abs(got)))
+    excess = np.abs(got - exact) - bound
+    return bool(np.all(excess <= 0)), float(excess.max()) if excess.size else 0.0
 
 
 def rms(x) -> float:

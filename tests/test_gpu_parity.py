@@ -1,7 +1,8 @@
 """GPU parity: every C-ABI entry point against the CPU oracle on the same seeded
 inputs.  Bars: keep lists and masks bit-exact given the same fp32 logits;
-gather and scatter bit-exact; logits within 1e-4 relative (floor 1e-2 RMS);
-FFN and block outputs within 2e-2 x RMS of the oracle's output."""
+gather and scatter bit-exact; logits within 1e-4 relative to max(|l|, RMS(l));
+FFN and block outputs (bf16) within 2e-2 x RMS of the oracle's unrounded fp64
+output plus half a bf16 ulp for the final rounding."""
 import zlib
 
 import numpy as np
@@ -11,7 +12,7 @@ import torch
 from oracle import cer_oracle as ora
 from paper_2608_29291_gb300 import cer
 from paper_2608_29291_gb300 import inputs as gen
-from tests.gpu_helpers import bf16_dev, bits_host, f32_dev, i32_dev, rel_err, rms, scorers
+from tests.gpu_helpers import bf16_dev, bits_host, f32_dev, i32_dev, out_err_ok, rel_err, rms, scorers
 
 pytestmark = pytest.mark.gpu
 
@@ -188,8 +189,8 @@ def test_routed_ffn_matches_oracle(M, d, I, C, pruned):
     cer.cer_routed_ffn(bf16_dev(X), bf16_dev(Wg), bf16_dev(Wu), bf16_dev(WdT), i32_dev(chan), Y)
     cer.cer_sync_status()
     want = ora.routed_ffn(X, Wg, Wu, WdT, chan if pruned else np.arange(I))
-    got = ora.bf16_to_f64(bits_host(Y))
-    assert np.max(np.abs(got - want)) <= OUT_TOL * rms(want)
+    ok, excess = out_err_ok(ora.bf16_to_f64(bits_host(Y)), want, OUT_TOL)
+    assert ok, excess
 
 
 # ------------------------------------------------------------------ fused block
@@ -245,7 +246,7 @@ def _check_block(w, inp, res, sample_rows=None, seed=0):
             routable = want_logits[b, w.r0:w.r1].astype(np.float64)
             kth = np.sort(routable)[::-1][w.K - 1]
             for i in diff:
-                assert abs(float(want_logits[b, i]) - kth) <= 4 * SCORE_TOL * max(abs(kth), 1e-2 * rms_l)
+                assert abs(float(want_logits[b, i]) - kth) <= 4 * SCORE_TOL * max(abs(kth), rms_l)
     # S5 bypass: dropped rows bit-identical
     dropped = res["mask"] == 0
     assert np.array_equal(res["out"][dropped], h[dropped])
@@ -257,9 +258,9 @@ def _check_block(w, inp, res, sample_rows=None, seed=0):
     tok = res["idx"].reshape(-1)[rows]
     X = h[b_of, tok]
     y = ora.routed_ffn(X, inp["Wg"], inp["Wu"], inp["WdT"], inp["chan"])
-    want = ora.bf16_to_f64(ora.round_to_bf16(ora.bf16_to_f64(X) + y))
-    got = ora.bf16_to_f64(res["out"][b_of, tok])
-    assert np.max(np.abs(got - want)) <= OUT_TOL * rms(want)
+    exact = ora.bf16_to_f64(X) + y
+    ok, excess = out_err_ok(ora.bf16_to_f64(res["out"][b_of, tok]), exact, OUT_TOL)
+    assert ok, excess
 
 
 def _small(name):
@@ -295,8 +296,11 @@ def test_routed_block_tiny_config_full_compare():
     full = ora.routed_block(inp["h"], inp["W1"], inp["w2"], None, inp["t"], w.task, w.r0, w.r1, w.K, inp["Wg"],
                             inp["Wu"], inp["WdT"], inp["chan"], inp["W1e"], inp["w2e"], inp["Ue"], None)
     if np.array_equal(full["idx"], res["idx"]):
-        diff = np.abs(ora.bf16_to_f64(res["out"]) - ora.bf16_to_f64(full["out"]))
-        assert diff.max() <= OUT_TOL * rms(ora.bf16_to_f64(full["out"]))
+        exact = ora.bf16_to_f64(inp["h"]).copy()
+        kept = full["idx"][0]
+        exact[0, kept] += full["Y"]
+        ok, excess = out_err_ok(ora.bf16_to_f64(res["out"]), exact, OUT_TOL)
+        assert ok, excess
 
 
 def test_routed_block_out_of_place_leaves_h():
