@@ -35,7 +35,7 @@ from paper_2608_29291_gb300 import runtime  # noqa: E402
 
 METRIC = "routed block tokens/s; FFN TFLOP/s & gather/scatter GB/s vs GB300 peak"
 UNIT = "tokens/s"
-KERNELS_PER_STEP = 5      # time-bias table, scorer GEMM, top-K, gate/up GEMM, down GEMM
+KERNELS_PER_STEP = 6      # time-bias table, scorer GEMM, top-K, row gather, gate/up GEMM, down GEMM
 FLUSH_BYTES = 256 << 20   # > 129 MB L2
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 GEMM_SOURCES = ("ffn_kernel.cu", "umma_gemm.cuh", "ptx.cuh")
@@ -228,9 +228,20 @@ def run_gpu(args, info):
     h0 = h.clone()          # pristine residual stream, restored before every step
     t = f32(inp["t"])
     Wg, Wu, WdT = bf(inp["Wg"]), bf(inp["Wu"]), bf(inp["WdT"])
-    chan = torch.from_numpy(inp["chan"]).to(dev) if w.C < w.I else None
+    pack_ms = None
+    if w.C < w.I:
+        # the static channel mask (one per layer) applied once, as at model load
+        chan_full = torch.from_numpy(inp["chan"]).to(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        cer.pack_ffn_weights(Wg, Wu, WdT, chan_full)            # warm
+        e0.record()
+        Wg, Wu, WdT = cer.pack_ffn_weights(Wg, Wu, WdT, chan_full)
+        e1.record()
+        torch.cuda.synchronize(dev)
+        pack_ms = e0.elapsed_time(e1)
+    chan = None
     ws = cer.workspace(cer.cer_routed_block_workspace_size(w.B, w.N, w.d, w.Hc, w.He if w.task else 0, w.task,
-                                                           w.r0, w.r1, w.K, w.C), dev)
+                                                           w.r0, w.r1, w.K, w.C, False), dev)
     flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream(dev)
 
@@ -250,7 +261,7 @@ def run_gpu(args, info):
     cer.cer_sync_status(stream)
 
     # ---- device-timed region: K steps, L2 flushed between steps
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(args.steps)]
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(args.steps)]
     clocks = ClockSampler(smi_index(info.local_rank))
     clocks.start()
     time.sleep(0.3)
@@ -263,7 +274,7 @@ def run_gpu(args, info):
     runtime.barrier(dist)
     clocks.stop()
     cer.cer_sync_status(stream)
-    stage = np.array([[e[j].elapsed_time(e[j + 1]) for j in range(4)] for e in evs])   # ms
+    stage = np.array([[e[j].elapsed_time(e[j + 1]) for j in range(5)] for e in evs])   # ms
     step_ms = stage.sum(axis=1)
     mean_ms = float(step_ms.mean())
     slow_ms = runtime.max_over_ranks(dist, mean_ms, device=dev)
@@ -294,14 +305,12 @@ def run_gpu(args, info):
         return 0
 
     peaks, peak_kind = load_peaks()
-    gateup_ms = float(stage[:, 2].mean())
+    score_ms, topk_ms, gather_ms, gateup_ms, down_ms = (float(x) for x in stage.mean(axis=0))
     gateup_flops = 4.0 * w.M * w.d * w.C
     achieved = gateup_flops / (gateup_ms * 1e-3) / 1e12
     peak = float(peaks["bf16_tflops"])
-    down_ms = float(stage[:, 3].mean())
     down_flops = 2.0 * w.M * w.d * w.C
-    score_ms = float(stage[:, 0].mean())
-    topk_ms = float(stage[:, 1].mean())
+    gather_bytes = 4.0 * w.M * w.d + 4.0 * w.M
 
     cpu = None
     if info.world == 1 and not args.no_cpu_baseline:
@@ -320,7 +329,12 @@ def run_gpu(args, info):
                      "peak_source": f"bf16_tflops (burst) of {peak_kind}",
                      "algorithmic_flops_per_launch": gateup_flops,
                      "traffic": profiled_traffic(w.name)},
-        "stages_ms": {"score": score_ms, "topk": topk_ms, "ffn_gateup": gateup_ms, "ffn_down_scatter": down_ms},
+        "stages_ms": {"score": score_ms, "topk": topk_ms, "gather": gather_ms, "ffn_gateup": gateup_ms,
+                      "ffn_down_scatter": down_ms},
+        "gather_gbs": gather_bytes / (gather_ms * 1e-3) / 1e9,
+        "ffn_weights": "kept-channel slices packed once from the full weights by cer_pack_ffn_weights "
+                       f"(static mask; {pack_ms:.3f} ms, not part of a step)" if pack_ms is not None else
+                       "all channels",
         "ffn_tflops": (gateup_flops + down_flops) / ((gateup_ms + down_ms) * 1e-3) / 1e12,
         "score_tflops": w.score_flops() / (score_ms * 1e-3) / 1e12,
         "cpu_baseline": cpu,

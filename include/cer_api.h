@@ -127,18 +127,31 @@ cer_status cer_gather(const void* h, int B, int N, int d, const int32_t* idx, in
  *   Wg,Wu bf16 [I, d]   gate and up projections, one row per channel
  *   WdT   bf16 [I, d]   down projection stored channel-major (row c is
  *                       W_down[:, c]), so that pruning is a row selection
- *   chan  int32 [C] kept channel indices in [0, I), or NULL for all (C == I);
- *         C a multiple of 64
+ *   chan  int32 [C] kept channel indices in [0, I), or NULL: then the weight
+ *         arrays hold exactly the C channels to use (C == I), e.g. the full
+ *         FFN or slices made once by cer_pack_ffn_weights; C a multiple of 64
  *   Y     bf16 [M, d] output
- * Two tcgen05 GEMMs (bf16 operands, fp32 accumulation in TMEM); the kept
- * weight rows are fetched by TMA row gathers straight from the full weights.
- * The SwiGLU activation passes through the workspace as bf16 [M, C].
- * Workspace: cer_routed_ffn_workspace_size(M, C).                            */
+ * Two tcgen05 GEMMs (bf16 operands, fp32 accumulation in TMEM) over dense
+ * TMA tiles; with chan != NULL the kept weight rows are first copied into the
+ * workspace (3*C*d*2 bytes moved twice per call).  The SwiGLU activation
+ * passes through the workspace as bf16 [M, C].
+ * Workspace: cer_routed_ffn_workspace_size(M, d, C, chan != NULL).         */
 cer_status cer_routed_ffn(const void* X, int M, int d,
                           const void* Wg, const void* Wu, const void* WdT, int I,
                           const int32_t* chan, int C, void* Y,
                           void* workspace, size_t workspace_bytes, cudaStream_t stream);
-size_t cer_routed_ffn_workspace_size(int M, int C);
+size_t cer_routed_ffn_workspace_size(int M, int d, int C, int with_chan);
+
+/* ------------------------------------------------------------------ weight slices
+ * The static channel-pruning mask of Sec. 3.4 (FFN pruning; App. A.4: the
+ * candidate mask is fixed per layer) applied once: copies the kept rows of
+ * Wg, Wu and WdT (all bf16 [I, d], d a multiple of 8) into Wg_out, Wu_out,
+ * WdT_out (bf16 [C, d]) in the order of chan (int32 [C], entries in [0, I)).
+ * Passing the outputs with chan == NULL and I == C to cer_routed_ffn or
+ * cer_routed_block runs the pruned FFN without per-call copies.           */
+cer_status cer_pack_ffn_weights(const void* Wg, const void* Wu, const void* WdT, int I, int d,
+                                const int32_t* chan, int C,
+                                void* Wg_out, void* Wu_out, void* WdT_out, cudaStream_t stream);
 
 /* ------------------------------------------------------------------ S5 scatter
  * Unpack (Sec. 3.4): h[b, idx[b, j], :] = bf16(h + Y[b*k_tot + j, :]) in place,
@@ -149,10 +162,11 @@ cer_status cer_scatter_add(void* h, int B, int N, int d, const int32_t* idx, int
                            const void* Y, cudaStream_t stream);
 
 /* ------------------------------------------------------------------ fused block
- * The whole routed block S1..S5 in four kernels on one stream:
+ * The whole routed block S1..S5 on one stream:
  *   scorer GEMM -> top-K (also reduces the scorer's partial sums) ->
- *   gate/up GEMM reading the kept rows of h by TMA row gather ->
- *   down GEMM whose epilogue adds into the kept rows of the output.
+ *   row gather of the kept tokens (and, with chan != NULL, of the kept
+ *   weight rows) -> gate/up GEMM with the SwiGLU epilogue -> down GEMM whose
+ *   epilogue adds into the kept rows of the output.
  *   h, out   bf16 [B, N, d]; out == h (or NULL) updates h in place and moves
  *            no bytes for dropped rows; otherwise out must not overlap h and
  *            dropped rows are copied (bypass)
@@ -162,11 +176,11 @@ cer_status cer_scatter_add(void* h, int B, int N, int d, const int32_t* idx, int
  *   logits   fp32 [B, N] output, or NULL
  *   idx      int32 [B, k_tot] output, or NULL
  *   mask     uint8 [B, N] output, or NULL
- *   stage_events  NULL, or n_stage_events == 5 caller-created CUDA events
- *            recorded on `stream` before the scorer, after the scorer, after
- *            the top-K, after the gate/up GEMM and after the down GEMM (for
- *            per-stage timing).
- * Workspace: cer_routed_block_workspace_size(...) with the same sizes.      */
+ *   stage_events  NULL, or n_stage_events == 6 caller-created CUDA events
+ *            recorded on `stream` at the start, after the scorer, after the
+ *            top-K, after the row gather, after the gate/up GEMM and after
+ *            the down GEMM (for per-stage timing).
+ * Workspace: cer_routed_block_workspace_size(..., chan != NULL).           */
 cer_status cer_routed_block(void* h, void* out, int B, int N, int d,
                             const cer_scorer* core, const cer_scorer* exp,
                             const float* t, int task, int r0, int r1, int K,
@@ -177,7 +191,7 @@ cer_status cer_routed_block(void* h, void* out, int B, int N, int d,
                             cudaEvent_t* stage_events, int n_stage_events,
                             cudaStream_t stream);
 size_t cer_routed_block_workspace_size(int B, int N, int d, int core_hidden, int exp_hidden,
-                                       int task, int r0, int r1, int K, int C);
+                                       int task, int r0, int r1, int K, int C, int with_chan);
 
 /* ------------------------------------------------------------------ status
  * cer_sync_status: synchronise `stream`, then return and clear the current

@@ -27,7 +27,7 @@ STATUS_NAMES = {0: "CER_OK", 1: "CER_ERR_NULL", 2: "CER_ERR_SHAPE", 3: "CER_ERR_
 
 # Every symbol include/cer_api.h declares.
 EXPORTS = ("cer_score", "cer_score_workspace_size", "cer_select_topk", "cer_gather", "cer_routed_ffn",
-           "cer_routed_ffn_workspace_size", "cer_scatter_add", "cer_routed_block",
+           "cer_routed_ffn_workspace_size", "cer_pack_ffn_weights", "cer_scatter_add", "cer_routed_block",
            "cer_routed_block_workspace_size", "cer_sync_status", "cer_get_error", "cer_status_string",
            "cer_version")
 
@@ -54,11 +54,12 @@ _SIGS = {
     "cer_select_topk": ([_vp, _i, _i, _i, _i, _i, _vp, _vp, _vp], _i),
     "cer_gather": ([_vp, _i, _i, _i, _vp, _i, _vp, _vp], _i),
     "cer_routed_ffn": ([_vp, _i, _i, _vp, _vp, _vp, _i, _vp, _i, _vp, _vp, _sz, _vp], _i),
-    "cer_routed_ffn_workspace_size": ([_i, _i], _sz),
+    "cer_routed_ffn_workspace_size": ([_i, _i, _i, _i], _sz),
+    "cer_pack_ffn_weights": ([_vp, _vp, _vp, _i, _i, _vp, _i, _vp, _vp, _vp, _vp], _i),
     "cer_scatter_add": ([_vp, _i, _i, _i, _vp, _i, _vp, _vp], _i),
     "cer_routed_block": ([_vp, _vp, _i, _i, _i, _SCP, _SCP, _vp, _i, _i, _i, _i, _vp, _vp, _vp, _i, _vp, _i,
                           _vp, _vp, _vp, _vp, _sz, _vp, _i, _vp], _i),
-    "cer_routed_block_workspace_size": ([_i, _i, _i, _i, _i, _i, _i, _i, _i, _i], _sz),
+    "cer_routed_block_workspace_size": ([_i, _i, _i, _i, _i, _i, _i, _i, _i, _i, _i], _sz),
     "cer_sync_status": ([_vp], _i),
     "cer_get_error": ([], ctypes.c_char_p),
     "cer_status_string": ([_i], ctypes.c_char_p),
@@ -145,8 +146,8 @@ def cer_gather(h, idx, X, stream=None):
     _check(load().cer_gather(_p(h), B, N, d, _p(idx), idx.shape[1], _p(X), _stream(stream)))
 
 
-def cer_routed_ffn_workspace_size(M, C) -> int:
-    return load().cer_routed_ffn_workspace_size(M, C)
+def cer_routed_ffn_workspace_size(M, d, C, with_chan) -> int:
+    return load().cer_routed_ffn_workspace_size(M, d, C, int(bool(with_chan)))
 
 
 def cer_routed_ffn(X, Wg, Wu, WdT, chan, Y, ws=None, stream=None):
@@ -154,9 +155,23 @@ def cer_routed_ffn(X, Wg, Wu, WdT, chan, Y, ws=None, stream=None):
     I = Wg.shape[0]
     C = I if chan is None else chan.numel()
     if ws is None:
-        ws = workspace(cer_routed_ffn_workspace_size(M, C), X.device)
+        ws = workspace(cer_routed_ffn_workspace_size(M, d, C, chan is not None), X.device)
     _check(load().cer_routed_ffn(_p(X), M, d, _p(Wg), _p(Wu), _p(WdT), I, _p(chan), C, _p(Y), _p(ws), ws.numel(),
                                  _stream(stream)))
+
+
+def cer_pack_ffn_weights(Wg, Wu, WdT, chan, Wg_out, Wu_out, WdT_out, stream=None):
+    I, d = Wg.shape
+    _check(load().cer_pack_ffn_weights(_p(Wg), _p(Wu), _p(WdT), I, d, _p(chan), chan.numel(), _p(Wg_out),
+                                       _p(Wu_out), _p(WdT_out), _stream(stream)))
+
+
+def pack_ffn_weights(Wg, Wu, WdT, chan, stream=None):
+    """Kept-channel slices (new [C, d] tensors) of the three FFN weights."""
+    C, d = chan.numel(), Wg.shape[1]
+    outs = [torch.empty((C, d), dtype=Wg.dtype, device=Wg.device) for _ in range(3)]
+    cer_pack_ffn_weights(Wg, Wu, WdT, chan, *outs, stream=stream)
+    return tuple(outs)
 
 
 def cer_scatter_add(h, idx, Y, stream=None):
@@ -164,21 +179,25 @@ def cer_scatter_add(h, idx, Y, stream=None):
     _check(load().cer_scatter_add(_p(h), B, N, d, _p(idx), idx.shape[1], _p(Y), _stream(stream)))
 
 
-def cer_routed_block_workspace_size(B, N, d, core_hidden, exp_hidden, task, r0, r1, K, C) -> int:
-    return load().cer_routed_block_workspace_size(B, N, d, core_hidden, exp_hidden, task, r0, r1, K, C)
+def cer_routed_block_workspace_size(B, N, d, core_hidden, exp_hidden, task, r0, r1, K, C, with_chan) -> int:
+    return load().cer_routed_block_workspace_size(B, N, d, core_hidden, exp_hidden, task, r0, r1, K, C,
+                                                  int(bool(with_chan)))
 
 
 def cer_routed_block(h, core: Scorer, exp: Optional[Scorer], t, task, r0, r1, K, Wg, Wu, WdT, chan,
                      out=None, logits=None, idx=None, mask=None, ws=None,
                      stage_events: Optional[Sequence[torch.cuda.Event]] = None, stream=None):
-    """The fused routed block; updates h in place when ``out`` is None or h."""
+    """The fused routed block; updates h in place when ``out`` is None or h.
+
+    With ``chan`` None the weights are used as given (all their rows are the
+    channels to run: the full FFN or slices from pack_ffn_weights)."""
     B, N, d = h.shape
     I = Wg.shape[0]
     C = I if chan is None else chan.numel()
     eh = exp.W1.shape[-2] if exp is not None else 0
     if ws is None:
-        ws = workspace(cer_routed_block_workspace_size(B, N, d, core.W1.shape[-2], eh, task, r0, r1, K, C),
-                       h.device)
+        ws = workspace(cer_routed_block_workspace_size(B, N, d, core.W1.shape[-2], eh, task, r0, r1, K, C,
+                                                       chan is not None), h.device)
     ev_arr, n_ev = None, 0
     if stage_events is not None:
         handles = []

@@ -94,7 +94,7 @@ size_t round256(size_t x) { return (x + 255) & ~size_t(255); }
 #define CER_ALIGN(p) CER_REQUIRE((p) == nullptr || aligned16(p), CER_ERR_ALIGN, "%s is not 16-byte aligned", #p)
 
 struct ScoreShape {
-  int Hc = 0, He = 0, gen = 0, n_chunks = 0, Ht = 0;
+  int Hc = 0, He = 0, gen = 0, max_partials = 0, Ht = 0;
 };
 
 cer_status check_scorer(const cer_scorer* s, const char* name, bool is_core, int* hidden) {
@@ -131,16 +131,15 @@ cer_status check_score_args(const void* h, int B, int N, int d, const cer_scorer
     if (s != CER_OK) return s;
     CER_PTR_IF(t, B > 0);
   }
-  const int bn = cer::score_chunk_width(sh->Hc, sh->He, sh->gen);
-  CER_REQUIRE(bn > 0, CER_ERR_SHAPE, "scorer hidden widths must be multiples of 64");
+  sh->max_partials = cer::score_max_partials(sh->Hc, sh->He, sh->gen);
+  CER_REQUIRE(sh->max_partials > 0, CER_ERR_SHAPE, "scorer hidden widths must be multiples of 64");
   sh->Ht = sh->Hc + (sh->gen ? sh->He : 0);
-  sh->n_chunks = sh->Ht / bn;
   return CER_OK;
 }
 
 size_t score_ws_bytes(int B, int N, const ScoreShape& sh) {
   return 2 * round256(static_cast<size_t>(B) * sh.Ht * sizeof(float)) +
-         round256(static_cast<size_t>(sh.n_chunks) * B * N * sizeof(float));
+         round256(static_cast<size_t>(sh.max_partials) * B * N * sizeof(float));
 }
 
 cer::ScoreWorkspace carve_score_ws(void* ws, int B, int N, const ScoreShape& sh) {
@@ -280,10 +279,9 @@ size_t cer_score_workspace_size(int B, int N, int core_hidden, int exp_hidden, i
   sh.Hc = core_hidden;
   sh.He = exp_hidden;
   sh.gen = (task == CER_TASK_GEN);
-  const int bn = cer::score_chunk_width(sh.Hc, sh.He, sh.gen);
-  if (bn == 0 || B < 0 || N < 0) return 0;
+  sh.max_partials = cer::score_max_partials(sh.Hc, sh.He, sh.gen);
+  if (sh.max_partials == 0 || B < 0 || N < 0) return 0;
   sh.Ht = sh.Hc + (sh.gen ? sh.He : 0);
-  sh.n_chunks = sh.Ht / bn;
   return score_ws_bytes(B, N, sh);
 }
 
@@ -305,9 +303,10 @@ cer_status cer_score(const void* h, int B, int N, int d, const cer_scorer* core,
   if (B == 0 || N == 0) return CER_OK;
   cer::ScoreWorkspace ws = carve_score_ws(workspace, B, N, sh);
   cer::ScoreArgs a = make_score_args(h, B, N, d, core, exp, t, sh, dev->status);
-  cudaError_t e = cer::launch_score(a, ws, dev->n_sm, stream);
+  int n_partials = 0;
+  cudaError_t e = cer::launch_score(a, ws, dev->n_sm, stream, &n_partials);
   if (e != cudaSuccess) return cuda_fail(e, "scorer launch");
-  e = cer::launch_score_reduce(ws.partial, sh.n_chunks, static_cast<size_t>(B) * N, logits, probs, dev->n_sm,
+  e = cer::launch_score_reduce(ws.partial, n_partials, static_cast<size_t>(B) * N, logits, probs, dev->n_sm,
                                stream);
   if (e != cudaSuccess) return cuda_fail(e, "score reduce launch");
   return CER_OK;
@@ -381,10 +380,70 @@ cer_status cer_scatter_add(void* h, int B, int N, int d, const int32_t* idx, int
   return CER_OK;
 }
 
-size_t cer_routed_ffn_workspace_size(int M, int C) {
-  if (M < 0 || C < 0) return 0;
-  return round256(static_cast<size_t>(M) * C * 2);
+cer_status cer_pack_ffn_weights(const void* Wg, const void* Wu, const void* WdT, int I, int d, const int32_t* chan,
+                                int C, void* Wg_out, void* Wu_out, void* WdT_out, cudaStream_t stream) {
+  CER_PTR(Wg);
+  CER_PTR(Wu);
+  CER_PTR(WdT);
+  CER_PTR(chan);
+  CER_PTR(Wg_out);
+  CER_PTR(Wu_out);
+  CER_PTR(WdT_out);
+  CER_ALIGN(Wg);
+  CER_ALIGN(Wu);
+  CER_ALIGN(WdT);
+  CER_ALIGN(chan);
+  CER_ALIGN(Wg_out);
+  CER_ALIGN(Wu_out);
+  CER_ALIGN(WdT_out);
+  CER_REQUIRE(d > 0 && d % 8 == 0, CER_ERR_SHAPE, "d=%d must be a positive multiple of 8", d);
+  CER_REQUIRE(I >= 1 && C >= 1 && C <= I, CER_ERR_SHAPE, "C=%d must be in [1, I=%d]", C, I);
+  DeviceInfo* dev = nullptr;
+  cer_status s = device_info(&dev);
+  if (s != CER_OK) return s;
+  const void* src[3] = {Wg, Wu, WdT};
+  void* dst[3] = {Wg_out, Wu_out, WdT_out};
+  for (int i = 0; i < 3; ++i) {
+    cudaError_t e = cer::launch_gather(static_cast<const __nv_bfloat16*>(src[i]), 1, I, d, chan, C,
+                                       static_cast<__nv_bfloat16*>(dst[i]), dev->status, dev->n_sm, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "weight pack launch");
+  }
+  return CER_OK;
 }
+
+size_t cer_routed_ffn_workspace_size(int M, int d, int C, int with_chan) {
+  if (M < 0 || d < 0 || C < 0) return 0;
+  size_t ws = round256(static_cast<size_t>(M) * C * 2);
+  if (with_chan) ws += 3 * round256(static_cast<size_t>(C) * d * 2);
+  return ws;
+}
+
+namespace {
+
+// Kept-channel slices of the FFN weights: the given arrays when chan is NULL
+// (they already hold exactly C channels), else packed into `ws`.
+cer_status ffn_weight_slices(const void* Wg, const void* Wu, const void* WdT, int I, int d, const int32_t* chan,
+                             int C, char** ws, const __nv_bfloat16* out[3], DeviceInfo* dev, cudaStream_t stream) {
+  if (chan == nullptr) {
+    out[0] = static_cast<const __nv_bfloat16*>(Wg);
+    out[1] = static_cast<const __nv_bfloat16*>(Wu);
+    out[2] = static_cast<const __nv_bfloat16*>(WdT);
+    return CER_OK;
+  }
+  const void* src[3] = {Wg, Wu, WdT};
+  const size_t slice = round256(static_cast<size_t>(C) * d * 2);
+  for (int i = 0; i < 3; ++i) {
+    __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(*ws);
+    *ws += slice;
+    cudaError_t e = cer::launch_gather(static_cast<const __nv_bfloat16*>(src[i]), 1, I, d, chan, C, dst, dev->status,
+                                       dev->n_sm, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "weight pack launch");
+    out[i] = dst;
+  }
+  return CER_OK;
+}
+
+}  // namespace
 
 cer_status cer_routed_ffn(const void* X, int M, int d, const void* Wg, const void* Wu, const void* WdT, int I,
                           const int32_t* chan, int C, void* Y, void* workspace, size_t workspace_bytes,
@@ -403,25 +462,25 @@ cer_status cer_routed_ffn(const void* X, int M, int d, const void* Wg, const voi
   CER_ALIGN(workspace);
   cer_status s = check_ffn_shape(M, d, I, chan, C);
   if (s != CER_OK) return s;
-  const size_t need = cer_routed_ffn_workspace_size(M, C);
+  const size_t need = cer_routed_ffn_workspace_size(M, d, C, chan != nullptr);
   CER_REQUIRE(M == 0 || (workspace != nullptr && workspace_bytes >= need), CER_ERR_WORKSPACE,
               "workspace of %zu bytes needed, %zu given", need, workspace_bytes);
   DeviceInfo* dev = nullptr;
   if ((s = device_info(&dev)) != CER_OK) return s;
   if (M == 0) return CER_OK;
+  char* ws = static_cast<char*>(workspace);
   cer::FfnArgs a{};
+  a.act = reinterpret_cast<__nv_bfloat16*>(ws);
+  ws += round256(static_cast<size_t>(M) * C * 2);
+  const __nv_bfloat16* w[3];
+  if ((s = ffn_weight_slices(Wg, Wu, WdT, I, d, chan, C, &ws, w, dev, stream)) != CER_OK) return s;
   a.X = static_cast<const __nv_bfloat16*>(X);
   a.M = M;
   a.d = d;
-  a.I = I;
   a.C = C;
-  a.N = 0;
-  a.k_tot = 1;
-  a.Wg = static_cast<const __nv_bfloat16*>(Wg);
-  a.Wu = static_cast<const __nv_bfloat16*>(Wu);
-  a.WdT = static_cast<const __nv_bfloat16*>(WdT);
-  a.chan = chan;
-  a.act = static_cast<__nv_bfloat16*>(workspace);
+  a.Wg = w[0];
+  a.Wu = w[1];
+  a.WdT = w[2];
   a.Y = static_cast<__nv_bfloat16*>(Y);
   a.scatter = 0;
   a.status = dev->status;
@@ -433,14 +492,14 @@ cer_status cer_routed_ffn(const void* X, int M, int d, const void* Wg, const voi
 }
 
 size_t cer_routed_block_workspace_size(int B, int N, int d, int core_hidden, int exp_hidden, int task, int r0,
-                                       int r1, int K, int C) {
-  (void)d;
+                                       int r1, int K, int C, int with_chan) {
   const size_t sc = cer_score_workspace_size(B, N, core_hidden, exp_hidden, task);
-  if (sc == 0 && B > 0 && N > 0) return 0;
-  if (B < 0 || N < 0 || r0 < 0 || r1 < r0 || r1 > N || K < 0 || K > r1 - r0 || C < 0) return 0;
+  if (sc == 0) return 0;
+  if (B < 0 || N < 0 || d < 0 || r0 < 0 || r1 < r0 || r1 > N || K < 0 || K > r1 - r0 || C < 0) return 0;
   const size_t k_tot = static_cast<size_t>(K) + (N - (r1 - r0));
   const size_t M = static_cast<size_t>(B) * k_tot;
-  return sc + round256(M * sizeof(int32_t)) + round256(M * C * 2);
+  return sc + round256(M * sizeof(int32_t)) + round256(M * d * 2) + cer_routed_ffn_workspace_size(
+                                                                          static_cast<int>(M), d, C, with_chan);
 }
 
 cer_status cer_routed_block(void* h, void* out, int B, int N, int d, const cer_scorer* core, const cer_scorer* exp,
@@ -468,11 +527,13 @@ cer_status cer_routed_block(void* h, void* out, int B, int N, int d, const cer_s
   CER_REQUIRE(0 <= K && K <= r1 - r0, CER_ERR_RANGE, "K=%d not in [0, N_r=%d]", K, r1 - r0);
   const int k_tot = K + N - (r1 - r0);
   const long long M64 = static_cast<long long>(B) * k_tot;
+  CER_REQUIRE(M64 < (1ll << 31), CER_ERR_SHAPE, "too many kept rows");
   s = check_ffn_shape(static_cast<int>(M64), d, I, chan, C);
   if (s != CER_OK) return s;
-  CER_REQUIRE(stage_events == nullptr || n_stage_events == 5, CER_ERR_RANGE,
-              "stage_events needs exactly 5 events (got %d)", n_stage_events);
-  const size_t need = cer_routed_block_workspace_size(B, N, d, sh.Hc, sh.He, task, r0, r1, K, C);
+  CER_REQUIRE(stage_events == nullptr || n_stage_events == 6, CER_ERR_RANGE,
+              "stage_events needs exactly 6 events (got %d)", n_stage_events);
+  const size_t need =
+      cer_routed_block_workspace_size(B, N, d, sh.Hc, sh.He, task, r0, r1, K, C, chan != nullptr);
   CER_REQUIRE(workspace != nullptr && workspace_bytes >= need, CER_ERR_WORKSPACE,
               "workspace of %zu bytes needed, %zu given", need, workspace_bytes);
   const bool in_place = (out == nullptr || out == h);
@@ -496,7 +557,7 @@ cer_status cer_routed_block(void* h, void* out, int B, int N, int d, const cer_s
     if (e != cudaSuccess) return cuda_fail(e, "bypass copy");
   }
   if (B == 0 || N == 0) {
-    for (int i = 1; i < 5; ++i) mark(i);
+    for (int i = 1; i < 6; ++i) mark(i);
     return CER_OK;
   }
   char* ws = static_cast<char*>(workspace);
@@ -504,18 +565,22 @@ cer_status cer_routed_block(void* h, void* out, int B, int N, int d, const cer_s
   ws += score_ws_bytes(B, N, sh);
   int32_t* idx_buf = idx ? idx : reinterpret_cast<int32_t*>(ws);
   ws += round256(static_cast<size_t>(M64) * sizeof(int32_t));
+  __nv_bfloat16* X = reinterpret_cast<__nv_bfloat16*>(ws);
+  ws += round256(static_cast<size_t>(M64) * d * 2);
   __nv_bfloat16* act = reinterpret_cast<__nv_bfloat16*>(ws);
+  ws += round256(static_cast<size_t>(M64) * C * 2);
 
   // S1: scorer GEMM -> partial sums
   cer::ScoreArgs sa = make_score_args(h, B, N, d, core, exp, t, sh, dev->status);
-  e = cer::launch_score(sa, sws, dev->n_sm, stream);
+  int n_partials = 0;
+  e = cer::launch_score(sa, sws, dev->n_sm, stream, &n_partials);
   if (e != cudaSuccess) return cuda_fail(e, "scorer launch");
   if ((e = mark(1)) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
 
   // S2: reduce partial sums + top-K keep list
   cer::TopkArgs ta{};
   ta.src = sws.partial;
-  ta.n_chunks = sh.n_chunks;
+  ta.n_chunks = n_partials;
   ta.chunk_stride = static_cast<size_t>(B) * N;
   ta.B = B;
   ta.N = N;
@@ -530,36 +595,43 @@ cer_status cer_routed_block(void* h, void* out, int B, int N, int d, const cer_s
   if (e != cudaSuccess) return cuda_fail(e, "top-K launch");
   if ((e = mark(2)) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
 
-  // S3+S4: gate/up GEMM on the kept rows of h (row gathers)
+  // S3: pack the kept rows (and, if a channel list is given, the kept weight rows)
+  const __nv_bfloat16* w[3];
+  if ((s = ffn_weight_slices(Wg, Wu, WdT, I, d, chan, C, &ws, w, dev, stream)) != CER_OK) return s;
+  e = cer::launch_gather(static_cast<const __nv_bfloat16*>(h), B, N, d, idx_buf, k_tot, X, dev->status, dev->n_sm,
+                         stream);
+  if (e != cudaSuccess) return cuda_fail(e, "gather launch");
+  if ((e = mark(3)) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+
+  // S4: gate/up GEMM with the SwiGLU epilogue
   cer::FfnArgs fa{};
+  fa.X = X;
+  fa.M = static_cast<int>(M64);
+  fa.d = d;
+  fa.C = C;
+  fa.Wg = w[0];
+  fa.Wu = w[1];
+  fa.WdT = w[2];
+  fa.act = act;
   fa.h = static_cast<const __nv_bfloat16*>(h);
+  fa.out = static_cast<__nv_bfloat16*>(dst);
   fa.idx = idx_buf;
   fa.N = N;
   fa.k_tot = k_tot;
-  fa.M = static_cast<int>(M64);
-  fa.d = d;
-  fa.I = I;
-  fa.C = C;
-  fa.Wg = static_cast<const __nv_bfloat16*>(Wg);
-  fa.Wu = static_cast<const __nv_bfloat16*>(Wu);
-  fa.WdT = static_cast<const __nv_bfloat16*>(WdT);
-  fa.chan = chan;
-  fa.act = act;
-  fa.out = static_cast<__nv_bfloat16*>(dst);
   fa.scatter = 1;
   fa.status = dev->status;
   if (M64 > 0) {
     e = cer::launch_ffn_gateup(fa, dev->n_sm, stream);
     if (e != cudaSuccess) return cuda_fail(e, "gate/up GEMM launch");
   }
-  if ((e = mark(3)) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+  if ((e = mark(4)) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
 
-  // S4+S5: down GEMM with the unpack fused into its epilogue
+  // S4+S5: down GEMM with the unpack (scatter-add into the residual) fused
   if (M64 > 0) {
     e = cer::launch_ffn_down(fa, dev->n_sm, stream);
     if (e != cudaSuccess) return cuda_fail(e, "down GEMM launch");
   }
-  if ((e = mark(4)) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+  if ((e = mark(5)) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
   return CER_OK;
 }
 

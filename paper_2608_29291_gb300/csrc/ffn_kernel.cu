@@ -1,17 +1,20 @@
-// ffn_kernel.cu -- S4 (+S3/S5 fused): the channel-pruned SwiGLU FFN on the
+// ffn_kernel.cu -- S4 (+S5 fused): the channel-pruned SwiGLU FFN on the
 // packed rows (Sec. 3.4 compaction and FFN pruning; SwiGLU of the Qwen2.5
-// backbone, App. A.5), as two tcgen05 GEMMs.
+// backbone, App. A.5), as two tcgen05 GEMMs over dense operands.
 //
-// gate/up:  act[m, c] = SiLU(Wg[Cs[c]] . x_m) * (Wu[Cs[c]] . x_m)
-//   A = packed rows (TMA tile of X) or, fused, rows of h picked by the keep
-//   list (TMA 4-row gathers, one per lane); B = 128 gate rows followed by the
-//   same 128 up rows of the kept channels, gathered straight from the full
-//   weights.  One 128x256 MMA tile yields gate and up for 128 channels, so the
-//   SwiGLU runs in the epilogue and act is written once, as bf16.
-// down:     y[m, n] = sum_c act[m, c] * WdT[Cs[c], n]
-//   A = act tile; B = MN-major tile of 64 kept channel rows of WdT x 256
-//   output columns (row gathers).  Epilogue: Y = bf16(y), or, fused, the
-//   unpack out[b, idx[m], n] = bf16(h[b, idx[m], n] + y) -- the kept rows are
+// The kept rows X [M, d] and the kept-channel weight slices Wg, Wu, WdT
+// [C, d] arrive packed (row gathers run as separate HBM-bound copies: TMA
+// 4-row gathers inside the GEMM producer measured 2.4x slower), so every
+// operand tile is one TMA box.
+//
+// gate/up:  act[m, c] = SiLU(Wg[c] . x_m) * (Wu[c] . x_m)
+//   One 128x256 MMA tile holds gate (columns 0..127) and up (128..255) for
+//   the same 128 channels, so the SwiGLU runs in the epilogue and act is
+//   written once, as bf16.
+// down:     y[m, n] = sum_c act[m, c] * WdT[c, n]
+//   B is MN-major: 64 channel rows x 256 output columns, four 64-column TMA
+//   boxes per K block.  Epilogue: Y = bf16(y), or, fused, the unpack
+//   out[b, idx[m], n] = bf16(h[b, idx[m], n] + y) -- the kept rows are
 //   distinct, so no atomics; dropped rows are never touched.
 #include <cuda_bf16.h>
 
@@ -20,14 +23,11 @@
 
 namespace cer {
 
-__device__ __forceinline__ float silu_mul(float g, float u) { return g / (1.0f + expf(-g)) * u; }
-
-__device__ __forceinline__ int checked_index(int v, int limit, int* status) {
-  if (v < 0 || v >= limit) {
-    record_status(status, CER_DEV_INDEX);
-    return 0;
-  }
-  return v;
+// SiLU(g) * u with the fast exponential and division: the result is rounded
+// to bf16 (8 significant bits), far coarser than their error.  The exponent
+// argument is clamped so 1 + e^-g stays finite (SiLU(g) ~ 0 there anyway).
+__device__ __forceinline__ float silu_mul(float g, float u) {
+  return __fdividef(g * u, 1.0f + __expf(fminf(-g, 80.0f)));
 }
 
 // ---------------------------------------------------------------- gate/up
@@ -39,62 +39,41 @@ struct GateUpProblem {
   static constexpr uint32_t kBStepBytes = 32;
 
   struct Params {
-    CUtensorMap tm_a;   // gather: h as [B*N, d], box 64 x 1; packed: X [M, d], box 64 x 128
-    CUtensorMap tm_wg;  // Wg [I, d], box 64 x 1
-    CUtensorMap tm_wu;  // Wu [I, d], box 64 x 1
-    const int32_t* idx;
-    const int32_t* chan;
+    CUtensorMap tm_x;   // X [M, d], box 64 x 128
+    CUtensorMap tm_wg;  // Wg [C, d], box 64 x 128
+    CUtensorMap tm_wu;  // Wu [C, d], box 64 x 128
     __nv_bfloat16* act;
     int* status;
-    int M, d, C, I, N, k_tot, n_mt, n_ct;
+    int M, d, C, n_mt, n_ct;
   };
   struct ProdState {
-    int rows[4];
-    int chs[4];
-    int mt;
+    int m0, c0;
   };
 
   __device__ static int num_tiles(const Params& p) { return p.n_mt * p.n_ct; }
   __device__ static int num_kb(const Params& p) { return p.d / 64; }
   __device__ static uint32_t stage_bytes(const Params&, int, int) { return kATileBytes + BN * 128; }
-
-  __device__ static void prod_tile(const Params& p, int tile, int lane, ProdState& st) {
-    const int ct = tile / p.n_mt;
-    st.mt = tile % p.n_mt;
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const int r = 4 * lane + i;
-      if (p.idx != nullptr) {
-        const int m = min(st.mt * 128 + r, p.M - 1);
-        const int tok = checked_index(__ldg(p.idx + m), p.N, p.status);
-        st.rows[i] = (m / p.k_tot) * p.N + tok;
-      }
-      const int c = min(ct * 128 + r, p.C - 1);
-      st.chs[i] = checked_index(p.chan ? __ldg(p.chan + c) : c, p.I, p.status);
-    }
+  __device__ static void prod_tile(const Params& p, int tile, int, ProdState& st) {
+    st.c0 = (tile / p.n_mt) * 128;
+    st.m0 = (tile % p.n_mt) * 128;
   }
-
   __device__ static void prod_kb(const Params& p, const ProdState& st, int, int kb, int lane, uint8_t* a,
                                  uint8_t* b, uint64_t* bar) {
-    const int x = kb * 64;
-    if (p.idx != nullptr) {
-      tma_gather4(a + lane * 512, &p.tm_a, bar, x, st.rows[0], st.rows[1], st.rows[2], st.rows[3]);
-    } else if (lane == 0) {
-      tma_load_2d(a, &p.tm_a, bar, x, st.mt * 128);
+    if (lane == 0) {
+      const int x = kb * 64;
+      tma_load_2d(a, &p.tm_x, bar, x, st.m0);
+      tma_load_2d(b, &p.tm_wg, bar, x, st.c0);
+      tma_load_2d(b + 128 * 128, &p.tm_wu, bar, x, st.c0);
     }
-    tma_gather4(b + lane * 512, &p.tm_wg, bar, x, st.chs[0], st.chs[1], st.chs[2], st.chs[3]);
-    tma_gather4(b + 128 * 128 + lane * 512, &p.tm_wu, bar, x, st.chs[0], st.chs[1], st.chs[2], st.chs[3]);
   }
-
   __device__ static uint64_t bdesc(uint32_t saddr) { return sdesc_kmajor_sw128(saddr); }
 
-  __device__ static void epilogue(const Params& p, int tile, int row, uint32_t taddr) {
+  __device__ static void epilogue(const Params& p, int tile, int row, int half, uint32_t taddr) {
     const int ct = tile / p.n_mt;
-    const int mt = tile % p.n_mt;
-    const int m = mt * 128 + row;
+    const int m = (tile % p.n_mt) * 128 + row;
     const bool valid = m < p.M;
 #pragma unroll 1
-    for (int c = 0; c < 4; ++c) {
+    for (int c = 2 * half; c < 2 * half + 2; ++c) {
       float g[32], u[32];
       tmem_ld2_32x32(taddr + c * 32, taddr + 128 + c * 32, g, u);
       const int ch0 = ct * 128 + c * 32;
@@ -116,22 +95,21 @@ struct DownProblem {
   static constexpr int BN = 256;
   static constexpr int STAGES = 4;
   static constexpr int B_MN_MAJOR = 1;
-  static constexpr uint32_t kBStepBytes = 2048;   // 16 K-rows = two 1024 B row groups
+  static constexpr uint32_t kBStepBytes = 2048;     // 16 K-rows = two 1024 B row groups
   static constexpr uint32_t kAtomBytes = 64 * 128;  // 64 K-rows x 64 columns
 
   struct Params {
     CUtensorMap tm_act;  // act [M, C], box 64 x 128
-    CUtensorMap tm_wdt;  // WdT [I, d], box 64 x 1
-    const int32_t* chan;
+    CUtensorMap tm_wdt;  // WdT [C, d], box 64 x 64
     const int32_t* idx;          // scatter mode: keep list [B][k_tot]
     const __nv_bfloat16* hin;    // scatter mode: residual input
     __nv_bfloat16* out;          // Y [M, d] or the residual output
     int* status;
     int scatter;
-    int M, d, C, I, N, k_tot, n_mt, n_nt;
+    int M, d, C, N, k_tot, n_mt, n_nt;
   };
   struct ProdState {
-    int mt, nt, n_atoms;
+    int m0, n0, n_atoms;
   };
 
   __device__ static int num_tiles(const Params& p) { return p.n_mt * p.n_nt; }
@@ -144,38 +122,23 @@ struct DownProblem {
     return kATileBytes + atoms(p, tile / p.n_mt) * kAtomBytes;
   }
   __device__ static void prod_tile(const Params& p, int tile, int, ProdState& st) {
-    st.nt = tile / p.n_mt;
-    st.mt = tile % p.n_mt;
-    st.n_atoms = atoms(p, st.nt);
+    const int nt = tile / p.n_mt;
+    st.n0 = nt * 256;
+    st.m0 = (tile % p.n_mt) * 128;
+    st.n_atoms = atoms(p, nt);
   }
   __device__ static void prod_kb(const Params& p, const ProdState& st, int, int kb, int lane, uint8_t* a,
                                  uint8_t* b, uint64_t* bar) {
-    if (lane == 0) tma_load_2d(a, &p.tm_act, bar, kb * 64, st.mt * 128);
-    const int g = lane & 15;
-    const int c0 = kb * 64 + 4 * g;
-    int ch[4];
-    if (p.chan != nullptr) {
-      const int4 v = __ldg(reinterpret_cast<const int4*>(p.chan + c0));
-      ch[0] = v.x; ch[1] = v.y; ch[2] = v.z; ch[3] = v.w;
-    } else {
-      ch[0] = c0; ch[1] = c0 + 1; ch[2] = c0 + 2; ch[3] = c0 + 3;
-    }
-#pragma unroll
-    for (int i = 0; i < 4; ++i) ch[i] = checked_index(ch[i], p.I, p.status);
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      const int at = 2 * (lane >> 4) + h;
-      if (at < st.n_atoms)
-        tma_gather4(b + at * kAtomBytes + g * 512, &p.tm_wdt, bar, st.nt * 256 + at * 64, ch[0], ch[1], ch[2], ch[3]);
+    if (lane == 0) {
+      tma_load_2d(a, &p.tm_act, bar, kb * 64, st.m0);
+      for (int at = 0; at < st.n_atoms; ++at) tma_load_2d(b + at * kAtomBytes, &p.tm_wdt, bar, st.n0 + at * 64, kb * 64);
     }
   }
-
   __device__ static uint64_t bdesc(uint32_t saddr) { return sdesc_mnmajor_sw128(saddr, kAtomBytes, 1024); }
 
-  __device__ static void epilogue(const Params& p, int tile, int row, uint32_t taddr) {
+  __device__ static void epilogue(const Params& p, int tile, int row, int half, uint32_t taddr) {
     const int nt = tile / p.n_mt;
-    const int mt = tile % p.n_mt;
-    const int m = mt * 128 + row;
+    const int m = (tile % p.n_mt) * 128 + row;
     bool valid = m < p.M;
     size_t dst_row = 0;
     if (valid) {
@@ -191,7 +154,7 @@ struct DownProblem {
       }
     }
 #pragma unroll 1
-    for (int c = 0; c < 8; ++c) {
+    for (int c = 4 * half; c < 4 * half + 4; ++c) {
       float v[32];
       tmem_ld_32x32(taddr + c * 32, v);
       const int n0 = nt * 256 + c * 32;
@@ -236,24 +199,14 @@ static cudaError_t launch_gemm(const typename P::Params& p, int tiles, int n_sm,
 
 cudaError_t launch_ffn_gateup(const FfnArgs& a, int n_sm, cudaStream_t stream) {
   GateUpProblem::Params p{};
-  if (a.idx != nullptr) {
-    if (!encode_bf16_2d(&p.tm_a, a.h, static_cast<uint64_t>(a.M / a.k_tot) * a.N, a.d, 64, 1))
-      return cudaErrorInvalidValue;
-  } else {
-    if (!encode_bf16_2d(&p.tm_a, a.X, a.M, a.d, 64, 128)) return cudaErrorInvalidValue;
-  }
-  if (!encode_bf16_2d(&p.tm_wg, a.Wg, a.I, a.d, 64, 1)) return cudaErrorInvalidValue;
-  if (!encode_bf16_2d(&p.tm_wu, a.Wu, a.I, a.d, 64, 1)) return cudaErrorInvalidValue;
-  p.idx = a.idx;
-  p.chan = a.chan;
+  if (!encode_bf16_2d(&p.tm_x, a.X, a.M, a.d, 64, 128)) return cudaErrorInvalidValue;
+  if (!encode_bf16_2d(&p.tm_wg, a.Wg, a.C, a.d, 64, 128)) return cudaErrorInvalidValue;
+  if (!encode_bf16_2d(&p.tm_wu, a.Wu, a.C, a.d, 64, 128)) return cudaErrorInvalidValue;
   p.act = a.act;
   p.status = a.status;
   p.M = a.M;
   p.d = a.d;
   p.C = a.C;
-  p.I = a.I;
-  p.N = a.N;
-  p.k_tot = a.k_tot;
   p.n_mt = (a.M + 127) / 128;
   p.n_ct = (a.C + 127) / 128;
   return launch_gemm<GateUpProblem>(p, p.n_mt * p.n_ct, n_sm, stream);
@@ -262,8 +215,7 @@ cudaError_t launch_ffn_gateup(const FfnArgs& a, int n_sm, cudaStream_t stream) {
 cudaError_t launch_ffn_down(const FfnArgs& a, int n_sm, cudaStream_t stream) {
   DownProblem::Params p{};
   if (!encode_bf16_2d(&p.tm_act, a.act, a.M, a.C, 64, 128)) return cudaErrorInvalidValue;
-  if (!encode_bf16_2d(&p.tm_wdt, a.WdT, a.I, a.d, 64, 1)) return cudaErrorInvalidValue;
-  p.chan = a.chan;
+  if (!encode_bf16_2d(&p.tm_wdt, a.WdT, a.C, a.d, 64, 64)) return cudaErrorInvalidValue;
   p.idx = a.idx;
   p.hin = a.h;
   p.out = a.scatter ? a.out : a.Y;
@@ -272,7 +224,6 @@ cudaError_t launch_ffn_down(const FfnArgs& a, int n_sm, cudaStream_t stream) {
   p.M = a.M;
   p.d = a.d;
   p.C = a.C;
-  p.I = a.I;
   p.N = a.N;
   p.k_tot = a.k_tot;
   p.n_mt = (a.M + 127) / 128;

@@ -40,11 +40,17 @@ struct ScoreArgs {
 struct ScoreWorkspace {
   float* bias_tab;  // [B][Hc + He]
   float* w2_tab;    // [B][Hc + He]
-  float* partial;   // [n_chunks][B*N]
+  float* partial;   // [n_partials][B*N], n_partials <= 2 * (Hc + He) / 64
 };
 
+// Largest hidden-chunk width the scorer may use for these widths (0: none).
 int score_chunk_width(int Hc, int He, int gen);
-cudaError_t launch_score(const ScoreArgs& a, const ScoreWorkspace& ws, int n_sm, cudaStream_t stream);
+// Upper bound of the partial-score rows the scorer writes.
+int score_max_partials(int Hc, int He, int gen);
+// Launches the bias-table and scorer kernels; *n_partials receives the number
+// of partial-score rows written (to be summed in order by the consumer).
+cudaError_t launch_score(const ScoreArgs& a, const ScoreWorkspace& ws, int n_sm, cudaStream_t stream,
+                         int* n_partials);
 cudaError_t launch_score_reduce(const float* partial, int n_chunks, size_t total, float* logits, float* probs,
                                 int n_sm, cudaStream_t stream);
 
@@ -71,21 +77,18 @@ cudaError_t launch_scatter_add(__nv_bfloat16* h, int B, int N, int d, const int3
 
 // ------------------------------------------------------------------ S4 FFN
 struct FfnArgs {
-  // A operand of the gate/up GEMM: either packed rows X [M, d] (idx == nullptr)
-  // or the kept rows of h [B, N, d] selected by idx [B][k_tot].
-  const __nv_bfloat16* X;
-  const __nv_bfloat16* h;
-  const int32_t* idx;
-  int N, k_tot;
-  int M, d, I, C;
-  const __nv_bfloat16* Wg;
+  const __nv_bfloat16* X;     // packed kept rows [M, d]
+  int M, d, C;
+  const __nv_bfloat16* Wg;    // kept-channel slices [C, d]
   const __nv_bfloat16* Wu;
   const __nv_bfloat16* WdT;
-  const int32_t* chan;   // nullable: all channels
-  __nv_bfloat16* act;    // workspace [M, C]
+  __nv_bfloat16* act;         // workspace [M, C]
   // Output: Y [M, d] (scatter == 0) or out[b, idx] = bf16(h + y) (scatter == 1).
   __nv_bfloat16* Y;
+  const __nv_bfloat16* h;
   __nv_bfloat16* out;
+  const int32_t* idx;
+  int N, k_tot;
   int scatter;
   int* status;
 };

@@ -6,7 +6,8 @@
 // chunks.  A work tile is (sequence b, 128-token row tile, hidden chunk); its
 // epilogue adds the per-sequence bias column (b1, or U emb(t_b) + b1e for the
 // expansion), applies the exact-erf GELU in fp32 and folds the chunk into a
-// per-token partial score w2 . GELU(.), written to partial[chunk][b*N + n].
+// per-token partial score w2 . GELU(.); each half of the chunk's columns
+// (one per group of four epilogue warps) writes partial[2*chunk + half][b*N + n].
 // The partial scores are summed in chunk order by the consumer (the reduce
 // kernel below, or the top-K kernel in the fused block), so the logits do not
 // depend on scheduling.
@@ -126,21 +127,21 @@ struct ScoreProblem {
   }
   __device__ static uint64_t bdesc(uint32_t saddr) { return sdesc_kmajor_sw128(saddr); }
 
-  __device__ static void epilogue(const Params& p, int tile, int row, uint32_t taddr) {
+  __device__ static void epilogue(const Params& p, int tile, int row, int half, uint32_t taddr) {
     int b, rt, chunk;
     decode(p, tile, b, rt, chunk);
     const float* bias = p.bias_tab + static_cast<size_t>(b) * p.Ht + chunk * BN;
     const float* w2 = p.w2_tab + static_cast<size_t>(b) * p.Ht + chunk * BN;
     float s = 0.f;
 #pragma unroll 1
-    for (int c = 0; c < BN / 32; ++c) {
+    for (int c = half * (BN / 64); c < (half + 1) * (BN / 64); ++c) {
       float v[32];
       tmem_ld_32x32(taddr + c * 32, v);
 #pragma unroll
       for (int j = 0; j < 32; ++j) s = fmaf(__ldg(w2 + c * 32 + j), gelu_erf(v[j] + __ldg(bias + c * 32 + j)), s);
     }
     const int n = rt * 128 + row;
-    if (n < p.N) p.partial[static_cast<size_t>(chunk) * p.B * p.N + static_cast<size_t>(b) * p.N + n] = s;
+    if (n < p.N) p.partial[static_cast<size_t>(2 * chunk + half) * p.B * p.N + static_cast<size_t>(b) * p.N + n] = s;
   }
 };
 
@@ -164,6 +165,25 @@ int score_chunk_width(int Hc, int He, int gen) {
     if (Hc % bn == 0 && (!gen || He % bn == 0)) return bn;
   }
   return 0;
+}
+
+int score_max_partials(int Hc, int He, int gen) {
+  if (score_chunk_width(Hc, He, gen) == 0) return 0;
+  return 2 * (Hc + (gen ? He : 0)) / 64;
+}
+
+// Chunk width for a launch: the widest that still gives every SM a tile,
+// else the narrowest available (more, smaller tiles).
+static int pick_chunk_width(const ScoreArgs& a, int n_sm) {
+  const int Ht = a.Hc + (a.gen ? a.He : 0);
+  const long rows = static_cast<long>(a.B) * ((a.N + 127) / 128);
+  int best = 0;
+  for (int bn : {256, 128, 64}) {
+    if (a.Hc % bn != 0 || (a.gen && a.He % bn != 0)) continue;
+    best = bn;
+    if (rows * (Ht / bn) >= n_sm) return bn;
+  }
+  return best;
 }
 
 template <int BN>
@@ -204,12 +224,15 @@ static cudaError_t launch_score_gemm(const ScoreArgs& a, const float* bias_tab, 
   return cudaGetLastError();
 }
 
-cudaError_t launch_score(const ScoreArgs& a, const ScoreWorkspace& ws, int n_sm, cudaStream_t stream) {
+cudaError_t launch_score(const ScoreArgs& a, const ScoreWorkspace& ws, int n_sm, cudaStream_t stream,
+                         int* n_partials) {
   const int emb_bytes = (a.gen && a.U) ? a.E * static_cast<int>(sizeof(float)) : 0;
   time_bias_kernel<<<a.B, 256, emb_bytes, stream>>>(a, ws.bias_tab, ws.w2_tab);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  switch (score_chunk_width(a.Hc, a.He, a.gen)) {
+  const int bn = pick_chunk_width(a, n_sm);
+  *n_partials = bn ? 2 * (a.Hc + (a.gen ? a.He : 0)) / bn : 0;
+  switch (bn) {
     case 256: return launch_score_gemm<256>(a, ws.bias_tab, ws.w2_tab, ws.partial, n_sm, stream);
     case 128: return launch_score_gemm<128>(a, ws.bias_tab, ws.w2_tab, ws.partial, n_sm, stream);
     case 64: return launch_score_gemm<64>(a, ws.bias_tab, ws.w2_tab, ws.partial, n_sm, stream);

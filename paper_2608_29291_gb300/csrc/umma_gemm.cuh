@@ -1,15 +1,16 @@
 // umma_gemm.cuh -- persistent, warp-specialised tcgen05 GEMM skeleton for
 // sm_103a, shared by the scorer and the two FFN contractions.
 //
-// One CTA per SM (192 threads, ~193 KB shared memory, 2*BN TMEM columns):
-//   warp 0     producer: TMA loads (tiled or 4-row gathers) of the A tile
-//              (128 rows x 64 bf16) and the B tile (BN rows x 64 bf16, or
-//              64 K-rows x BN for an MN-major B) into a STAGES-deep ring;
+// One CTA per SM (320 threads, ~193 KB shared memory, 2*BN TMEM columns):
+//   warp 0     producer: TMA box loads of the A tile (128 rows x 64 bf16)
+//              and the B tile (BN rows x 64 bf16, or 64 K-rows x BN for an
+//              MN-major B) into a STAGES-deep ring;
 //   warp 1     allocates TMEM, one elected lane issues tcgen05.mma
 //              (M=128, N=BN, K=16) four times per 64-wide K block and
 //              commits the ring slot back to the producer;
-//   warps 2-5  epilogue: read the fp32 accumulator out of TMEM (lane = tile
-//              row) and apply the problem's fused epilogue.
+//   warps 2-9  epilogue: read the fp32 accumulator out of TMEM (lane = tile
+//              row; warps 2-5 take the first half of the columns, warps 6-9
+//              the second) and apply the problem's fused epilogue.
 // The accumulator is double-buffered in TMEM so the epilogue of tile i
 // overlaps the MMAs of tile i+1.  Tiles are visited with a stride of
 // gridDim.x.  Every wait is bounded (ptx.cuh); on a timeout the CTA unwinds,
@@ -19,14 +20,17 @@
 //   BN, STAGES, B_MN_MAJOR, kBStepBytes, Params (with `int* status`),
 //   num_tiles(p), num_kb(p), prod_tile(p, tile, lane, state),
 //   prod_kb(p, state, tile, kb, lane, a_smem, b_smem, bar),
-//   stage_bytes(p, tile, kb), bdesc(saddr), epilogue(p, tile, row, taddr).
+//   stage_bytes(p, tile, kb), bdesc(saddr),
+//   epilogue(p, tile, row, half, taddr): columns [half*BN/2, (half+1)*BN/2)
+//   of accumulator row `row`, taddr addressing column 0 of that row's lanes.
 #pragma once
 
 #include "ptx.cuh"
 
 namespace cer {
 
-constexpr int kGemmThreads = 192;
+constexpr int kEpiWarps = 8;
+constexpr int kGemmThreads = 64 + 32 * kEpiWarps;
 constexpr uint32_t kATileBytes = 128 * 128;  // 128 rows x 64 bf16
 
 template <int BN>
@@ -88,7 +92,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) umma_gemm_kernel(const __grid
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull[a], 1);
-      mbar_init(&tempty[a], 128);
+      mbar_init(&tempty[a], 32 * kEpiWarps);
     }
     mbar_init(drain, 1);
     *abort_flag = 0;
@@ -190,13 +194,14 @@ __global__ void __launch_bounds__(kGemmThreads, 1) umma_gemm_kernel(const __grid
     // ---------------------------------------------------------------- epilogue
     const int q = warp & 3;            // TMEM lane quadrant this warp may access
     const int row = q * 32 + lane;     // accumulator row = TMEM lane
+    const int half = (warp - 2) >> 2;  // which half of the accumulator columns
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
       if (!warp_wait(&tfull[acc], acc_phase, abort_flag, p.status)) break;
       tc_fence_after();
       const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BN);
-      P::epilogue(p, tile, row, taddr);
+      P::epilogue(p, tile, row, half, taddr);
       tc_fence_before();
       mbar_arrive(&tempty[acc]);
       if (++acc == 2) {

@@ -41,17 +41,25 @@ def test_library_exports_every_declared_symbol(lib):
         assert lib.cer_status_string(code).decode() == name
 
 
+def _r256(x):
+    return (x + 255) // 256 * 256
+
+
 def test_workspace_sizes(lib):
-    # scorer: bias + w2 tables [B][Ht] and partial sums [chunks][B*N], 256-byte rounded
-    assert lib.cer_score_workspace_size(4, 1024, 256, 0, 0) == 2 * 4096 + 1 * 4 * 1024 * 4
-    assert lib.cer_score_workspace_size(2, 4096, 512, 512, 1) == 2 * 8192 + 4 * 2 * 4096 * 4
-    assert lib.cer_score_workspace_size(1, 256, 64, 64, 1) == 2 * 512 + 2 * 256 * 4
+    # scorer: bias + w2 tables [B][Ht] and at most 2*Ht/64 partial-score rows of B*N
+    assert lib.cer_score_workspace_size(4, 1024, 256, 0, 0) == 2 * 4096 + 8 * 4 * 1024 * 4
+    assert lib.cer_score_workspace_size(2, 4096, 512, 512, 1) == 2 * 8192 + 32 * 2 * 4096 * 4
+    assert lib.cer_score_workspace_size(1, 256, 64, 64, 1) == 2 * 512 + 4 * 256 * 4
     assert lib.cer_score_workspace_size(1, 10, 100, 0, 0) == 0          # hidden not a multiple of 64
-    assert lib.cer_routed_ffn_workspace_size(2348, 6720) == (2348 * 6720 * 2 + 255) // 256 * 256
-    ws = lib.cer_routed_block_workspace_size(4, 1024, 1536, 256, 0, 0, 0, 729, 292, 6720)
+    # FFN: act [M, C] bf16, plus three [C, d] slices when a channel list is packed per call
+    assert lib.cer_routed_ffn_workspace_size(2348, 1536, 6720, 0) == _r256(2348 * 6720 * 2)
+    assert lib.cer_routed_ffn_workspace_size(2348, 1536, 6720, 1) == _r256(2348 * 6720 * 2) + 3 * _r256(6720 * 1536 * 2)
     M = 4 * (292 + 1024 - 729)
-    assert ws == lib.cer_score_workspace_size(4, 1024, 256, 0, 0) + (M * 4 + 255) // 256 * 256 + \
-        (M * 6720 * 2 + 255) // 256 * 256
+    for wc in (0, 1):
+        ws = lib.cer_routed_block_workspace_size(4, 1024, 1536, 256, 0, 0, 0, 729, 292, 6720, wc)
+        assert ws == lib.cer_score_workspace_size(4, 1024, 256, 0, 0) + _r256(M * 4) + _r256(M * 1536 * 2) + \
+            lib.cer_routed_ffn_workspace_size(M, 1536, 6720, wc)
+    assert lib.cer_routed_block_workspace_size(4, 1024, 1536, 256, 0, 0, 0, 729, 730, 6720, 0) == 0  # K > N_r
 
 
 FAKE = ctypes.c_void_p(1 << 20)      # 16-byte aligned, never dereferenced: checks fail first
@@ -79,6 +87,13 @@ def test_ffn_argument_checks(lib):
     assert f(FAKE, 10, 128, FAKE, FAKE, FAKE, 512, FAKE, 576, FAKE, FAKE, 1 << 20, None) == 2   # C > I
     assert f(FAKE, 1000, 128, FAKE, FAKE, FAKE, 512, FAKE, 256, FAKE, FAKE, 16, None) == 9      # workspace
     assert f(FAKE, 10, 128, None, FAKE, FAKE, 512, FAKE, 256, FAKE, FAKE, 1 << 20, None) == 1   # NULL Wg
+
+
+def test_pack_argument_checks(lib):
+    f = lib.cer_pack_ffn_weights
+    assert f(FAKE, FAKE, FAKE, 512, 128, None, 256, FAKE, FAKE, FAKE, None) == 1      # NULL chan
+    assert f(FAKE, FAKE, FAKE, 512, 100, FAKE, 256, FAKE, FAKE, FAKE, None) == 2      # d % 8
+    assert f(FAKE, FAKE, FAKE, 512, 128, FAKE, 600, FAKE, FAKE, FAKE, None) == 2      # C > I
 
 
 def test_score_argument_checks(lib):

@@ -209,17 +209,23 @@ def _inputs(w):
     return gen.make_inputs(w, ffn_weights=_WEIGHTS[key])
 
 
-def _run_block(w, inp, out_of_place=False):
+def _run_block(w, inp, out_of_place=False, prepacked=True):
+    """The fused block on the GPU.  prepacked: kept-channel weight slices made
+    once by cer_pack_ffn_weights (chan=None in the block); else the block gets
+    the full weights and the channel list."""
     core, exp = scorers(inp)
     h = bf16_dev(inp["h"])
     out = torch.empty_like(h) if out_of_place else None
     logits = torch.empty((w.B, w.N), dtype=torch.float32, device="cuda")
     idx = torch.empty((w.B, w.k_tot), dtype=torch.int32, device="cuda")
     mask = torch.empty((w.B, w.N), dtype=torch.uint8, device="cuda")
+    Wg, Wu, WdT = bf16_dev(inp["Wg"]), bf16_dev(inp["Wu"]), bf16_dev(inp["WdT"])
     chan = i32_dev(inp["chan"]) if w.C < w.I else None
+    if prepacked and chan is not None:
+        Wg, Wu, WdT = cer.pack_ffn_weights(Wg, Wu, WdT, chan)
+        chan = None
     cer.cer_routed_block(h, core, exp if w.task == 1 else None, f32_dev(inp["t"]), w.task, w.r0, w.r1, w.K,
-                         bf16_dev(inp["Wg"]), bf16_dev(inp["Wu"]), bf16_dev(inp["WdT"]), chan,
-                         out=out, logits=logits, idx=idx, mask=mask)
+                         Wg, Wu, WdT, chan, out=out, logits=logits, idx=idx, mask=mask)
     cer.cer_sync_status()
     res = dict(out=bits_host(out if out_of_place else h), logits=logits.cpu().numpy(), idx=idx.cpu().numpy(),
                mask=mask.cpu().numpy())
@@ -281,11 +287,22 @@ def _small(name):
 
 @pytest.mark.parametrize("name", ["ragged_gen", "und_text_tail", "k0", "dense_all_kept", "segments", "one_token",
                                   "d3584"])
-def test_routed_block_small(name):
+@pytest.mark.parametrize("prepacked", [True, False], ids=["packed", "chan"])
+def test_routed_block_small(name, prepacked):
     w = _small(name)
     inp = gen.make_inputs(w)
-    res = _run_block(w, inp)
+    res = _run_block(w, inp, prepacked=prepacked)
     _check_block(w, inp, res)
+
+
+def test_pack_ffn_weights_bit_exact():
+    I, d, C = 1000, 264, 333
+    Wg, Wu, WdT = (gen.bf16_normal(5, n, (I, d), 0.1) for n in ("g", "u", "d"))
+    chan = gen.channel_keep_set(5, "c", I, C)
+    outs = cer.pack_ffn_weights(bf16_dev(Wg), bf16_dev(Wu), bf16_dev(WdT), i32_dev(chan))
+    cer.cer_sync_status()
+    for W, o in zip((Wg, Wu, WdT), outs):
+        assert np.array_equal(bits_host(o), W[chan])
 
 
 def test_routed_block_tiny_config_full_compare():
@@ -316,11 +333,11 @@ def test_stage_events_are_recorded():
     inp = gen.make_inputs(w)
     core, exp = scorers(inp)
     h = bf16_dev(inp["h"])
-    evs = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(6)]
     cer.cer_routed_block(h, core, exp, f32_dev(inp["t"]), 1, w.r0, w.r1, w.K, bf16_dev(inp["Wg"]),
                          bf16_dev(inp["Wu"]), bf16_dev(inp["WdT"]), i32_dev(inp["chan"]), stage_events=evs)
     cer.cer_sync_status()
-    times = [evs[i].elapsed_time(evs[i + 1]) for i in range(4)]
+    times = [evs[i].elapsed_time(evs[i + 1]) for i in range(5)]
     assert all(t >= 0 for t in times) and sum(times) > 0
 
 
