@@ -58,18 +58,18 @@ def gemm_source_hash() -> str:
 
 
 def profiled_traffic(workload: str):
-    """DRAM bytes per gate/up launch from the committed ncu summary, if it was
-    taken on this workload with the current kernel sources; else None."""
-    path = os.path.join(ROOT, "profiles", "ffn_gateup_traffic.md")
-    if not os.path.exists(path):
-        return None
-    text = open(path).read()
-    m_src = re.search(r"kernel_source_hash:\s*([0-9a-f]+)", text)
-    m_wl = re.search(r"workload:\s*(\S+)", text)
-    m_b = re.search(r"dram_bytes_per_launch:\s*([0-9]+)", text)
-    if not (m_src and m_wl and m_b) or m_src.group(1) != gemm_source_hash() or m_wl.group(1) != workload:
-        return None
-    return int(m_b.group(1))
+    """DRAM bytes per gate/up launch from a committed ncu summary
+    (profiles/ffn_gateup_*.md) taken on this workload with the current kernel
+    sources; None if there is none."""
+    import glob
+    for path in sorted(glob.glob(os.path.join(ROOT, "profiles", "ffn_gateup_*.md"))):
+        text = open(path).read()
+        m_src = re.search(r"kernel_source_hash:\s*([0-9a-f]+)", text)
+        m_wl = re.search(r"workload:\s*(\S+)", text)
+        m_b = re.search(r"dram_bytes_per_launch:\s*([0-9]+)", text)
+        if m_src and m_wl and m_b and m_src.group(1) == gemm_source_hash() and m_wl.group(1) == workload:
+            return int(m_b.group(1))
+    return None
 
 
 class ClockSampler:
