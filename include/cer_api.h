@@ -98,6 +98,26 @@ cer_status cer_score(const void* h, int B, int N, int d,
                      void* workspace, size_t workspace_bytes, cudaStream_t stream);
 size_t cer_score_workspace_size(int B, int N, int core_hidden, int exp_hidden, int task);
 
+/* ------------------------------------------------------------------ S1 without allocation
+ * cer_score_static: cer_score for callers that cannot allocate device memory
+ * (a plug-in or custom-operator host that gives its operators no workspace
+ * and forbids allocation after load, or a real-time loop whose memory budget
+ * is fixed at start-up).  The paper has no counterpart: this is a deployment
+ * convenience of this library.  Same arguments and results as cer_score, but
+ * no workspace: the scratch lives in one static device array of 4 MiB
+ * (4194304 bytes), present on every GPU that loads the library until the
+ * process exits.  Sizes whose cer_score_workspace_size() exceeds 4 MiB are
+ * rejected with CER_ERR_WORKSPACE before any work is enqueued.  The call
+ * allocates nothing.  Its first call on a device looks up the array's device
+ * address (with that device current); make that first call before any
+ * stream capture.  All calls share the array: calls whose GPU work can
+ * overlap (other streams, other host threads) race on it; calls on one
+ * stream are safe.                                                          */
+cer_status cer_score_static(const void* h, int B, int N, int d,
+                            const cer_scorer* core, const cer_scorer* exp,
+                            const float* t, int task,
+                            float* logits, float* probs, cudaStream_t stream);
+
 /* ------------------------------------------------------------------ S2 select
  * Keep set R of Eq. 4 (Sec. 3.4) per sequence: the K tokens of [r0, r1) with
  * the largest logit (ranking logits equals ranking sigmoid(l), App. B.2), ties

@@ -26,7 +26,7 @@ STATUS_NAMES = {0: "CER_OK", 1: "CER_ERR_NULL", 2: "CER_ERR_SHAPE", 3: "CER_ERR_
                 9: "CER_ERR_WORKSPACE", 10: "CER_ERR_INDEX"}
 
 # Every symbol include/cer_api.h declares.
-EXPORTS = ("cer_score", "cer_score_workspace_size", "cer_select_topk", "cer_gather", "cer_routed_ffn",
+EXPORTS = ("cer_score", "cer_score_workspace_size", "cer_score_static", "cer_select_topk", "cer_gather", "cer_routed_ffn",
            "cer_routed_ffn_workspace_size", "cer_pack_ffn_weights", "cer_scatter_add", "cer_routed_block",
            "cer_routed_block_workspace_size", "cer_sync_status", "cer_get_error", "cer_status_string",
            "cer_version")
@@ -51,6 +51,7 @@ _SCP = ctypes.POINTER(CerScorerC)
 _SIGS = {
     "cer_score": ([_vp, _i, _i, _i, _SCP, _SCP, _vp, _i, _vp, _vp, _vp, _sz, _vp], _i),
     "cer_score_workspace_size": ([_i, _i, _i, _i, _i], _sz),
+    "cer_score_static": ([_vp, _i, _i, _i, _SCP, _SCP, _vp, _i, _vp, _vp, _vp], _i),
     "cer_select_topk": ([_vp, _i, _i, _i, _i, _i, _vp, _vp, _vp], _i),
     "cer_gather": ([_vp, _i, _i, _i, _vp, _i, _vp, _vp], _i),
     "cer_routed_ffn": ([_vp, _i, _i, _vp, _vp, _vp, _i, _vp, _i, _vp, _vp, _sz, _vp], _i),
@@ -134,6 +135,14 @@ def cer_score(h, core: Scorer, exp: Optional[Scorer], t, task, logits, probs=Non
         ws = workspace(need, h.device)
     _check(load().cer_score(_p(h), B, N, d, _sref(core), _sref(exp), _p(t), task, _p(logits), _p(probs),
                             _p(ws), ws.numel(), _stream(stream)))
+
+
+def cer_score_static(h, core: Scorer, exp: Optional[Scorer], t, task, logits, probs=None, stream=None):
+    """cer_score without a workspace: the scratch is the library's static
+    4 MiB device array (for callers that cannot allocate; see cer_api.h)."""
+    B, N, d = h.shape
+    _check(load().cer_score_static(_p(h), B, N, d, _sref(core), _sref(exp), _p(t), task, _p(logits), _p(probs),
+                                   _stream(stream)))
 
 
 def cer_select_topk(logits, r0, r1, K, idx, mask=None, stream=None):

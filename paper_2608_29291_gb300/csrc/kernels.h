@@ -8,12 +8,17 @@
 #include <cstddef>
 #include <cstdint>
 
+#include "../../include/cer_api.h"
+
 namespace cer {
 
 // Encode a 2-D bf16 tensor map (rows x cols, row pitch cols*2 bytes) with a
 // box of box_cols x box_rows elements, 128-byte swizzle, zero fill.
 bool encode_bf16_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_cols,
                     uint32_t box_rows);
+
+// Record a printf-style message for cer_get_error() and return `status`.
+cer_status internal_fail(cer_status status, const char* fmt, ...);
 
 // Raise a kernel's dynamic shared-memory limit to `bytes` (its largest
 // launch) once per device.
