@@ -10,10 +10,13 @@
 // gate/up:  act[m, c] = SiLU(Wg[c] . x_m) * (Wu[c] . x_m)
 //   One 128x256 MMA tile holds gate (columns 0..127) and up (128..255) for
 //   the same 128 channels, so the SwiGLU runs in the epilogue and act is
-//   written once, as bf16.
+//   written once, as bf16: each half of the epilogue warps stages its
+//   128 x 64 act box in shared memory (128-byte swizzle, conflict-free) and
+//   one thread writes it with a TMA store, overlapping the next tile.
 // down:     y[m, n] = sum_c act[m, c] * WdT[c, n]
-//   B is MN-major: 64 channel rows x 256 output columns, four 64-column TMA
-//   boxes per K block.  Epilogue: Y = bf16(y), or, fused, the unpack
+//   B is MN-major: 64 channel rows x BN output columns (BN = 128, 192 or 256,
+//   picked per launch so the tiles fill the SMs), one 64-column TMA box per
+//   64 columns per K block.  Epilogue: Y = bf16(y), or, fused, the unpack
 //   out[b, idx[m], n] = bf16(h[b, idx[m], n] + y) -- the kept rows are
 //   distinct, so no atomics; dropped rows are never touched.
 #include <cuda_bf16.h>
@@ -32,71 +35,113 @@ __device__ __forceinline__ float silu_mul(float g, float u) {
 
 // ---------------------------------------------------------------- gate/up
 
-struct GateUpProblem {
+template <int EPI_WARPS_>
+struct GateUpProblemT {
   static constexpr int BN = 256;
   static constexpr int STAGES = 4;
   static constexpr int B_MN_MAJOR = 0;
+  static constexpr int EPI_WARPS = EPI_WARPS_;
+  static constexpr int kGroups = EPI_WARPS / 4;
+  // Two CTAs per cluster take adjacent 128-row tiles of the same 128
+  // channels: rank 0 fetches the gate rows of the B tile, rank 1 the up rows,
+  // each multicast to both, so each CTA reads 32 KB instead of 48 KB of L2
+  // per K block.
+  static constexpr int CLUSTER = 2;
   static constexpr uint32_t kBStepBytes = 32;
+  static constexpr uint32_t kBoxBytes = 128 * 128;          // 128 rows x 64 bf16
+  static constexpr uint32_t kEpiSmemBytes = 2 * kBoxBytes;  // the act tile as two TMA boxes
 
   struct Params {
-    CUtensorMap tm_x;   // X [M, d], box 64 x 128
-    CUtensorMap tm_wg;  // Wg [C, d], box 64 x 128
-    CUtensorMap tm_wu;  // Wu [C, d], box 64 x 128
-    __nv_bfloat16* act;
+    CUtensorMap tm_x;    // X [M, d], box 64 x 128
+    CUtensorMap tm_wg;   // Wg [C, d], box 64 x 128
+    CUtensorMap tm_wu;   // Wu [C, d], box 64 x 128
+    CUtensorMap tm_act;  // act [M, C], box 64 x 128 (store)
     int* status;
-    int M, d, C, n_mt, n_ct;
+    int M, d, C, n_mt, n_mtp, n_ct;
   };
   struct ProdState {
-    int m0, c0;
+    int m0, c0, rank;
   };
 
-  __device__ static int num_tiles(const Params& p) { return p.n_mt * p.n_ct; }
+  // Cluster tile t covers row tiles 2*(t % n_mtp) + {0, 1} and channel tile t / n_mtp.
+  __device__ static int num_tiles(const Params& p) { return p.n_mtp * p.n_ct; }
   __device__ static int num_kb(const Params& p) { return p.d / 64; }
   __device__ static uint32_t stage_bytes(const Params&, int, int) { return kATileBytes + BN * 128; }
-  __device__ static void prod_tile(const Params& p, int tile, int, ProdState& st) {
-    st.c0 = (tile / p.n_mt) * 128;
-    st.m0 = (tile % p.n_mt) * 128;
+  __device__ static void prod_tile(const Params& p, int tile, int rank, ProdState& st) {
+    st.c0 = (tile / p.n_mtp) * 128;
+    st.m0 = (2 * (tile % p.n_mtp) + rank) * 128;   // rows past M load as zeros
+    st.rank = rank;
   }
   __device__ static void prod_kb(const Params& p, const ProdState& st, int, int kb, int lane, uint8_t* a,
                                  uint8_t* b, uint64_t* bar) {
     if (lane == 0) {
       const int x = kb * 64;
       tma_load_2d(a, &p.tm_x, bar, x, st.m0);
-      tma_load_2d(b, &p.tm_wg, bar, x, st.c0);
-      tma_load_2d(b + 128 * 128, &p.tm_wu, bar, x, st.c0);
+      if (st.rank == 0)
+        tma_load_2d_multicast(b, &p.tm_wg, bar, x, st.c0, 0x3);
+      else
+        tma_load_2d_multicast(b + 128 * 128, &p.tm_wu, bar, x, st.c0, 0x3);
     }
   }
   __device__ static uint64_t bdesc(uint32_t saddr) { return sdesc_kmajor_sw128(saddr); }
 
-  __device__ static void epilogue(const Params& p, int tile, int row, int half, uint32_t taddr) {
-    const int ct = tile / p.n_mt;
-    const int m = (tile % p.n_mt) * 128 + row;
-    const bool valid = m < p.M;
+  // Group `grp` (four warps, 128 threads, one accumulator row each) produces
+  // the 64-channel boxes grp*2/kGroups .. of the tile's 128 channels.
+  __device__ static bool epilogue(const Params& p, int tile, int row, int grp, uint32_t taddr, EpiCtx& ctx) {
+    const int ct = tile / p.n_mtp;
+    const int mt = 2 * (tile % p.n_mtp) + ctx.rank;
+    const bool leader = (row == 0);
 #pragma unroll 1
-    for (int c = 2 * half; c < 2 * half + 2; ++c) {
-      float g[32], u[32];
-      tmem_ld2_32x32(taddr + c * 32, taddr + 128 + c * 32, g, u);
-      const int ch0 = ct * 128 + c * 32;
-      if (valid && ch0 < p.C) {
+    for (int bi = 0; bi < 2 / kGroups; ++bi) {
+      const int bx = grp * (2 / kGroups) + bi;     // box: channels [64*bx, 64*bx + 64)
+      uint8_t* box = ctx.smem + bx * kBoxBytes;
+      if (leader) bulk_wait_group_read0();         // the previous store has read the boxes
+      if (!ctx.sync()) return false;
+      uint8_t* my_row = box + row * 128;
+#pragma unroll 1
+      for (int c = 0; c < 2; ++c) {
+        float g[32], u[32];
+        const int col = 64 * bx + 32 * c;
+        tmem_ld2_32x32(taddr + col, taddr + 128 + col, g, u);
         uint32_t pk[16];
 #pragma unroll
         for (int j = 0; j < 16; ++j) pk[j] = pack_bf16x2(silu_mul(g[2 * j], u[2 * j]), silu_mul(g[2 * j + 1], u[2 * j + 1]));
-        uint4* dst = reinterpret_cast<uint4*>(p.act + static_cast<size_t>(m) * p.C + ch0);
 #pragma unroll
-        for (int v = 0; v < 4; ++v) dst[v] = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+        for (int v = 0; v < 4; ++v) {
+          const int chunk16 = (4 * c + v) ^ (row & 7);   // 128-byte swizzle of the TMA box
+          *reinterpret_cast<uint4*>(my_row + chunk16 * 16) = make_uint4(pk[4 * v], pk[4 * v + 1], pk[4 * v + 2], pk[4 * v + 3]);
+        }
+      }
+      fence_proxy_async_smem();
+      if (!ctx.sync()) return false;
+      const int x = ct * 128 + 64 * bx;
+      if (leader && x < p.C && mt < p.n_mt) {
+        tma_store_2d(&p.tm_act, box, x, mt * 128);
+        bulk_commit_group();
       }
     }
+    return true;
+  }
+  __device__ static void epilogue_done(const Params&, int row, int) {
+    if (row == 0) bulk_wait_group0();
   }
 };
 
+using GateUpProblem = GateUpProblemT<4>;
+
 // ---------------------------------------------------------------- down
 
+template <int BN_>
 struct DownProblem {
-  static constexpr int BN = 256;
-  static constexpr int STAGES = 4;
+  static constexpr int BN = BN_;
+  static constexpr int ATOMS = BN / 64;
+  static constexpr int STAGES = BN == 256 ? 4 : BN == 192 ? 5 : 6;
   static constexpr int B_MN_MAJOR = 1;
+  static constexpr int EPI_WARPS = 8;
+  static constexpr int CLUSTER = 1;
   static constexpr uint32_t kBStepBytes = 2048;     // 16 K-rows = two 1024 B row groups
   static constexpr uint32_t kAtomBytes = 64 * 128;  // 64 K-rows x 64 columns
+  static constexpr uint32_t kEpiSmemBytes = 0;
 
   struct Params {
     CUtensorMap tm_act;  // act [M, C], box 64 x 128
@@ -115,15 +160,15 @@ struct DownProblem {
   __device__ static int num_tiles(const Params& p) { return p.n_mt * p.n_nt; }
   __device__ static int num_kb(const Params& p) { return p.C / 64; }
   __device__ static int atoms(const Params& p, int nt) {
-    const int left = (p.d - nt * 256) / 64;
-    return left < 4 ? left : 4;
+    const int left = (p.d - nt * BN) / 64;
+    return left < ATOMS ? left : ATOMS;
   }
   __device__ static uint32_t stage_bytes(const Params& p, int tile, int) {
     return kATileBytes + atoms(p, tile / p.n_mt) * kAtomBytes;
   }
   __device__ static void prod_tile(const Params& p, int tile, int, ProdState& st) {
     const int nt = tile / p.n_mt;
-    st.n0 = nt * 256;
+    st.n0 = nt * BN;
     st.m0 = (tile % p.n_mt) * 128;
     st.n_atoms = atoms(p, nt);
   }
@@ -136,7 +181,8 @@ struct DownProblem {
   }
   __device__ static uint64_t bdesc(uint32_t saddr) { return sdesc_mnmajor_sw128(saddr, kAtomBytes, 1024); }
 
-  __device__ static void epilogue(const Params& p, int tile, int row, int half, uint32_t taddr) {
+  __device__ static void epilogue_done(const Params&, int, int) {}
+  __device__ static bool epilogue(const Params& p, int tile, int row, int half, uint32_t taddr, EpiCtx&) {
     const int nt = tile / p.n_mt;
     const int m = (tile % p.n_mt) * 128 + row;
     bool valid = m < p.M;
@@ -153,11 +199,12 @@ struct DownProblem {
         dst_row = static_cast<size_t>(m);
       }
     }
+    constexpr int kChunksPerHalf = BN / 64;
 #pragma unroll 1
-    for (int c = 4 * half; c < 4 * half + 4; ++c) {
+    for (int c = kChunksPerHalf * half; c < kChunksPerHalf * (half + 1); ++c) {
       float v[32];
       tmem_ld_32x32(taddr + c * 32, v);
-      const int n0 = nt * 256 + c * 32;
+      const int n0 = nt * BN + c * 32;
       if (valid && n0 < p.d) {
         uint32_t pk[16];
         if (p.scatter) {
@@ -181,20 +228,51 @@ struct DownProblem {
         for (int q = 0; q < 4; ++q) dst[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
       }
     }
+    return true;
   }
 };
 
 // ---------------------------------------------------------------- launchers
 
+// `tiles` counts cluster tiles; one cluster of P::CLUSTER CTAs per tile at a
+// time, as many clusters as the SMs hold.
 template <class P>
 static cudaError_t launch_gemm(const typename P::Params& p, int tiles, int n_sm, cudaStream_t stream) {
   if (tiles == 0) return cudaSuccess;
   const size_t smem = gemm_smem_bytes<P>();
   cudaError_t e = ensure_max_smem(reinterpret_cast<const void*>(umma_gemm_kernel<P>), smem);
   if (e != cudaSuccess) return e;
-  const int grid = tiles < n_sm ? tiles : n_sm;
-  umma_gemm_kernel<P><<<grid, kGemmThreads, smem, stream>>>(p);
-  return cudaGetLastError();
+  if (P::CLUSTER == 1) {
+    const int grid = tiles < n_sm ? tiles : n_sm;
+    umma_gemm_kernel<P><<<grid, gemm_threads<P>(), smem, stream>>>(p);
+    return cudaGetLastError();
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.blockDim = dim3(gemm_threads<P>(), 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = P::CLUSTER;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  // The persistent grid holds only as many clusters as can be resident at
+  // once (SM pairs inside GPC boundaries), so no cluster waits for another.
+  static int resident[64] = {0};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  int& max_clusters = resident[dev & 63];
+  if (max_clusters == 0) {
+    cfg.gridDim = dim3(n_sm / P::CLUSTER * P::CLUSTER, 1, 1);
+    int n = 0;
+    e = cudaOccupancyMaxActiveClusters(&n, umma_gemm_kernel<P>, &cfg);
+    if (e != cudaSuccess) return e;
+    max_clusters = n > 0 ? n : 1;
+  }
+  cfg.gridDim = dim3((tiles < max_clusters ? tiles : max_clusters) * P::CLUSTER, 1, 1);
+  return cudaLaunchKernelEx(&cfg, umma_gemm_kernel<P>, p);
 }
 
 cudaError_t launch_ffn_gateup(const FfnArgs& a, int n_sm, cudaStream_t stream) {
@@ -202,18 +280,21 @@ cudaError_t launch_ffn_gateup(const FfnArgs& a, int n_sm, cudaStream_t stream) {
   if (!encode_bf16_2d(&p.tm_x, a.X, a.M, a.d, 64, 128)) return cudaErrorInvalidValue;
   if (!encode_bf16_2d(&p.tm_wg, a.Wg, a.C, a.d, 64, 128)) return cudaErrorInvalidValue;
   if (!encode_bf16_2d(&p.tm_wu, a.Wu, a.C, a.d, 64, 128)) return cudaErrorInvalidValue;
-  p.act = a.act;
+  if (!encode_bf16_2d(&p.tm_act, a.act, a.M, a.C, 64, 128)) return cudaErrorInvalidValue;
   p.status = a.status;
   p.M = a.M;
   p.d = a.d;
   p.C = a.C;
   p.n_mt = (a.M + 127) / 128;
+  p.n_mtp = (p.n_mt + 1) / 2;
   p.n_ct = (a.C + 127) / 128;
-  return launch_gemm<GateUpProblem>(p, p.n_mt * p.n_ct, n_sm, stream);
+  return launch_gemm<GateUpProblem>(p, p.n_mtp * p.n_ct, n_sm, stream);
 }
 
-cudaError_t launch_ffn_down(const FfnArgs& a, int n_sm, cudaStream_t stream) {
-  DownProblem::Params p{};
+template <int BN>
+static cudaError_t launch_down(const FfnArgs& a, int n_sm, cudaStream_t stream) {
+  using P = DownProblem<BN>;
+  typename P::Params p{};
   if (!encode_bf16_2d(&p.tm_act, a.act, a.M, a.C, 64, 128)) return cudaErrorInvalidValue;
   if (!encode_bf16_2d(&p.tm_wdt, a.WdT, a.C, a.d, 64, 64)) return cudaErrorInvalidValue;
   p.idx = a.idx;
@@ -227,8 +308,33 @@ cudaError_t launch_ffn_down(const FfnArgs& a, int n_sm, cudaStream_t stream) {
   p.N = a.N;
   p.k_tot = a.k_tot;
   p.n_mt = (a.M + 127) / 128;
-  p.n_nt = (a.d + 255) / 256;
-  return launch_gemm<DownProblem>(p, p.n_mt * p.n_nt, n_sm, stream);
+  p.n_nt = (a.d + BN - 1) / BN;
+  return launch_gemm<P>(p, p.n_mt * p.n_nt, n_sm, stream);
+}
+
+// N-tile width of the down GEMM: the one with the least per-SM work
+// (waves x width), the wider on a tie.
+int down_tile_width(int M, int d, int n_sm) {
+  const long n_mt = (M + 127) / 128;
+  int best = 256;
+  long best_cost = -1;
+  for (int bn : {256, 192, 128}) {
+    const long tiles = n_mt * ((d + bn - 1) / bn);
+    const long cost = ((tiles + n_sm - 1) / n_sm) * bn;
+    if (best_cost < 0 || cost < best_cost) {
+      best_cost = cost;
+      best = bn;
+    }
+  }
+  return best;
+}
+
+cudaError_t launch_ffn_down(const FfnArgs& a, int n_sm, cudaStream_t stream) {
+  switch (down_tile_width(a.M, a.d, n_sm)) {
+    case 192: return launch_down<192>(a, n_sm, stream);
+    case 128: return launch_down<128>(a, n_sm, stream);
+    default: return launch_down<256>(a, n_sm, stream);
+  }
 }
 
 }  // namespace cer

@@ -42,6 +42,12 @@ struct ScoreArgs {
   int* status;
 };
 
+// Frequencies of the sinusoidal progress embedding divided by 2*pi, in fp64:
+// g[j] = 10000^(-j/(E/2)) / (2*pi), j < E/2 <= 512 (computed on the host).
+struct EmbFreqTable {
+  double g[512];
+};
+
 struct ScoreWorkspace {
   float* bias_tab;  // [B][Hc + He]
   float* w2_tab;    // [B][Hc + He]

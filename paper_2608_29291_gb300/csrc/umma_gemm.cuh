@@ -1,36 +1,51 @@
 // umma_gemm.cuh -- persistent, warp-specialised tcgen05 GEMM skeleton for
 // sm_103a, shared by the scorer and the two FFN contractions.
 //
-// One CTA per SM (320 threads, ~193 KB shared memory, 2*BN TMEM columns):
+// One CTA per SM (64 + 32*EPI_WARPS threads, up to ~225 KB shared memory,
+// 2*BN TMEM columns):
 //   warp 0     producer: TMA box loads of the A tile (128 rows x 64 bf16)
 //              and the B tile (BN rows x 64 bf16, or 64 K-rows x BN for an
 //              MN-major B) into a STAGES-deep ring;
 //   warp 1     allocates TMEM, one elected lane issues tcgen05.mma
 //              (M=128, N=BN, K=16) four times per 64-wide K block and
 //              commits the ring slot back to the producer;
-//   warps 2-9  epilogue: read the fp32 accumulator out of TMEM (lane = tile
-//              row; warps 2-5 take the first half of the columns, warps 6-9
-//              the second) and apply the problem's fused epilogue.
+//   warps 2..  epilogue, EPI_WARPS = 4 or 8: read the fp32 accumulator out of
+//              TMEM (lane = tile row; with 8 warps, warps 2-5 take the first
+//              half of the columns and warps 6-9 the second) and apply the
+//              problem's fused epilogue.
 // The accumulator is double-buffered in TMEM so the epilogue of tile i
-// overlaps the MMAs of tile i+1.  Tiles are visited with a stride of
-// gridDim.x.  Every wait is bounded (ptx.cuh); on a timeout the CTA unwinds,
+// overlaps the MMAs of tile i+1.  Tiles are visited with a stride of the
+// number of clusters.  With CLUSTER == 2 the two CTAs of a cluster work on
+// one cluster tile (two adjacent 128-row tiles sharing a B tile): each loads
+// half of B and multicasts it to both, each MMA commit frees the ring slot
+// in both CTAs, and cluster barriers bracket start-up and teardown so no CTA
+// exits while its peer may still write into its shared memory.  Every wait is bounded (ptx.cuh); on a timeout the CTA unwinds,
 // waits briefly for its own copies and MMAs, frees TMEM and exits.
 //
 // A problem class P supplies:
-//   BN, STAGES, B_MN_MAJOR, kBStepBytes, Params (with `int* status`),
-//   num_tiles(p), num_kb(p), prod_tile(p, tile, lane, state),
+//   BN, STAGES, B_MN_MAJOR, EPI_WARPS, CLUSTER, kBStepBytes,
+//   Params (with `int* status`), num_tiles(p) (cluster tiles),
+//   num_kb(p), prod_tile(p, tile, rank, state),
 //   prod_kb(p, state, tile, kb, lane, a_smem, b_smem, bar),
 //   stage_bytes(p, tile, kb), bdesc(saddr),
-//   epilogue(p, tile, row, half, taddr): columns [half*BN/2, (half+1)*BN/2)
-//   of accumulator row `row`, taddr addressing column 0 of that row's lanes.
+//   kEpiSmemBytes (shared memory reserved for the epilogue, may be 0),
+//   epilogue(p, tile, row, half, taddr, ctx) -> false to abort (ctx.rank is
+//   the CTA's rank in its cluster): columns
+//   [half*BN/H, (half+1)*BN/H) of accumulator row `row` (H = EPI_WARPS/4
+//   groups of four warps), taddr addressing
+//   column 0 of that row's lanes, ctx the reserved shared memory and a
+//   bounded barrier over the 128 threads of the half;
+//   epilogue_done(p, row, half): once, after the last tile.
 #pragma once
 
 #include "ptx.cuh"
 
 namespace cer {
 
-constexpr int kEpiWarps = 8;
-constexpr int kGemmThreads = 64 + 32 * kEpiWarps;
+template <class P>
+constexpr int gemm_threads() {
+  return 64 + 32 * P::EPI_WARPS;
+}
 constexpr uint32_t kATileBytes = 128 * 128;  // 128 rows x 64 bf16
 
 template <int BN>
@@ -41,7 +56,7 @@ struct TmemCols {
 
 template <class P>
 constexpr size_t gemm_smem_bytes() {
-  return 1024 + static_cast<size_t>(P::STAGES) * (kATileBytes + P::BN * 128) + 256;
+  return 1024 + static_cast<size_t>(P::STAGES) * (kATileBytes + P::BN * 128) + P::kEpiSmemBytes + 256;
 }
 
 // A short, abort-independent wait used only while unwinding.
@@ -62,8 +77,29 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volati
   return ok != 0;
 }
 
+// What an epilogue half (4 warps, 128 threads) shares: the reserved shared
+// memory and a barrier over its threads whose wait is bounded like every
+// other wait (an mbarrier of count 128; each thread tracks the phase).
+struct EpiCtx {
+  uint8_t* smem;
+  int rank;
+  uint64_t* half_bar;
+  uint32_t phase;
+  volatile int* abort_flag;
+  int* status;
+  __device__ __forceinline__ bool sync() {
+    mbar_arrive(half_bar);
+    const bool ok = mbar_wait(half_bar, phase, abort_flag, status);
+    phase ^= 1;
+    return ok;
+  }
+};
+
 template <class P>
-__global__ void __launch_bounds__(kGemmThreads, 1) umma_gemm_kernel(const __grid_constant__ typename P::Params p) {
+__global__ void __launch_bounds__(gemm_threads<P>(), 1) umma_gemm_kernel(const __grid_constant__ typename P::Params p) {
+  static_assert(P::EPI_WARPS == 4 || P::EPI_WARPS == 8, "epilogue is one or two groups of four warps");
+  static_assert(P::CLUSTER == 1 || P::CLUSTER == 2, "clusters of one or two CTAs");
+  constexpr uint16_t kPairMask = 0x3;
   constexpr int BN = P::BN;
   constexpr int STAGES = P::STAGES;
   constexpr uint32_t B_BYTES = BN * 128;
@@ -74,27 +110,34 @@ __global__ void __launch_bounds__(kGemmThreads, 1) umma_gemm_kernel(const __grid
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* a_ring = smem;
   uint8_t* b_ring = smem + STAGES * kATileBytes;
-  uint64_t* full = reinterpret_cast<uint64_t*>(b_ring + STAGES * B_BYTES);
+  uint8_t* epi_smem = b_ring + STAGES * B_BYTES;  // 1024-byte aligned
+  uint64_t* full = reinterpret_cast<uint64_t*>(epi_smem + P::kEpiSmemBytes);
   uint64_t* empty = full + STAGES;
   uint64_t* tfull = empty + STAGES;
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tempty + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  uint64_t* half_bar = drain + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(half_bar + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  const int rank = P::CLUSTER > 1 ? static_cast<int>(cluster_ctarank()) : 0;
+  const int cluster_id = blockIdx.x / P::CLUSTER;
+  const int n_clusters = gridDim.x / P::CLUSTER;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
+      mbar_init(&empty[s], P::CLUSTER);   // one MMA commit from each CTA of the cluster
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull[a], 1);
-      mbar_init(&tempty[a], 32 * kEpiWarps);
+      mbar_init(&tempty[a], 32 * P::EPI_WARPS);
     }
     mbar_init(drain, 1);
+    mbar_init(&half_bar[0], 128);
+    mbar_init(&half_bar[1], 128);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -103,7 +146,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1) umma_gemm_kernel(const __grid
     tmem_relinquish();
   }
   tc_fence_before();
-  __syncthreads();
+  if (P::CLUSTER > 1) {
+    cluster_sync();      // the peer's barriers exist before any multicast reaches them
+  } else {
+    __syncthreads();
+  }
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
@@ -117,8 +164,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1) umma_gemm_kernel(const __grid
     uint32_t phase = 0;
     long issued = 0;
     bool ok = true;
-    for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
-      P::prod_tile(p, tile, lane, st);
+    for (int tile = cluster_id; tile < ntiles && ok; tile += n_clusters) {
+      P::prod_tile(p, tile, rank, st);
       for (int kb = 0; kb < nkb; ++kb) {
         if (!warp_wait(&empty[stage], phase ^ 1, abort_flag, p.status)) {
           ok = false;
@@ -148,7 +195,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1) umma_gemm_kernel(const __grid
     uint32_t acc_phase = 0;
     bool ok = true;
     bool issued_any = false;
-    for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
+    for (int tile = cluster_id; tile < ntiles && ok; tile += n_clusters) {
       if (!warp_wait(&tempty[acc], acc_phase ^ 1, abort_flag, p.status)) {
         ok = false;
         break;
@@ -169,7 +216,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1) umma_gemm_kernel(const __grid
             umma_bf16(d_tmem, sdesc_kmajor_sw128(a_base + k * 32), P::bdesc(b_base + k * P::kBStepBytes), IDESC,
                       (kb | k) != 0 ? 1u : 0u);
           }
-          umma_commit(&empty[stage]);
+          if (P::CLUSTER > 1)
+            umma_commit_multicast(&empty[stage], kPairMask);   // frees the slot in both CTAs
+          else
+            umma_commit(&empty[stage]);
           issued_any = true;
         }
         __syncwarp();
@@ -195,24 +245,31 @@ __global__ void __launch_bounds__(kGemmThreads, 1) umma_gemm_kernel(const __grid
     const int q = warp & 3;            // TMEM lane quadrant this warp may access
     const int row = q * 32 + lane;     // accumulator row = TMEM lane
     const int half = (warp - 2) >> 2;  // which half of the accumulator columns
+    EpiCtx ctx{epi_smem, rank, &half_bar[half], 0u, abort_flag, p.status};
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+    for (int tile = cluster_id; tile < ntiles; tile += n_clusters) {
       if (!warp_wait(&tfull[acc], acc_phase, abort_flag, p.status)) break;
       tc_fence_after();
       const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BN);
-      P::epilogue(p, tile, row, half, taddr);
+      const bool ok = P::epilogue(p, tile, row, half, taddr, ctx);
       tc_fence_before();
       mbar_arrive(&tempty[acc]);
+      if (!ok) break;
       if (++acc == 2) {
         acc = 0;
         acc_phase ^= 1;
       }
     }
+    P::epilogue_done(p, row, half);
   }
 
   tc_fence_before();
-  __syncthreads();
+  if (P::CLUSTER > 1) {
+    cluster_sync();      // the peer no longer multicasts into this CTA
+  } else {
+    __syncthreads();
+  }
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem_base, TMEM_COLS);

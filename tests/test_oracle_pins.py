@@ -434,3 +434,4 @@ def test_pins_catch_planted_mistake(name, monkeypatch):
 
 def test_pins_pass_unmutated():
     assert _all_pin_failures() == []
+
