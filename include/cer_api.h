@@ -79,7 +79,7 @@ typedef struct cer_scorer {
 } cer_scorer;
 
 /* ------------------------------------------------------------------ S1 score
- * Routing logits of Eq. 1 (Sec. 3.2): l^U = c(h) for understanding,
+ * Routing logits of Eq. 4 (Sec. 3.2, core_expansion_formulation): l^U = c(h) for understanding,
  * l^G = c(h) + e_{m(t)}(h) for generation.
  *   h        bf16 [B, N, d]; d a multiple of 64, <= 16384
  *   core     the core scorer (n_segments must be 1, U must be NULL)
@@ -87,7 +87,7 @@ typedef struct cer_scorer {
  *            (may be NULL for CER_TASK_UND); its hidden width may differ
  *   t        fp32 [B] denoising progress per sequence (read for CER_TASK_GEN)
  *   logits   fp32 [B, N] output
- *   probs    fp32 [B, N] output p = sigmoid(l) of Eq. 4, or NULL
+ *   probs    fp32 [B, N] output p = sigmoid(l) of Eq. 6, or NULL
  * Workspace: cer_score_workspace_size(B, N, core->hidden, exp hidden, task).
  * The GEMM runs on tcgen05 tensor cores (bf16 operands, fp32 accumulation);
  * bias, GELU and the w2 dot product are applied in fp32.                     */
@@ -119,7 +119,7 @@ cer_status cer_score_static(const void* h, int B, int N, int d,
                             float* logits, float* probs, cudaStream_t stream);
 
 /* ------------------------------------------------------------------ S2 select
- * Keep set R of Eq. 4 (Sec. 3.4) per sequence: the K tokens of [r0, r1) with
+ * Keep set R of Eq. 6 (Sec. 3.4, router_inference_outputs) per sequence: the K tokens of [r0, r1) with
  * the largest logit (ranking logits equals ranking sigmoid(l), App. B.2), ties
  * to the lower token index, -0.0 equal to +0.0, -inf allowed; plus every
  * token outside [r0, r1).  Exact: integer radix select on order-preserving

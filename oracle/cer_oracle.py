@@ -13,10 +13,10 @@ numpy exp/cos/sin/floor, scipy.special.erf, Python's ``sorted``.
 
 Paper passages followed (CE-Router, "Core-Expansion Routing and Unified
 Computation Scheduling"):
-  * Sec. 3.2, Eq. 1 (core_expansion_formulation): logits l^U = c_l(h),
+  * Sec. 3.2, Eq. 4 (core_expansion_formulation): logits l^U = c_l(h),
     l^G = c_l(h) + e_{l,m(t)}(h); core and expansions are token-wise MLPs with a
     scalar output; M segments of the denoising timesteps.
-  * Sec. 3.4, Eq. 4 (router_inference_outputs): p = sigmoid(l), R = TopK(p, K);
+  * Sec. 3.4, Eq. 6 (router_inference_outputs): p = sigmoid(l), R = TopK(p, K);
     App. B.2: the sigmoid is monotonic, so ranking logits gives the same set.
   * Sec. 3.4, task-adaptive token compaction: R is packed into a shorter
     sequence for the FFN, D bypasses unchanged.
@@ -36,6 +36,21 @@ Readings where the paper is silent or leaves a choice open:
     the update is not scaled by p;
   * block output bf16(h + y) for kept rows: the fp64 sum rounded to fp32, then
     to bf16 (round to nearest even at both steps); dropped rows bit-identical.
+
+UCS statistics (Sec. 3.4, Unified Computation Scheduling):
+  * Eq. 8 (ffn_saliency), Eq. 9 (ffn_leakage): channel saliency on the
+    retained tokens and the leakage of the pruned channel set;
+  * Eq. 7 (redundancy_gap): mean input-output cosine over all tokens minus
+    the mean over the retained tokens;
+  * Eq. 10 (drop_jaccard), Eq. 11 (rda): Jaccard similarity of two drop sets and
+    its random-adjusted form.
+  Readings: the drop set D is the routable tokens not kept (tokens outside
+  the routable range are never dropped); the expected random Jaccard is the
+  ratio of expectations E|A&B| / E|A|B| with E|A&B| = |A||B|/n for uniformly
+  random drop sets of the same sizes among the n routable tokens; an empty
+  union gives J = 1, J_rand = 1 gives RDA = 1 (identical patterns); the
+  retained set R is every kept token; a zero-norm pair has cosine 1 when the
+  vectors are equal, else 0; empty R gives g = 0.
 
 Parity status: every function below is pinned by tests/test_oracle_pins.py
 (hand-computed example, brute-force top-k, closed forms, library special cases,
@@ -105,7 +120,7 @@ def mlp_score(x: np.ndarray, W1: np.ndarray, w2: np.ndarray, bias: np.ndarray) -
 
 
 def score(h, W1, w2, b1, t, task, W1e=None, w2e=None, Ue=None, b1e=None) -> np.ndarray:
-    """Routing logits of Eq. 1 for every token; returns fp32 [B, N].
+    """Routing logits of Eq. 4 for every token; returns fp32 [B, N].
 
     h: bf16 bits [B, N, d].  Core: W1 bf16 [Hc, d], w2 fp32 [Hc], b1 fp32 [Hc] or None.
     Expansion (generation only): W1e bf16 [S, He, d], w2e fp32 [S, He],
@@ -135,14 +150,14 @@ def score(h, W1, w2, b1, t, task, W1e=None, w2e=None, Ue=None, b1e=None) -> np.n
 
 
 def sigmoid(x: np.ndarray) -> np.ndarray:
-    """Bounded importance p = sigmoid(l) of Eq. 4, in fp64."""
+    """Bounded importance p = sigmoid(l) of Eq. 6, in fp64."""
     return 1.0 / (1.0 + np.exp(-np.asarray(x, dtype=np.float64)))
 
 
 # ---------------------------------------------------------------- selection
 
 def select_topk(logits: np.ndarray, r0: int, r1: int, K: int):
-    """Per-sequence keep set R (Eq. 4): the K routable tokens of largest logit
+    """Per-sequence keep set R (Eq. 6): the K routable tokens of largest logit
     (ties to the lower index, -0.0 == +0.0) plus every token outside [r0, r1).
 
     Returns idx int32 [B, k_tot] (ascending token order) and mask uint8 [B, N].
@@ -181,7 +196,7 @@ def routed_ffn(X: np.ndarray, Wg: np.ndarray, Wu: np.ndarray, WdT: np.ndarray,
 
     y = sum_{c in Cs} WdT[c, :] * SiLU(Wg[c] . x) * (Wu[c] . x), with WdT the
     down projection stored channel-major (row c is W_down[:, c], the vector whose
-    norm enters the saliency of Eq. 5).
+    norm enters the saliency of Eq. 8).
     """
     cs = np.asarray(chan, dtype=np.int64)
     x = bf16_to_f64(X)
@@ -211,3 +226,92 @@ def routed_block(h, W1, w2, b1, t, task, r0, r1, K, Wg, Wu, WdT, chan,
     Y = routed_ffn(X, Wg, Wu, WdT, chan)
     out = scatter_add(h, idx, Y)
     return {"logits": logits, "idx": idx, "mask": mask, "Y": Y, "out": out}
+
+
+# ---------------------------------------------------------------- UCS statistics
+
+def drop_set(mask_row: np.ndarray, r0: int, r1: int) -> np.ndarray:
+    """D: the routable tokens [r0, r1) that are not kept (bool over [0, N))."""
+    d = np.zeros(mask_row.shape[0], dtype=bool)
+    d[r0:r1] = np.asarray(mask_row[r0:r1]) == 0
+    return d
+
+
+def drop_jaccard(mask_t, mask_ref, r0, r1):
+    """Eq. 10 per sequence: |D_t & D_ref| / |D_t | D_ref|; also returns the counts
+    (|D_t|, |D_ref|, |D_t & D_ref|)."""
+    mask_t, mask_ref = np.atleast_2d(mask_t), np.atleast_2d(mask_ref)
+    B = mask_t.shape[0]
+    J = np.empty(B)
+    counts = np.empty((B, 3), dtype=np.int64)
+    for b in range(B):
+        Dt, Dr = drop_set(mask_t[b], r0, r1), drop_set(mask_ref[b], r0, r1)
+        inter, union = int(np.sum(Dt & Dr)), int(np.sum(Dt | Dr))
+        J[b] = 1.0 if union == 0 else inter / union
+        counts[b] = (int(Dt.sum()), int(Dr.sum()), inter)
+    return J, counts
+
+
+def expected_random_jaccard(a: int, b: int, n: int) -> float:
+    """J_rand of Eq. 11 (reading): E|A&B| / E|A|B| for uniformly random drop sets
+    of sizes a and b among n tokens, E|A&B| = a b / n."""
+    if a + b == 0 or n == 0:
+        return 1.0
+    e = a * b / n
+    return e / ((a + b) - e)
+
+
+def rda(J: float, J_rand: float) -> float:
+    """Eq. 11: (J - J_rand) / (1 - J_rand); J_rand = 1 gives 1 (identical patterns)."""
+    if J_rand == 1.0:
+        return 1.0
+    return (J - J_rand) / (1.0 - J_rand)
+
+
+def drop_set_stats(mask_t, mask_ref, r0, r1):
+    """Per sequence (J, J_rand, RDA) in fp64."""
+    J, counts = drop_jaccard(mask_t, mask_ref, r0, r1)
+    n = r1 - r0
+    Jr = np.array([expected_random_jaccard(int(c[0]), int(c[1]), n) for c in counts])
+    R = np.array([rda(J[b], Jr[b]) for b in range(len(J))])
+    return J, Jr, R, counts
+
+
+def cosine(a: np.ndarray, b: np.ndarray) -> float:
+    na, nb = float(np.sqrt(np.dot(a, a))), float(np.sqrt(np.dot(b, b)))
+    if na == 0.0 or nb == 0.0:
+        return 1.0 if np.array_equal(a, b) else 0.0
+    return float(np.dot(a, b)) / (na * nb)
+
+
+def redundancy_gap(h_in, h_out, mask):
+    """Eq. 7 per sequence: g = mean_all cos(h_in_i, h_out_i) - mean_{i in R} cos(...).
+
+    h_in, h_out: bf16 bits [B, N, d]; mask: uint8 [B, N] (1 = retained)."""
+    a, o = bf16_to_f64(h_in), bf16_to_f64(h_out)
+    B, N, _ = a.shape
+    g = np.empty(B)
+    for b in range(B):
+        cos = np.array([cosine(a[b, i], o[b, i]) for i in range(N)])
+        kept = np.asarray(mask[b]) != 0
+        g[b] = 0.0 if not kept.any() else cos.mean() - cos[kept].mean()
+    return g
+
+
+def ffn_saliency(X, Wg, Wu, WdT):
+    """Eq. 8 over all I channels: s_c = mean_{i in R} |z_{i,c}| * ||W_down[:, c]||_2,
+    z the SwiGLU activation SiLU(Wg x) * (Wu x) of retained row x (rows of X)."""
+    x = bf16_to_f64(X)
+    g = x @ bf16_to_f64(Wg).T
+    u = x @ bf16_to_f64(Wu).T
+    with np.errstate(over="ignore"):
+        z = g / (1.0 + np.exp(-g)) * u
+    col_norm = np.sqrt(np.sum(bf16_to_f64(WdT) ** 2, axis=1))     # ||W_down[:, c]|| = ||WdT[c]||
+    return np.abs(z).mean(axis=0) * col_norm
+
+
+def ffn_leakage(saliency: np.ndarray, pruned) -> float:
+    """Eq. 9: the share of the total saliency held by the channels the static
+    mask proposes to remove."""
+    total = float(np.sum(saliency))
+    return float(np.sum(saliency[np.asarray(pruned, dtype=np.int64)])) / total if total > 0 else 0.0

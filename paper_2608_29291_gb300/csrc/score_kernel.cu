@@ -1,5 +1,5 @@
 // score_kernel.cu -- S1: routing logits of the core and expansion scorers
-// (Sec. 3.2, Eq. 1) on tcgen05 tensor cores.
+// (Sec. 3.2, Eq. 4, core_expansion_formulation) on tcgen05 tensor cores.
 //
 // The hidden layers of the core scorer and of the active expansion scorer are
 // one GEMM, h [B*N, d] x [W1 ; W1e[m(t_b)]]^T, split into BN-wide hidden

@@ -1,5 +1,5 @@
 // topk_kernel.cu -- S2: the per-sequence keep set R = TopK(sigmoid(l), K) of
-// Eq. 4 (Sec. 3.4), computed exactly on the fp32 logits (the sigmoid is
+// Eq. 6 (router_inference_outputs, Sec. 3.4), computed exactly on the fp32 logits (the sigmoid is
 // monotonic, App. B.2).
 //
 // One 1024-thread CTA per sequence keeps the N order-preserving 32-bit keys in

@@ -435,3 +435,120 @@ def test_pins_catch_planted_mistake(name, monkeypatch):
 def test_pins_pass_unmutated():
     assert _all_pin_failures() == []
 
+
+
+# ------------------------------------------------------------------ UCS statistics (Sec. 3.4)
+
+def test_drop_jaccard_and_rda_hand_examples():
+    """Eq. 10 / Eq. 11 by hand.  N = 6, routable [1, 5): tokens 0 and 5 are never dropped."""
+    m_t = np.array([[1, 0, 0, 1, 1, 1]], np.uint8)     # D_t = {1, 2}
+    m_ref = np.array([[0, 0, 1, 0, 1, 0]], np.uint8)   # D_ref = {1, 3} (0 and 5 not routable)
+    J, Jr, R, counts = ora.drop_set_stats(m_t, m_ref, 1, 5)
+    assert counts[0].tolist() == [2, 2, 1]
+    assert J[0] == 1 / 3                      # |{1}| / |{1, 2, 3}|
+    assert abs(Jr[0] - 1 / 3) < 1e-15         # E|A&B| = 2*2/4 = 1, E|A|B| = 4 - 1 = 3
+    assert abs(R[0]) < 1e-15                  # exactly chance level
+    J, Jr, R, _ = ora.drop_set_stats(m_t, m_t, 1, 5)
+    assert J[0] == 1.0 and R[0] == 1.0        # identical drop sets
+    m_dis = np.array([[1, 1, 1, 0, 0, 1]], np.uint8)   # D = {3, 4}, disjoint from D_t
+    J, Jr, R, _ = ora.drop_set_stats(m_t, m_dis, 1, 5)
+    assert J[0] == 0.0 and abs(R[0] + 0.5) < 1e-15     # (0 - 1/3) / (1 - 1/3)
+    none = np.ones((1, 6), np.uint8)
+    J, Jr, R, _ = ora.drop_set_stats(none, none, 1, 5)
+    assert J[0] == 1.0 and R[0] == 1.0        # nothing dropped on either side
+
+
+def test_random_jaccard_reading_pieces_by_brute_force():
+    """The J_rand reading is E|A&B| / E|A|B|; both expectations are exact for
+    uniformly random subsets of the given sizes (enumerated here)."""
+    n = 6
+    for a in range(n + 1):
+        for b in range(n + 1):
+            inter, union, cnt = 0, 0, 0
+            for A in itertools.combinations(range(n), a):
+                for B in itertools.combinations(range(n), b):
+                    sa, sb = set(A), set(B)
+                    inter += len(sa & sb)
+                    union += len(sa | sb)
+                    cnt += 1
+            e_i, e_u = inter / cnt, union / cnt
+            assert abs(e_i - a * b / n) < 1e-12
+            assert abs(e_u - (a + b - a * b / n)) < 1e-12
+            want = 1.0 if a + b == 0 else e_i / e_u
+            assert abs(ora.expected_random_jaccard(a, b, n) - want) < 1e-12
+
+
+def test_drop_jaccard_invariants():
+    rng = np.random.default_rng(21)
+    for _ in range(50):
+        N = int(rng.integers(1, 40))
+        r0 = int(rng.integers(0, N))
+        r1 = int(rng.integers(r0, N + 1))
+        a = rng.integers(0, 2, (2, N)).astype(np.uint8)
+        b = rng.integers(0, 2, (2, N)).astype(np.uint8)
+        J1, _, R1, _ = ora.drop_set_stats(a, b, r0, r1)
+        J2, _, R2, _ = ora.drop_set_stats(b, a, r0, r1)
+        assert np.array_equal(J1, J2) and np.allclose(R1, R2)      # symmetric
+        assert np.all((J1 >= 0) & (J1 <= 1)) and np.all(R1 <= 1 + 1e-12)
+        a2 = a.copy()
+        a2[:, :r0] ^= 1
+        a2[:, r1:] ^= 1
+        assert np.array_equal(ora.drop_set_stats(a2, b, r0, r1)[0], J1)   # non-routable tokens ignored
+
+
+def test_redundancy_gap_hand_example_and_identity():
+    """Eq. 7 by hand: cos = [1, 0, 1], R = {1, 2}: g = 2/3 - 1/2 = 1/6."""
+    h_in = _bits([[[1, 0], [0, 1], [1, 1]]])
+    h_out = _bits([[[1, 0], [1, 0], [1, 1]]])
+    g = ora.redundancy_gap(h_in, h_out, np.array([[0, 1, 1]], np.uint8))
+    assert abs(g[0] - 1 / 6) < 1e-15
+    g = ora.redundancy_gap(h_in, h_in, np.array([[1, 0, 1]], np.uint8))
+    assert abs(g[0]) < 1e-15                               # unchanged layer: no gap (fp64 rounding of sqrt 2)
+    g = ora.redundancy_gap(h_in, h_out, np.array([[0, 0, 0]], np.uint8))
+    assert g[0] == 0.0                                     # empty retained set
+    assert ora.cosine(np.zeros(3), np.zeros(3)) == 1.0 and ora.cosine(np.zeros(3), np.ones(3)) == 0.0
+
+
+def test_cosine_matches_torch_library():
+    rng = np.random.default_rng(22)
+    a, b = rng.normal(size=(2, 50, 33))
+    want = F.cosine_similarity(torch.tensor(a), torch.tensor(b), dim=1).numpy()
+    got = np.array([ora.cosine(a[i], b[i]) for i in range(50)])
+    assert np.allclose(got, want, rtol=1e-13, atol=1e-14)
+
+
+def test_ffn_saliency_and_leakage_hand_example():
+    """Eq. 8 / Eq. 9 by hand, SiLU arguments only 0 and +-1: rows x = e1, e2;
+    z = [[2s, 0, 0], [0, 0, s]] (s = sigma(1)); mean |z| = [s, 0, s/2];
+    ||W_down[:, c]|| = [5, 1, 2] -> saliency [5s, 0, s]."""
+    s = 0.7310585786300049
+    X = _bits([[1, 0], [0, 1]])
+    Wg = _bits([[1, 0], [0, 0], [-1, 1]])
+    Wu = _bits([[2, 0], [1, 1], [0, 1]])
+    WdT = _bits([[3, 4], [1, 0], [0, 2]])
+    sal = ora.ffn_saliency(X, Wg, Wu, WdT)
+    assert np.allclose(sal, [5 * s, 0.0, s], rtol=0, atol=1e-15)
+    assert abs(ora.ffn_leakage(sal, [2]) - 1 / 6) < 1e-15
+    assert ora.ffn_leakage(sal, [1]) == 0.0
+    assert abs(ora.ffn_leakage(sal, [0, 2]) - 1.0) < 1e-15
+    assert ora.ffn_leakage(sal, []) == 0.0
+
+
+def test_zero_leakage_means_pruned_ffn_equals_full_ffn():
+    """If the channels proposed for removal carry no saliency (Eq. 9 gives 0),
+    removing them leaves the FFN output on the retained rows unchanged."""
+    rng = np.random.default_rng(23)
+    M, d, I = 6, 16, 12
+    X = gen.f32_to_bf16_bits(rng.normal(0, 1, (M, d)).astype(np.float32))
+    Wg, Wu, WdT = (gen.f32_to_bf16_bits(rng.normal(0, .3, (I, d)).astype(np.float32)) for _ in range(3))
+    P = np.array([1, 4, 7])
+    WdT[P] = 0                                    # ||W_down[:, c]|| = 0 for c in P
+    sal = ora.ffn_saliency(X, Wg, Wu, WdT)
+    assert ora.ffn_leakage(sal, P) == 0.0
+    keep = np.setdiff1d(np.arange(I), P).astype(np.int32)
+    assert np.allclose(ora.routed_ffn(X, Wg, Wu, WdT, keep), ora.routed_ffn(X, Wg, Wu, WdT, np.arange(I)),
+                       rtol=1e-13, atol=1e-13)
+    # and scaling a down-projection row by 2 scales that channel's saliency by 2
+    W2 = WdT.copy()
+    W2[0] = gen.f32_to_bf16_bits(ora.bf16_to_f64(WdT[0]).astype(np.float32) * 2)
+    assert abs(ora.ffn_saliency(X, Wg, Wu, W2)[0] - 2 * sal[0]) < 1e-12 * max(1, sal[0])
