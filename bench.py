@@ -143,6 +143,47 @@ def workload_config(w: gen.Workload, flush: bool) -> dict:
             "inputs": "seeded synthetic (SplitMix64 normals), resident in HBM"}
 
 
+def measure_ucs(cer, torch, w, h0, h, flush, stream, dev, core, exp, t, Wg, Wu, WdT, ws, reps=20):
+    """Time the UCS statistics kernels on the workload's own tensors: the keep
+    masks of two block calls (t and t_ref = the same inputs with t + 0.05) and
+    the redundancy gap of the block's input and output."""
+    masks = []
+    for dt in (0.0, 0.05):
+        h.copy_(h0)
+        m = torch.empty((w.B, w.N), dtype=torch.uint8, device=dev)
+        cer.cer_routed_block(h, core, exp, (t + dt).clamp(max=1.0), w.task, w.r0, w.r1, w.K, Wg, Wu, WdT, None,
+                             mask=m, ws=ws, stream=stream)
+        masks.append(m)
+    jac = torch.empty(w.B, dtype=torch.float32, device=dev)
+    rda = torch.empty_like(jac)
+    gap = torch.empty_like(jac)
+    skip = torch.empty(w.B, dtype=torch.uint8, device=dev)
+    gws = cer.workspace(cer.load().cer_redundancy_gap_workspace_size(w.B, w.N), dev)
+
+    def timed(fn):
+        ms = []
+        for i in range(reps + 3):
+            flush.fill_(float(i))
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            fn()
+            b.record(stream)
+            b.synchronize()
+            if i >= 3:
+                ms.append(a.elapsed_time(b))
+        return float(np.mean(ms))
+
+    t_drop = timed(lambda: cer.cer_drop_set_stats(masks[0], masks[1], w.r0, w.r1, jac, None, rda, stream=stream))
+    t_gap = timed(lambda: cer.cer_redundancy_gap(h0, h, masks[1], 0.004, gap, skip, ws=gws, stream=stream))
+    cer.cer_sync_status(stream)
+    gap_bytes = 2.0 * w.B * w.N * w.d * 2 + w.B * w.N
+    return {"drop_set_stats_us": t_drop * 1e3, "redundancy_gap_us": t_gap * 1e3,
+            "redundancy_gap_gbs": gap_bytes / (t_gap * 1e-3) / 1e9,
+            "jaccard_t_vs_t+0.05": [round(float(x), 4) for x in jac.cpu().numpy()],
+            "rda_t_vs_t+0.05": [round(float(x), 4) for x in rda.cpu().numpy()],
+            "redundancy_gap": [round(float(x), 6) for x in gap.cpu().numpy()]}
+
+
 # ------------------------------------------------------------------ CPU oracle timing
 
 def time_oracle(w: gen.Workload, inp: dict, min_seconds: float, max_reps: int = 50):
@@ -301,6 +342,10 @@ def run_gpu(args, info):
     h2d = h_host.numel() * 2 + t_host.numel() * 4
     d2h = out_host.numel() * 2
 
+    # ---- UCS statistics on this step's tensors (Sec. 3.4): drop-set J/RDA of
+    # two keep masks, redundancy gap of the block's input and output
+    ucs = measure_ucs(cer, torch, w, h0, h, flush, stream, dev, core, exp, t, Wg, Wu, WdT, ws)
+
     if not info.is_root:
         return 0
 
@@ -340,6 +385,8 @@ def run_gpu(args, info):
         "cpu_baseline": cpu,
         "e2e": {"value": tokens / (e2e_ms * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
+        "ucs": {**ucs, "redundancy_gap_hbm_frac": ucs["redundancy_gap_gbs"] / float(peaks["hbm_gbs"]),
+                "peak_source": f"hbm_gbs of {peak_kind}"},
         "gpu_launches": KERNELS_PER_STEP * args.steps,
         "clocks": clocks.summary(),
     }

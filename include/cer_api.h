@@ -213,6 +213,42 @@ cer_status cer_routed_block(void* h, void* out, int B, int N, int d,
 size_t cer_routed_block_workspace_size(int B, int N, int d, int core_hidden, int exp_hidden,
                                        int task, int r0, int r1, int K, int C, int with_chan);
 
+/* ------------------------------------------------------------------ UCS statistics
+ * Signals of Unified Computation Scheduling (Sec. 3.4), computed from the
+ * router's decisions.
+ *
+ * cer_drop_set_stats: drop-set similarity of two routing decisions per
+ * sequence (Eq. 10 and Eq. 11; diffusion-head cache reuse compares t with the
+ * last refresh, early exit compares adjacent steps).  D is the routable tokens
+ * [r0, r1) a keep mask does not keep.
+ *   mask_t, mask_ref  uint8 [B, N] keep masks (1 = kept), e.g. from
+ *                     cer_select_topk or cer_routed_block
+ *   jaccard  fp32 [B]  J = |D_t & D_ref| / |D_t | D_ref| (1 if both empty)
+ *   j_rand   fp32 [B]  expected J of random drop sets of the same sizes among
+ *                      the n = r1 - r0 routable tokens, taken as
+ *                      E|A&B| / E|A|B| with E|A&B| = |A||B|/n; or NULL
+ *   rda      fp32 [B]  (J - J_rand) / (1 - J_rand) (1 if J_rand = 1); or NULL
+ *   counts   int32 [B, 3]  |D_t|, |D_ref|, |D_t & D_ref|; or NULL
+ * The counts are exact; the ratios are formed in fp64 from them.            */
+cer_status cer_drop_set_stats(const uint8_t* mask_t, const uint8_t* mask_ref, int B, int N, int r0, int r1,
+                              float* jaccard, float* j_rand, float* rda, int32_t* counts,
+                              cudaStream_t stream);
+
+/* cer_redundancy_gap: layer-skipping statistic of Eq. 7 per sequence,
+ * g = mean over all tokens of cos(h_in_i, h_out_i) minus the mean over the
+ * retained tokens R (mask 1); skip[b] = (g <= delta), delta_LS = 0.0040 in
+ * App. A.4.
+ *   h_in, h_out  bf16 [B, N, d] (d a multiple of 8), the block's input and output
+ *   mask         uint8 [B, N]
+ *   gap          fp32 [B] output; skip uint8 [B] output or NULL
+ * Cosines accumulate in fp32 per token (a zero-norm pair counts 1 if equal,
+ * else 0); the means are fp64.  Empty R gives g = 0.
+ * Workspace: cer_redundancy_gap_workspace_size(B, N).                      */
+cer_status cer_redundancy_gap(const void* h_in, const void* h_out, const uint8_t* mask, int B, int N, int d,
+                              float delta, float* gap, uint8_t* skip,
+                              void* workspace, size_t workspace_bytes, cudaStream_t stream);
+size_t cer_redundancy_gap_workspace_size(int B, int N);
+
 /* ------------------------------------------------------------------ status
  * cer_sync_status: synchronise `stream`, then return and clear the current
  * device's status word (the first kernel-detected error since the last call),

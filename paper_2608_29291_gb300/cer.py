@@ -28,7 +28,8 @@ STATUS_NAMES = {0: "CER_OK", 1: "CER_ERR_NULL", 2: "CER_ERR_SHAPE", 3: "CER_ERR_
 # Every symbol include/cer_api.h declares.
 EXPORTS = ("cer_score", "cer_score_workspace_size", "cer_score_static", "cer_select_topk", "cer_gather", "cer_routed_ffn",
            "cer_routed_ffn_workspace_size", "cer_pack_ffn_weights", "cer_scatter_add", "cer_routed_block",
-           "cer_routed_block_workspace_size", "cer_sync_status", "cer_get_error", "cer_status_string",
+           "cer_routed_block_workspace_size", "cer_drop_set_stats", "cer_redundancy_gap",
+           "cer_redundancy_gap_workspace_size", "cer_sync_status", "cer_get_error", "cer_status_string",
            "cer_version")
 
 
@@ -61,6 +62,9 @@ _SIGS = {
     "cer_routed_block": ([_vp, _vp, _i, _i, _i, _SCP, _SCP, _vp, _i, _i, _i, _i, _vp, _vp, _vp, _i, _vp, _i,
                           _vp, _vp, _vp, _vp, _sz, _vp, _i, _vp], _i),
     "cer_routed_block_workspace_size": ([_i, _i, _i, _i, _i, _i, _i, _i, _i, _i, _i], _sz),
+    "cer_drop_set_stats": ([_vp, _vp, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _vp], _i),
+    "cer_redundancy_gap": ([_vp, _vp, _vp, _i, _i, _i, _f, _vp, _vp, _vp, _sz, _vp], _i),
+    "cer_redundancy_gap_workspace_size": ([_i, _i], _sz),
     "cer_sync_status": ([_vp], _i),
     "cer_get_error": ([], ctypes.c_char_p),
     "cer_status_string": ([_i], ctypes.c_char_p),
@@ -219,6 +223,20 @@ def cer_routed_block(h, core: Scorer, exp: Optional[Scorer], t, task, r0, r1, K,
     _check(load().cer_routed_block(_p(h), _p(out), B, N, d, _sref(core), _sref(exp), _p(t), task, r0, r1, K,
                                    _p(Wg), _p(Wu), _p(WdT), I, _p(chan), C, _p(logits), _p(idx), _p(mask),
                                    _p(ws), ws.numel(), ev_arr, n_ev, _stream(stream)))
+
+
+def cer_drop_set_stats(mask_t, mask_ref, r0, r1, jaccard, j_rand=None, rda=None, counts=None, stream=None):
+    B, N = mask_t.shape
+    _check(load().cer_drop_set_stats(_p(mask_t), _p(mask_ref), B, N, r0, r1, _p(jaccard), _p(j_rand), _p(rda),
+                                     _p(counts), _stream(stream)))
+
+
+def cer_redundancy_gap(h_in, h_out, mask, delta, gap, skip=None, ws=None, stream=None):
+    B, N, d = h_in.shape
+    if ws is None:
+        ws = workspace(load().cer_redundancy_gap_workspace_size(B, N), h_in.device)
+    _check(load().cer_redundancy_gap(_p(h_in), _p(h_out), _p(mask), B, N, d, float(delta), _p(gap), _p(skip),
+                                     _p(ws), ws.numel(), _stream(stream)))
 
 
 def cer_sync_status(stream=None) -> None:

@@ -645,4 +645,60 @@ cer_status cer_routed_block(void* h, void* out, int B, int N, int d, const cer_s
   return CER_OK;
 }
 
+cer_status cer_drop_set_stats(const uint8_t* mask_t, const uint8_t* mask_ref, int B, int N, int r0, int r1,
+                              float* jaccard, float* j_rand, float* rda, int32_t* counts, cudaStream_t stream) {
+  const bool any = static_cast<long long>(B) * N > 0;
+  CER_PTR_IF(mask_t, any);
+  CER_PTR_IF(mask_ref, any);
+  CER_PTR_IF(jaccard, B > 0);
+  CER_ALIGN(mask_t);
+  CER_ALIGN(mask_ref);
+  CER_ALIGN(jaccard);
+  CER_ALIGN(j_rand);
+  CER_ALIGN(rda);
+  CER_ALIGN(counts);
+  CER_REQUIRE(B >= 0 && N >= 0, CER_ERR_SHAPE, "B=%d N=%d must be >= 0", B, N);
+  CER_REQUIRE(0 <= r0 && r0 <= r1 && r1 <= N, CER_ERR_RANGE, "routable range [%d, %d) not inside [0, %d]", r0, r1, N);
+  DeviceInfo* dev = nullptr;
+  cer_status s = device_info(&dev);
+  if (s != CER_OK) return s;
+  cudaError_t e = cer::launch_drop_stats(mask_t, mask_ref, B, N, r0, r1, jaccard, j_rand, rda, counts, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "drop-set statistics launch");
+  return CER_OK;
+}
+
+size_t cer_redundancy_gap_workspace_size(int B, int N) {
+  if (B < 0 || N < 0) return 0;
+  return round256(static_cast<size_t>(B) * N * sizeof(float));
+}
+
+cer_status cer_redundancy_gap(const void* h_in, const void* h_out, const uint8_t* mask, int B, int N, int d,
+                              float delta, float* gap, uint8_t* skip, void* workspace, size_t workspace_bytes,
+                              cudaStream_t stream) {
+  const bool any = static_cast<long long>(B) * N > 0;
+  CER_PTR_IF(h_in, any);
+  CER_PTR_IF(h_out, any);
+  CER_PTR_IF(mask, any);
+  CER_PTR_IF(gap, B > 0);
+  CER_ALIGN(h_in);
+  CER_ALIGN(h_out);
+  CER_ALIGN(mask);
+  CER_ALIGN(gap);
+  CER_ALIGN(skip);
+  CER_ALIGN(workspace);
+  CER_REQUIRE(B >= 0 && N >= 0, CER_ERR_SHAPE, "B=%d N=%d must be >= 0", B, N);
+  CER_REQUIRE(d > 0 && d % 8 == 0, CER_ERR_SHAPE, "d=%d must be a positive multiple of 8", d);
+  const size_t need = cer_redundancy_gap_workspace_size(B, N);
+  CER_REQUIRE(!any || (workspace != nullptr && workspace_bytes >= need), CER_ERR_WORKSPACE,
+              "workspace of %zu bytes needed, %zu given", need, workspace_bytes);
+  DeviceInfo* dev = nullptr;
+  cer_status s = device_info(&dev);
+  if (s != CER_OK) return s;
+  cudaError_t e = cer::launch_redundancy_gap(static_cast<const __nv_bfloat16*>(h_in),
+                                             static_cast<const __nv_bfloat16*>(h_out), mask, B, N, d, delta, gap,
+                                             skip, static_cast<float*>(workspace), dev->n_sm, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "redundancy-gap launch");
+  return CER_OK;
+}
+
 }  // extern "C"

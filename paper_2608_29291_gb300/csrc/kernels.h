@@ -106,4 +106,11 @@ struct FfnArgs {
 cudaError_t launch_ffn_gateup(const FfnArgs& a, int n_sm, cudaStream_t stream);
 cudaError_t launch_ffn_down(const FfnArgs& a, int n_sm, cudaStream_t stream);
 
+// ------------------------------------------------------------------ UCS statistics
+cudaError_t launch_drop_stats(const uint8_t* mask_t, const uint8_t* mask_ref, int B, int N, int r0, int r1,
+                              float* jac, float* jrand, float* rda, int32_t* counts, cudaStream_t stream);
+cudaError_t launch_redundancy_gap(const __nv_bfloat16* h_in, const __nv_bfloat16* h_out, const uint8_t* mask,
+                                  int B, int N, int d, float delta, float* gap, uint8_t* skip, float* cos_ws,
+                                  int n_sm, cudaStream_t stream);
+
 }  // namespace cer
