@@ -143,10 +143,12 @@ def workload_config(w: gen.Workload, flush: bool) -> dict:
             "inputs": "seeded synthetic (SplitMix64 normals), resident in HBM"}
 
 
-def measure_ucs(cer, torch, w, h0, h, flush, stream, dev, core, exp, t, Wg, Wu, WdT, ws, reps=20):
-    """Time the UCS statistics kernels on the workload's own tensors: the keep
-    masks of two block calls (t and t_ref = the same inputs with t + 0.05) and
-    the redundancy gap of the block's input and output."""
+def measure_ucs(cer, torch, w, h0, h, flush, stream, dev, core, exp, t, Wg, Wu, WdT, ws, inp, reps=20):
+    """Time the UCS kernels on the workload's own tensors: the keep masks of two
+    block calls (t and t_ref = the same inputs with t + 0.05), the redundancy
+    gap of the block's input and output, and the whole block with the FFN gate
+    (gate/up over all I channels, leakage of the mask's pruned channels,
+    delta_FFN = 0.150 as in App. A.4)."""
     masks = []
     for dt in (0.0, 0.05):
         h.copy_(h0)
@@ -176,12 +178,42 @@ def measure_ucs(cer, torch, w, h0, h, flush, stream, dev, core, exp, t, Wg, Wu, 
     t_drop = timed(lambda: cer.cer_drop_set_stats(masks[0], masks[1], w.r0, w.r1, jac, None, rda, stream=stream))
     t_gap = timed(lambda: cer.cer_redundancy_gap(h0, h, masks[1], 0.004, gap, skip, ws=gws, stream=stream))
     cer.cer_sync_status(stream)
+    gated = {}
+    if w.C < w.I and w.I % 64 == 0:
+        def bf(bits):
+            return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).to(dev)
+        Wg_g, Wu_g, WdT_g, norms, _ = cer.gate_weights(bf(inp["Wg"]), bf(inp["Wu"]), bf(inp["WdT"]),
+                                                       torch.from_numpy(inp["chan"]).to(dev))
+        leak = torch.empty(1, dtype=torch.float32, device=dev)
+        flag = torch.empty(1, dtype=torch.uint8, device=dev)
+        gws2 = cer.workspace(cer.load().cer_routed_block_gated_workspace_size(
+            w.B, w.N, w.d, w.Hc, w.He if w.task else 0, w.task, w.r0, w.r1, w.K, w.I), dev)
+
+        def gated_step():
+            h.copy_(h0)
+            flush.fill_(1.0)
+
+        ms = []
+        for i in range(reps + 3):
+            gated_step()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            cer.cer_routed_block_gated(h, core, exp, t, w.task, w.r0, w.r1, w.K, Wg_g, Wu_g, WdT_g, w.C, norms,
+                                       0.150, None, leak, flag, ws=gws2, stream=stream)
+            b.record(stream)
+            b.synchronize()
+            if i >= 3:
+                ms.append(a.elapsed_time(b))
+        cer.cer_sync_status(stream)
+        gated = {"gated_block_ms": float(np.mean(ms)), "gated_block_tokens_per_s": w.B * w.N / (np.mean(ms) * 1e-3),
+                 "ffn_leakage": round(float(leak.item()), 5), "pruned_ffn_taken": bool(flag.item()),
+                 "delta_ffn": 0.150}
     gap_bytes = 2.0 * w.B * w.N * w.d * 2 + w.B * w.N
     return {"drop_set_stats_us": t_drop * 1e3, "redundancy_gap_us": t_gap * 1e3,
             "redundancy_gap_gbs": gap_bytes / (t_gap * 1e-3) / 1e9,
             "jaccard_t_vs_t+0.05": [round(float(x), 4) for x in jac.cpu().numpy()],
             "rda_t_vs_t+0.05": [round(float(x), 4) for x in rda.cpu().numpy()],
-            "redundancy_gap": [round(float(x), 6) for x in gap.cpu().numpy()]}
+            "redundancy_gap": [round(float(x), 6) for x in gap.cpu().numpy()], **gated}
 
 
 # ------------------------------------------------------------------ CPU oracle timing
@@ -344,7 +376,7 @@ def run_gpu(args, info):
 
     # ---- UCS statistics on this step's tensors (Sec. 3.4): drop-set J/RDA of
     # two keep masks, redundancy gap of the block's input and output
-    ucs = measure_ucs(cer, torch, w, h0, h, flush, stream, dev, core, exp, t, Wg, Wu, WdT, ws)
+    ucs = measure_ucs(cer, torch, w, h0, h, flush, stream, dev, core, exp, t, Wg, Wu, WdT, ws, inp)
 
     if not info.is_root:
         return 0

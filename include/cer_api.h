@@ -213,6 +213,47 @@ cer_status cer_routed_block(void* h, void* out, int B, int N, int d,
 size_t cer_routed_block_workspace_size(int B, int N, int d, int core_hidden, int exp_hidden,
                                        int task, int r0, int r1, int K, int C, int with_chan);
 
+/* ------------------------------------------------------------------ UCS FFN gate
+ * FFN pruning of Unified Computation Scheduling (Sec. 3.4 (2), Eq. 8 and
+ * Eq. 9; App. A.4: delta_FFN = 0.150).  The static mask proposes a pruned
+ * channel set P; per call, the saliency of every channel on the retained rows,
+ *   s_c = mean_i |z_{i,c}| * ||W_down[:, c]||_2,
+ * gives the leakage lambda = sum_{c in P} s_c / sum_c s_c, and the pruned FFN
+ * runs only if lambda <= delta (else the full FFN).  The saliency needs the
+ * activation of every channel, so the gate/up GEMM runs over all I channels;
+ * the decision sets how many channels the down GEMM contracts -- on the
+ * device, without a host round trip.  One decision per call, over every
+ * retained row of the batch (one sequence per call gives the per-sample rule).
+ *
+ * Weights: Wg, Wu, WdT bf16 [I, d] holding all channels with the C_keep
+ * kept channels first and the mask's pruned channels after (pack once with
+ * cer_pack_ffn_weights and that permutation as chan); norms fp32 [I] the
+ * W_down column norms in the same order (cer_ffn_channel_norms, once).
+ * I and C_keep multiples of 64.  Outputs: saliency fp32 [I] or NULL, leakage
+ * fp32 [1] or NULL, use_pruned uint8 [1] (1 = pruned FFN ran) or NULL.     */
+cer_status cer_ffn_channel_norms(const void* WdT, int I, int d, float* norms, cudaStream_t stream);
+
+cer_status cer_routed_ffn_gated(const void* X, int M, int d,
+                                const void* Wg, const void* Wu, const void* WdT, int I, int C_keep,
+                                const float* norms, float delta, void* Y,
+                                float* saliency, float* leakage, uint8_t* use_pruned,
+                                void* workspace, size_t workspace_bytes, cudaStream_t stream);
+size_t cer_routed_ffn_gated_workspace_size(int M, int d, int I);
+
+/* The fused block with the gate (arguments as for cer_routed_block and the
+ * gated FFN above; stage event 4 follows the gate/up GEMM and the gate).   */
+cer_status cer_routed_block_gated(void* h, void* out, int B, int N, int d,
+                                  const cer_scorer* core, const cer_scorer* exp,
+                                  const float* t, int task, int r0, int r1, int K,
+                                  const void* Wg, const void* Wu, const void* WdT, int I, int C_keep,
+                                  const float* norms, float delta,
+                                  float* saliency, float* leakage, uint8_t* use_pruned,
+                                  float* logits, int32_t* idx, uint8_t* mask,
+                                  void* workspace, size_t workspace_bytes,
+                                  cudaEvent_t* stage_events, int n_stage_events, cudaStream_t stream);
+size_t cer_routed_block_gated_workspace_size(int B, int N, int d, int core_hidden, int exp_hidden,
+                                             int task, int r0, int r1, int K, int I);
+
 /* ------------------------------------------------------------------ UCS statistics
  * Signals of Unified Computation Scheduling (Sec. 3.4), computed from the
  * router's decisions.

@@ -28,7 +28,9 @@ STATUS_NAMES = {0: "CER_OK", 1: "CER_ERR_NULL", 2: "CER_ERR_SHAPE", 3: "CER_ERR_
 # Every symbol include/cer_api.h declares.
 EXPORTS = ("cer_score", "cer_score_workspace_size", "cer_score_static", "cer_select_topk", "cer_gather", "cer_routed_ffn",
            "cer_routed_ffn_workspace_size", "cer_pack_ffn_weights", "cer_scatter_add", "cer_routed_block",
-           "cer_routed_block_workspace_size", "cer_drop_set_stats", "cer_redundancy_gap",
+           "cer_routed_block_workspace_size", "cer_ffn_channel_norms", "cer_routed_ffn_gated",
+           "cer_routed_ffn_gated_workspace_size", "cer_routed_block_gated", "cer_routed_block_gated_workspace_size",
+           "cer_drop_set_stats", "cer_redundancy_gap",
            "cer_redundancy_gap_workspace_size", "cer_sync_status", "cer_get_error", "cer_status_string",
            "cer_version")
 
@@ -62,6 +64,12 @@ _SIGS = {
     "cer_routed_block": ([_vp, _vp, _i, _i, _i, _SCP, _SCP, _vp, _i, _i, _i, _i, _vp, _vp, _vp, _i, _vp, _i,
                           _vp, _vp, _vp, _vp, _sz, _vp, _i, _vp], _i),
     "cer_routed_block_workspace_size": ([_i, _i, _i, _i, _i, _i, _i, _i, _i, _i, _i], _sz),
+    "cer_ffn_channel_norms": ([_vp, _i, _i, _vp, _vp], _i),
+    "cer_routed_ffn_gated": ([_vp, _i, _i, _vp, _vp, _vp, _i, _i, _vp, _f, _vp, _vp, _vp, _vp, _vp, _sz, _vp], _i),
+    "cer_routed_ffn_gated_workspace_size": ([_i, _i, _i], _sz),
+    "cer_routed_block_gated": ([_vp, _vp, _i, _i, _i, _SCP, _SCP, _vp, _i, _i, _i, _i, _vp, _vp, _vp, _i, _i, _vp,
+                                _f, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp, _i, _vp], _i),
+    "cer_routed_block_gated_workspace_size": ([_i, _i, _i, _i, _i, _i, _i, _i, _i, _i], _sz),
     "cer_drop_set_stats": ([_vp, _vp, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _vp], _i),
     "cer_redundancy_gap": ([_vp, _vp, _vp, _i, _i, _i, _f, _vp, _vp, _vp, _sz, _vp], _i),
     "cer_redundancy_gap_workspace_size": ([_i, _i], _sz),
@@ -211,18 +219,67 @@ def cer_routed_block(h, core: Scorer, exp: Optional[Scorer], t, task, r0, r1, K,
     if ws is None:
         ws = workspace(cer_routed_block_workspace_size(B, N, d, core.W1.shape[-2], eh, task, r0, r1, K, C,
                                                        chan is not None), h.device)
-    ev_arr, n_ev = None, 0
-    if stage_events is not None:
-        handles = []
-        for ev in stage_events:
-            if ev.cuda_event == 0:     # torch creates the event lazily: force it
-                ev.record()
-            handles.append(ev.cuda_event)
-        ev_arr = (ctypes.c_void_p * len(handles))(*handles)
-        n_ev = len(handles)
+    ev_arr, n_ev = _event_array(stage_events)
     _check(load().cer_routed_block(_p(h), _p(out), B, N, d, _sref(core), _sref(exp), _p(t), task, r0, r1, K,
                                    _p(Wg), _p(Wu), _p(WdT), I, _p(chan), C, _p(logits), _p(idx), _p(mask),
                                    _p(ws), ws.numel(), ev_arr, n_ev, _stream(stream)))
+
+
+def _event_array(stage_events):
+    if stage_events is None:
+        return None, 0
+    handles = []
+    for ev in stage_events:
+        if ev.cuda_event == 0:     # torch creates the event lazily: force it
+            ev.record()
+        handles.append(ev.cuda_event)
+    return (ctypes.c_void_p * len(handles))(*handles), len(handles)
+
+
+def cer_ffn_channel_norms(WdT, norms, stream=None):
+    I, d = WdT.shape
+    _check(load().cer_ffn_channel_norms(_p(WdT), I, d, _p(norms), _stream(stream)))
+
+
+def gate_weights(Wg, Wu, WdT, chan, stream=None):
+    """Weights for the UCS FFN gate: all I channels, the kept ones (chan) first,
+    then the rest in ascending order; plus their W_down column norms."""
+    I = Wg.shape[0]
+    keep = chan.to(torch.int64)
+    rest = torch.ones(I, dtype=torch.bool, device=chan.device)
+    rest[keep] = False
+    perm = torch.cat([keep, torch.nonzero(rest).flatten()]).to(torch.int32).contiguous()
+    Wg_p, Wu_p, WdT_p = pack_ffn_weights(Wg, Wu, WdT, perm, stream=stream)
+    norms = torch.empty(I, dtype=torch.float32, device=Wg.device)
+    cer_ffn_channel_norms(WdT_p, norms, stream=stream)
+    return Wg_p, Wu_p, WdT_p, norms, perm
+
+
+def cer_routed_ffn_gated(X, Wg, Wu, WdT, C_keep, norms, delta, Y, saliency=None, leakage=None, use_pruned=None,
+                         ws=None, stream=None):
+    M, d = X.shape
+    I = Wg.shape[0]
+    if ws is None:
+        ws = workspace(load().cer_routed_ffn_gated_workspace_size(M, d, I), X.device)
+    _check(load().cer_routed_ffn_gated(_p(X), M, d, _p(Wg), _p(Wu), _p(WdT), I, C_keep, _p(norms), float(delta),
+                                       _p(Y), _p(saliency), _p(leakage), _p(use_pruned), _p(ws), ws.numel(),
+                                       _stream(stream)))
+
+
+def cer_routed_block_gated(h, core: Scorer, exp: Optional[Scorer], t, task, r0, r1, K, Wg, Wu, WdT, C_keep, norms,
+                           delta, saliency=None, leakage=None, use_pruned=None, out=None, logits=None, idx=None,
+                           mask=None, ws=None, stage_events=None, stream=None):
+    B, N, d = h.shape
+    I = Wg.shape[0]
+    eh = exp.W1.shape[-2] if exp is not None else 0
+    if ws is None:
+        ws = workspace(load().cer_routed_block_gated_workspace_size(B, N, d, core.W1.shape[-2], eh, task, r0, r1, K,
+                                                                    I), h.device)
+    ev_arr, n_ev = _event_array(stage_events)
+    _check(load().cer_routed_block_gated(_p(h), _p(out), B, N, d, _sref(core), _sref(exp), _p(t), task, r0, r1, K,
+                                         _p(Wg), _p(Wu), _p(WdT), I, C_keep, _p(norms), float(delta), _p(saliency),
+                                         _p(leakage), _p(use_pruned), _p(logits), _p(idx), _p(mask), _p(ws),
+                                         ws.numel(), ev_arr, n_ev, _stream(stream)))
 
 
 def cer_drop_set_stats(mask_t, mask_ref, r0, r1, jaccard, j_rand=None, rda=None, counts=None, stream=None):

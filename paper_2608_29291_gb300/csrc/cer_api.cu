@@ -512,11 +512,63 @@ size_t cer_routed_block_workspace_size(int B, int N, int d, int core_hidden, int
                                                                           static_cast<int>(M), d, C, with_chan);
 }
 
-cer_status cer_routed_block(void* h, void* out, int B, int N, int d, const cer_scorer* core, const cer_scorer* exp,
-                            const float* t, int task, int r0, int r1, int K, const void* Wg, const void* Wu,
-                            const void* WdT, int I, const int32_t* chan, int C, float* logits, int32_t* idx,
-                            uint8_t* mask, void* workspace, size_t workspace_bytes, cudaEvent_t* stage_events,
-                            int n_stage_events, cudaStream_t stream) {
+}  // extern "C"
+
+namespace {
+
+// The UCS FFN gate of the fused block (Sec. 3.4 (2)): the FFN weights hold
+// all I channels with the C_keep kept ones first; the gate/up GEMM runs over
+// all of them, Eq. 8 / Eq. 9 give the leakage of the pruned tail, and the
+// down GEMM contracts C_keep or I channels accordingly.
+struct GateArgs {
+  int C_keep;
+  const float* norms;
+  float delta;
+  float* saliency;
+  float* leakage;
+  uint8_t* use_pruned;
+};
+
+size_t gate_ws_bytes(long long M, int I) {
+  const size_t n_parts = 2 * static_cast<size_t>((M + 127) / 128);
+  return round256(n_parts * I * sizeof(float)) + round256(2 * static_cast<size_t>((I + 255) / 256) * sizeof(float)) +
+         256;  // + leakage and decision when the caller passes NULL
+}
+
+cer_status check_gate(const GateArgs* g, int I, int C) {
+  if (g == nullptr) return CER_OK;
+  CER_PTR(g->norms);
+  CER_ALIGN(g->norms);
+  CER_ALIGN(g->saliency);
+  CER_ALIGN(g->leakage);
+  CER_REQUIRE(C == I, CER_ERR_SHAPE, "the gated FFN takes all I channels (C=%d, I=%d)", C, I);
+  CER_REQUIRE(g->C_keep >= 64 && g->C_keep <= I && g->C_keep % 64 == 0, CER_ERR_SHAPE,
+              "C_keep=%d must be a multiple of 64 in [64, I=%d]", g->C_keep, I);
+  return CER_OK;
+}
+
+// Saliency, leakage and the decision from the gate/up GEMM's column sums; the
+// decision flag then drives the down GEMM's contraction length (fa.use_small_k).
+// gate_ws: colsum | per-block partial sums | leakage / decision fallbacks.
+cer_status run_gate(const GateArgs& g, cer::FfnArgs& fa, char* gate_ws, cudaStream_t stream) {
+  const int n_parts = 2 * ((fa.M + 127) / 128);
+  char* p = gate_ws + round256(static_cast<size_t>(n_parts) * fa.C * sizeof(float));
+  float* part_ws = reinterpret_cast<float*>(p);
+  p += round256(2 * static_cast<size_t>((fa.C + 255) / 256) * sizeof(float));
+  float* leak = g.leakage ? g.leakage : reinterpret_cast<float*>(p);
+  uint8_t* flag = g.use_pruned ? g.use_pruned : reinterpret_cast<uint8_t*>(p + 16);
+  cudaError_t e = cer::launch_ffn_gate(fa.colsum, n_parts, fa.M, fa.C, g.C_keep, g.norms, g.delta, g.saliency,
+                                       part_ws, leak, flag, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "FFN gate launch");
+  fa.use_small_k = flag;
+  return CER_OK;
+}
+
+cer_status routed_block_impl(void* h, void* out, int B, int N, int d, const cer_scorer* core, const cer_scorer* exp,
+                             const float* t, int task, int r0, int r1, int K, const void* Wg, const void* Wu,
+                             const void* WdT, int I, const int32_t* chan, int C, float* logits, int32_t* idx,
+                             uint8_t* mask, void* workspace, size_t workspace_bytes, cudaEvent_t* stage_events,
+                             int n_stage_events, const GateArgs* gate, cudaStream_t stream) {
   ScoreShape sh;
   cer_status s = check_score_args(h, B, N, d, core, exp, t, task, &sh);
   if (s != CER_OK) return s;
@@ -540,10 +592,12 @@ cer_status cer_routed_block(void* h, void* out, int B, int N, int d, const cer_s
   CER_REQUIRE(M64 < (1ll << 31), CER_ERR_SHAPE, "too many kept rows");
   s = check_ffn_shape(static_cast<int>(M64), d, I, chan, C);
   if (s != CER_OK) return s;
+  if ((s = check_gate(gate, I, C)) != CER_OK) return s;
+  CER_REQUIRE(gate == nullptr || chan == nullptr, CER_ERR_RANGE, "the gated FFN takes packed weights (chan NULL)");
   CER_REQUIRE(stage_events == nullptr || n_stage_events == 6, CER_ERR_RANGE,
               "stage_events needs exactly 6 events (got %d)", n_stage_events);
-  const size_t need =
-      cer_routed_block_workspace_size(B, N, d, sh.Hc, sh.He, task, r0, r1, K, C, chan != nullptr);
+  const size_t need = cer_routed_block_workspace_size(B, N, d, sh.Hc, sh.He, task, r0, r1, K, C, chan != nullptr) +
+                      (gate ? gate_ws_bytes(M64, I) : 0);
   CER_REQUIRE(workspace != nullptr && workspace_bytes >= need, CER_ERR_WORKSPACE,
               "workspace of %zu bytes needed, %zu given", need, workspace_bytes);
   const bool in_place = (out == nullptr || out == h);
@@ -579,6 +633,7 @@ cer_status cer_routed_block(void* h, void* out, int B, int N, int d, const cer_s
   ws += round256(static_cast<size_t>(M64) * d * 2);
   __nv_bfloat16* act = reinterpret_cast<__nv_bfloat16*>(ws);
   ws += round256(static_cast<size_t>(M64) * C * 2);
+  char* gate_ws = ws + (chan ? 3 * round256(static_cast<size_t>(C) * d * 2) : 0);
 
   // S1: scorer GEMM -> partial sums
   cer::ScoreArgs sa = make_score_args(h, B, N, d, core, exp, t, sh, dev->status);
@@ -630,9 +685,16 @@ cer_status cer_routed_block(void* h, void* out, int B, int N, int d, const cer_s
   fa.k_tot = k_tot;
   fa.scatter = 1;
   fa.status = dev->status;
+  if (gate) {
+    fa.colsum = reinterpret_cast<float*>(gate_ws);
+    fa.C_small = gate->C_keep;
+  }
   if (M64 > 0) {
     e = cer::launch_ffn_gateup(fa, dev->n_sm, stream);
     if (e != cudaSuccess) return cuda_fail(e, "gate/up GEMM launch");
+  }
+  if (gate) {
+    if ((s = run_gate(*gate, fa, gate_ws, stream)) != CER_OK) return s;
   }
   if ((e = mark(4)) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
 
@@ -642,6 +704,107 @@ cer_status cer_routed_block(void* h, void* out, int B, int N, int d, const cer_s
     if (e != cudaSuccess) return cuda_fail(e, "down GEMM launch");
   }
   if ((e = mark(5)) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+  return CER_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+cer_status cer_routed_block(void* h, void* out, int B, int N, int d, const cer_scorer* core, const cer_scorer* exp,
+                            const float* t, int task, int r0, int r1, int K, const void* Wg, const void* Wu,
+                            const void* WdT, int I, const int32_t* chan, int C, float* logits, int32_t* idx,
+                            uint8_t* mask, void* workspace, size_t workspace_bytes, cudaEvent_t* stage_events,
+                            int n_stage_events, cudaStream_t stream) {
+  return routed_block_impl(h, out, B, N, d, core, exp, t, task, r0, r1, K, Wg, Wu, WdT, I, chan, C, logits, idx,
+                           mask, workspace, workspace_bytes, stage_events, n_stage_events, nullptr, stream);
+}
+
+size_t cer_routed_block_gated_workspace_size(int B, int N, int d, int core_hidden, int exp_hidden, int task, int r0,
+                                             int r1, int K, int I) {
+  const size_t base = cer_routed_block_workspace_size(B, N, d, core_hidden, exp_hidden, task, r0, r1, K, I, 0);
+  if (base == 0) return 0;
+  const long long M = static_cast<long long>(B) * (K + N - (r1 - r0));
+  return base + gate_ws_bytes(M, I);
+}
+
+cer_status cer_routed_block_gated(void* h, void* out, int B, int N, int d, const cer_scorer* core,
+                                  const cer_scorer* exp, const float* t, int task, int r0, int r1, int K,
+                                  const void* Wg, const void* Wu, const void* WdT, int I, int C_keep,
+                                  const float* norms, float delta, float* saliency, float* leakage,
+                                  uint8_t* use_pruned, float* logits, int32_t* idx, uint8_t* mask, void* workspace,
+                                  size_t workspace_bytes, cudaEvent_t* stage_events, int n_stage_events,
+                                  cudaStream_t stream) {
+  GateArgs g{C_keep, norms, delta, saliency, leakage, use_pruned};
+  return routed_block_impl(h, out, B, N, d, core, exp, t, task, r0, r1, K, Wg, Wu, WdT, I, nullptr, I, logits, idx,
+                           mask, workspace, workspace_bytes, stage_events, n_stage_events, &g, stream);
+}
+
+cer_status cer_ffn_channel_norms(const void* WdT, int I, int d, float* norms, cudaStream_t stream) {
+  CER_PTR(WdT);
+  CER_PTR(norms);
+  CER_ALIGN(WdT);
+  CER_ALIGN(norms);
+  CER_REQUIRE(I >= 1 && d > 0 && d % 8 == 0, CER_ERR_SHAPE, "I=%d d=%d (d a positive multiple of 8)", I, d);
+  DeviceInfo* dev = nullptr;
+  cer_status s = device_info(&dev);
+  if (s != CER_OK) return s;
+  cudaError_t e = cer::launch_row_norms(static_cast<const __nv_bfloat16*>(WdT), I, d, norms, dev->n_sm, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "channel-norm launch");
+  return CER_OK;
+}
+
+size_t cer_routed_ffn_gated_workspace_size(int M, int d, int I) {
+  if (M < 0 || d < 0 || I < 0) return 0;
+  return cer_routed_ffn_workspace_size(M, d, I, 0) + gate_ws_bytes(M, I);
+}
+
+cer_status cer_routed_ffn_gated(const void* X, int M, int d, const void* Wg, const void* Wu, const void* WdT, int I,
+                                int C_keep, const float* norms, float delta, void* Y, float* saliency,
+                                float* leakage, uint8_t* use_pruned, void* workspace, size_t workspace_bytes,
+                                cudaStream_t stream) {
+  CER_PTR_IF(X, M > 0);
+  CER_PTR(Wg);
+  CER_PTR(Wu);
+  CER_PTR(WdT);
+  CER_PTR_IF(Y, M > 0);
+  CER_ALIGN(X);
+  CER_ALIGN(Wg);
+  CER_ALIGN(Wu);
+  CER_ALIGN(WdT);
+  CER_ALIGN(Y);
+  CER_ALIGN(workspace);
+  cer_status s = check_ffn_shape(M, d, I, nullptr, I);
+  if (s != CER_OK) return s;
+  GateArgs g{C_keep, norms, delta, saliency, leakage, use_pruned};
+  if ((s = check_gate(&g, I, I)) != CER_OK) return s;
+  const size_t need = cer_routed_ffn_gated_workspace_size(M, d, I);
+  CER_REQUIRE(M == 0 || (workspace != nullptr && workspace_bytes >= need), CER_ERR_WORKSPACE,
+              "workspace of %zu bytes needed, %zu given", need, workspace_bytes);
+  DeviceInfo* dev = nullptr;
+  if ((s = device_info(&dev)) != CER_OK) return s;
+  if (M == 0) return CER_OK;
+  char* ws = static_cast<char*>(workspace);
+  cer::FfnArgs a{};
+  a.act = reinterpret_cast<__nv_bfloat16*>(ws);
+  ws += round256(static_cast<size_t>(M) * I * 2);
+  a.X = static_cast<const __nv_bfloat16*>(X);
+  a.M = M;
+  a.d = d;
+  a.C = I;
+  a.C_small = C_keep;
+  a.Wg = static_cast<const __nv_bfloat16*>(Wg);
+  a.Wu = static_cast<const __nv_bfloat16*>(Wu);
+  a.WdT = static_cast<const __nv_bfloat16*>(WdT);
+  a.Y = static_cast<__nv_bfloat16*>(Y);
+  a.scatter = 0;
+  a.colsum = reinterpret_cast<float*>(ws);
+  a.status = dev->status;
+  cudaError_t e = cer::launch_ffn_gateup(a, dev->n_sm, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "gate/up GEMM launch");
+  if ((s = run_gate(g, a, ws, stream)) != CER_OK) return s;
+  e = cer::launch_ffn_down(a, dev->n_sm, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "down GEMM launch");
   return CER_OK;
 }
 

@@ -56,6 +56,7 @@ struct GateUpProblemT {
     CUtensorMap tm_wg;   // Wg [C, d], box 64 x 128
     CUtensorMap tm_wu;   // Wu [C, d], box 64 x 128
     CUtensorMap tm_act;  // act [M, C], box 64 x 128 (store)
+    float* colsum;       // optional [2 * n_mt][C]: sum of |act| over each half of a row tile
     int* status;
     int M, d, C, n_mt, n_mtp, n_ct;
   };
@@ -119,6 +120,20 @@ struct GateUpProblemT {
         tma_store_2d(&p.tm_act, box, x, mt * 128);
         bulk_commit_group();
       }
+      if (p.colsum != nullptr && mt < p.n_mt) {
+        // Column sums of |act| for the UCS saliency (Eq. 8): thread `row`
+        // sums channel row % 64 of the box over rows [64 * (row / 64), +64),
+        // reading the staged (swizzled) box; rows past M hold zeros.
+        const int j = row & 63, rh = row >> 6;
+        float acc = 0.f;
+#pragma unroll 8
+        for (int r = 64 * rh; r < 64 * rh + 64; ++r) {
+          const int off = r * 128 + ((((j >> 3) ^ (r & 7))) << 4) + ((j & 7) << 1);
+          acc += fabsf(__bfloat162float(*reinterpret_cast<const __nv_bfloat16*>(box + off)));
+        }
+        const int ch = x + j;
+        if (ch < p.C) p.colsum[static_cast<size_t>(2 * mt + rh) * p.C + ch] = acc;
+      }
     }
     return true;
   }
@@ -149,16 +164,19 @@ struct DownProblem {
     const int32_t* idx;          // scatter mode: keep list [B][k_tot]
     const __nv_bfloat16* hin;    // scatter mode: residual input
     __nv_bfloat16* out;          // Y [M, d] or the residual output
+    const uint8_t* use_small_k;  // optional device flag: contract only the first C_small channels
     int* status;
     int scatter;
-    int M, d, C, N, k_tot, n_mt, n_nt;
+    int M, d, C, C_small, N, k_tot, n_mt, n_nt;
   };
   struct ProdState {
     int m0, n0, n_atoms;
   };
 
   __device__ static int num_tiles(const Params& p) { return p.n_mt * p.n_nt; }
-  __device__ static int num_kb(const Params& p) { return p.C / 64; }
+  __device__ static int num_kb(const Params& p) {
+    return (p.use_small_k != nullptr && *p.use_small_k) ? p.C_small / 64 : p.C / 64;
+  }
   __device__ static int atoms(const Params& p, int nt) {
     const int left = (p.d - nt * BN) / 64;
     return left < ATOMS ? left : ATOMS;
@@ -281,6 +299,7 @@ cudaError_t launch_ffn_gateup(const FfnArgs& a, int n_sm, cudaStream_t stream) {
   if (!encode_bf16_2d(&p.tm_wg, a.Wg, a.C, a.d, 64, 128)) return cudaErrorInvalidValue;
   if (!encode_bf16_2d(&p.tm_wu, a.Wu, a.C, a.d, 64, 128)) return cudaErrorInvalidValue;
   if (!encode_bf16_2d(&p.tm_act, a.act, a.M, a.C, 64, 128)) return cudaErrorInvalidValue;
+  p.colsum = a.colsum;
   p.status = a.status;
   p.M = a.M;
   p.d = a.d;
@@ -300,11 +319,13 @@ static cudaError_t launch_down(const FfnArgs& a, int n_sm, cudaStream_t stream) 
   p.idx = a.idx;
   p.hin = a.h;
   p.out = a.scatter ? a.out : a.Y;
+  p.use_small_k = a.use_small_k;
   p.status = a.status;
   p.scatter = a.scatter;
   p.M = a.M;
   p.d = a.d;
   p.C = a.C;
+  p.C_small = a.C_small;
   p.N = a.N;
   p.k_tot = a.k_tot;
   p.n_mt = (a.M + 127) / 128;

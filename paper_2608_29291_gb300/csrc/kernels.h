@@ -101,10 +101,25 @@ struct FfnArgs {
   const int32_t* idx;
   int N, k_tot;
   int scatter;
+  // UCS FFN gate (Sec. 3.4, Eq. 8/9): gate/up also writes column sums of
+  // |act| (colsum [2 * ceil(M/128)][C], optional); the down GEMM contracts
+  // only the first C_small channels when *use_small_k is set (optional).
+  float* colsum;
+  const uint8_t* use_small_k;
+  int C_small;
   int* status;
 };
 cudaError_t launch_ffn_gateup(const FfnArgs& a, int n_sm, cudaStream_t stream);
 cudaError_t launch_ffn_down(const FfnArgs& a, int n_sm, cudaStream_t stream);
+
+// ------------------------------------------------------------------ UCS FFN gate
+// saliency s_c = (sum_parts colsum[part][c] / M) * norm_c; leakage =
+// sum_{c >= C_keep} s_c / sum_c s_c; *use_pruned = leakage <= delta.
+// part_ws holds 2 * ceil(I / 256) floats.
+cudaError_t launch_ffn_gate(const float* colsum, int n_parts, int M, int I, int C_keep, const float* norms,
+                            float delta, float* saliency, float* part_ws, float* leakage, uint8_t* use_pruned,
+                            cudaStream_t stream);
+cudaError_t launch_row_norms(const __nv_bfloat16* W, int rows, int d, float* norms, int n_sm, cudaStream_t stream);
 
 // ------------------------------------------------------------------ UCS statistics
 cudaError_t launch_drop_stats(const uint8_t* mask_t, const uint8_t* mask_ref, int B, int N, int r0, int r1,

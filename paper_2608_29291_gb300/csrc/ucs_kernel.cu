@@ -168,7 +168,105 @@ __global__ void __launch_bounds__(kStatThreads) gap_reduce_kernel(const float* _
   if (skip) skip[b] = g <= static_cast<double>(delta) ? 1 : 0;
 }
 
+// ---------------------------------------------------------------- Eq. 8 / 9
+
+// Per channel: s_c = mean over the retained rows of |z_c| times
+// ||W_down[:, c]|| (the column norms are a static per-layer input); each block
+// also sums its channels' saliency split at C_keep (kept channels first,
+// the mask's pruned channels after), fixed order.
+constexpr int kGateThreads = 256;
+
+__global__ void __launch_bounds__(kGateThreads) saliency_kernel(const float* __restrict__ colsum, int n_parts,
+                                                                 int M, int I, int C_keep,
+                                                                 const float* __restrict__ norms, float* saliency,
+                                                                 float* part_ws) {
+  __shared__ double red[2][kGateThreads / 32];
+  const int c = blockIdx.x * kGateThreads + threadIdx.x;
+  double s = 0.0;
+  if (c < I) {
+    float acc = 0.f;
+    for (int q = 0; q < n_parts; ++q) acc += colsum[static_cast<size_t>(q) * I + c];
+    s = static_cast<double>(acc) / M * norms[c];
+    if (saliency) saliency[c] = static_cast<float>(s);
+  }
+  double kept = (c < C_keep) ? s : 0.0, pruned = (c >= C_keep) ? s : 0.0;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    kept += __shfl_xor_sync(0xffffffffu, kept, off);
+    pruned += __shfl_xor_sync(0xffffffffu, pruned, off);
+  }
+  if ((threadIdx.x & 31) == 0) {
+    red[0][threadIdx.x >> 5] = kept;
+    red[1][threadIdx.x >> 5] = pruned;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    kept = pruned = 0.0;
+    for (int w = 0; w < kGateThreads / 32; ++w) {
+      kept += red[0][w];
+      pruned += red[1][w];
+    }
+    part_ws[2 * blockIdx.x] = static_cast<float>(kept);
+    part_ws[2 * blockIdx.x + 1] = static_cast<float>(pruned);
+  }
+}
+
+// One thread: leakage of Eq. 9 and the pruned-or-full decision.
+__global__ void leakage_kernel(const float* part_ws, int n_blocks, float delta, float* leakage, uint8_t* use_pruned) {
+  if (threadIdx.x != 0 || blockIdx.x != 0) return;
+  double kept = 0.0, pruned = 0.0;
+  for (int b = 0; b < n_blocks; ++b) {
+    kept += part_ws[2 * b];
+    pruned += part_ws[2 * b + 1];
+  }
+  const double total = kept + pruned;
+  const double lam = total > 0.0 ? pruned / total : 0.0;
+  if (leakage) *leakage = static_cast<float>(lam);
+  *use_pruned = lam <= static_cast<double>(delta) ? 1 : 0;
+}
+
+// One warp per row: ||W[r, :]||_2 in fp32 (static per-layer input of Eq. 8).
+__global__ void __launch_bounds__(kStatThreads) row_norm_kernel(const uint4* __restrict__ W, int d8, int rows,
+                                                                 float* __restrict__ norms) {
+  const int lane = threadIdx.x & 31;
+  const int wpb = blockDim.x >> 5;
+  for (int r = blockIdx.x * wpb + (threadIdx.x >> 5); r < rows; r += gridDim.x * wpb) {
+    float s = 0.f;
+    for (int c = lane; c < d8; c += 32) {
+      const uint4 v = __ldg(W + static_cast<size_t>(r) * d8 + c);
+      const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w4[k]));
+        s = fmaf(f.x, f.x, fmaf(f.y, f.y, s));
+      }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+    if (lane == 0) norms[r] = sqrtf(s);
+  }
+}
+
 // ---------------------------------------------------------------- launchers
+
+cudaError_t launch_ffn_gate(const float* colsum, int n_parts, int M, int I, int C_keep, const float* norms,
+                            float delta, float* saliency, float* part_ws, float* leakage, uint8_t* use_pruned,
+                            cudaStream_t stream) {
+  const int blocks = (I + kGateThreads - 1) / kGateThreads;
+  saliency_kernel<<<blocks, kGateThreads, 0, stream>>>(colsum, n_parts, M, I, C_keep, norms, saliency, part_ws);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  leakage_kernel<<<1, 32, 0, stream>>>(part_ws, blocks, delta, leakage, use_pruned);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_row_norms(const __nv_bfloat16* W, int rows, int d, float* norms, int n_sm, cudaStream_t stream) {
+  if (rows == 0) return cudaSuccess;
+  int blocks = (rows + 7) / 8;
+  if (blocks > n_sm * 8) blocks = n_sm * 8;
+  row_norm_kernel<<<blocks, kStatThreads, 0, stream>>>(reinterpret_cast<const uint4*>(W), d / 8, rows, norms);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_drop_stats(const uint8_t* mask_t, const uint8_t* mask_ref, int B, int N, int r0, int r1,
                               float* jac, float* jrand, float* rda, int32_t* counts, cudaStream_t stream) {
