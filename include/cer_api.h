@@ -283,7 +283,7 @@ cer_status cer_drop_set_stats(const uint8_t* mask_t, const uint8_t* mask_ref, in
  *   mask         uint8 [B, N]
  *   gap          fp32 [B] output; skip uint8 [B] output or NULL
  * Cosines accumulate in fp32 per token (a zero-norm pair counts 1 if equal,
- * else 0); the means are fp64.  Empty R gives g = 0.
+ * else 0); the means are fp32 fixed-order tree sums.  Empty R gives g = 0.
  * Workspace: cer_redundancy_gap_workspace_size(B, N).                      */
 cer_status cer_redundancy_gap(const void* h_in, const void* h_out, const uint8_t* mask, int B, int N, int d,
                               float delta, float* gap, uint8_t* skip,

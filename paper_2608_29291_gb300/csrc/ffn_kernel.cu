@@ -146,20 +146,22 @@ using GateUpProblem = GateUpProblemT<4>;
 
 // ---------------------------------------------------------------- down
 
-template <int BN_>
+// CL = 2: two CTAs per cluster take adjacent N tiles of the same 128 rows;
+// each loads 64 of the act tile's rows and multicasts them to both.
+template <int BN_, int CL>
 struct DownProblem {
   static constexpr int BN = BN_;
   static constexpr int ATOMS = BN / 64;
   static constexpr int STAGES = BN == 256 ? 4 : BN == 192 ? 5 : 6;
   static constexpr int B_MN_MAJOR = 1;
   static constexpr int EPI_WARPS = 8;
-  static constexpr int CLUSTER = 1;
+  static constexpr int CLUSTER = CL;
   static constexpr uint32_t kBStepBytes = 2048;     // 16 K-rows = two 1024 B row groups
   static constexpr uint32_t kAtomBytes = 64 * 128;  // 64 K-rows x 64 columns
   static constexpr uint32_t kEpiSmemBytes = 0;
 
   struct Params {
-    CUtensorMap tm_act;  // act [M, C], box 64 x 128
+    CUtensorMap tm_act;  // act [M, C], box 64 x 128 (64 x 64 with CL = 2)
     CUtensorMap tm_wdt;  // WdT [C, d], box 64 x 64
     const int32_t* idx;          // scatter mode: keep list [B][k_tot]
     const __nv_bfloat16* hin;    // scatter mode: residual input
@@ -167,41 +169,48 @@ struct DownProblem {
     const uint8_t* use_small_k;  // optional device flag: contract only the first C_small channels
     int* status;
     int scatter;
-    int M, d, C, C_small, N, k_tot, n_mt, n_nt;
+    int M, d, C, C_small, N, k_tot, n_mt, n_nt, n_ntc;   // n_ntc: N-tile groups of CL
   };
   struct ProdState {
-    int m0, n0, n_atoms;
+    int m0, n0, n_atoms, rank;
   };
 
-  __device__ static int num_tiles(const Params& p) { return p.n_mt * p.n_nt; }
+  // Cluster tile t: row tile t % n_mt, N tiles CL * (t / n_mt) + rank.
+  __device__ static int num_tiles(const Params& p) { return p.n_mt * p.n_ntc; }
+  __device__ static int ntile(const Params& p, int tile, int rank) { return CL * (tile / p.n_mt) + rank; }
   __device__ static int num_kb(const Params& p) {
     return (p.use_small_k != nullptr && *p.use_small_k) ? p.C_small / 64 : p.C / 64;
   }
   __device__ static int atoms(const Params& p, int nt) {
-    const int left = (p.d - nt * BN) / 64;
-    return left < ATOMS ? left : ATOMS;
+    const int left = (p.d - nt * BN) / 64;    // an N tile past d (odd pair) loads no B
+    return left < 0 ? 0 : left < ATOMS ? left : ATOMS;
   }
   __device__ static uint32_t stage_bytes(const Params& p, int tile, int) {
-    return kATileBytes + atoms(p, tile / p.n_mt) * kAtomBytes;
+    return kATileBytes + atoms(p, ntile(p, tile, static_cast<int>(CL > 1 ? cluster_ctarank() : 0))) * kAtomBytes;
   }
-  __device__ static void prod_tile(const Params& p, int tile, int, ProdState& st) {
-    const int nt = tile / p.n_mt;
+  __device__ static void prod_tile(const Params& p, int tile, int rank, ProdState& st) {
+    const int nt = ntile(p, tile, rank);
     st.n0 = nt * BN;
     st.m0 = (tile % p.n_mt) * 128;
     st.n_atoms = atoms(p, nt);
+    st.rank = rank;
   }
   __device__ static void prod_kb(const Params& p, const ProdState& st, int, int kb, int lane, uint8_t* a,
                                  uint8_t* b, uint64_t* bar) {
     if (lane == 0) {
-      tma_load_2d(a, &p.tm_act, bar, kb * 64, st.m0);
+      if (CL == 1) {
+        tma_load_2d(a, &p.tm_act, bar, kb * 64, st.m0);
+      } else {
+        tma_load_2d_multicast(a + st.rank * (kATileBytes / 2), &p.tm_act, bar, kb * 64, st.m0 + 64 * st.rank, 0x3);
+      }
       for (int at = 0; at < st.n_atoms; ++at) tma_load_2d(b + at * kAtomBytes, &p.tm_wdt, bar, st.n0 + at * 64, kb * 64);
     }
   }
   __device__ static uint64_t bdesc(uint32_t saddr) { return sdesc_mnmajor_sw128(saddr, kAtomBytes, 1024); }
 
   __device__ static void epilogue_done(const Params&, int, int) {}
-  __device__ static bool epilogue(const Params& p, int tile, int row, int half, uint32_t taddr, EpiCtx&) {
-    const int nt = tile / p.n_mt;
+  __device__ static bool epilogue(const Params& p, int tile, int row, int half, uint32_t taddr, EpiCtx& ctx) {
+    const int nt = ntile(p, tile, ctx.rank);
     const int m = (tile % p.n_mt) * 128 + row;
     bool valid = m < p.M;
     size_t dst_row = 0;
@@ -262,20 +271,8 @@ static cudaError_t launch_gemm(const typename P::Params& p, int tiles, int n_sm,
   if (e != cudaSuccess) return e;
   if (P::CLUSTER == 1) {
     const int grid = tiles < n_sm ? tiles : n_sm;
-    umma_gemm_kernel<P><<<grid, gemm_threads<P>(), smem, stream>>>(p);
-    return cudaGetLastError();
+    return launch_k(umma_gemm_kernel<P>, dim3(grid), dim3(gemm_threads<P>()), smem, stream, 1, p);
   }
-  cudaLaunchConfig_t cfg = {};
-  cfg.blockDim = dim3(gemm_threads<P>(), 1, 1);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = P::CLUSTER;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
   // The persistent grid holds only as many clusters as can be resident at
   // once (SM pairs inside GPC boundaries), so no cluster waits for another.
   static int resident[64] = {0};
@@ -283,14 +280,25 @@ static cudaError_t launch_gemm(const typename P::Params& p, int tiles, int n_sm,
   cudaGetDevice(&dev);
   int& max_clusters = resident[dev & 63];
   if (max_clusters == 0) {
+    cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(n_sm / P::CLUSTER * P::CLUSTER, 1, 1);
+    cfg.blockDim = dim3(gemm_threads<P>(), 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = P::CLUSTER;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
     int n = 0;
     e = cudaOccupancyMaxActiveClusters(&n, umma_gemm_kernel<P>, &cfg);
     if (e != cudaSuccess) return e;
     max_clusters = n > 0 ? n : 1;
   }
-  cfg.gridDim = dim3((tiles < max_clusters ? tiles : max_clusters) * P::CLUSTER, 1, 1);
-  return cudaLaunchKernelEx(&cfg, umma_gemm_kernel<P>, p);
+  const int grid = (tiles < max_clusters ? tiles : max_clusters) * P::CLUSTER;
+  return launch_k(umma_gemm_kernel<P>, dim3(grid), dim3(gemm_threads<P>()), smem, stream, P::CLUSTER, p);
 }
 
 cudaError_t launch_ffn_gateup(const FfnArgs& a, int n_sm, cudaStream_t stream) {
@@ -310,11 +318,11 @@ cudaError_t launch_ffn_gateup(const FfnArgs& a, int n_sm, cudaStream_t stream) {
   return launch_gemm<GateUpProblem>(p, p.n_mtp * p.n_ct, n_sm, stream);
 }
 
-template <int BN>
+template <int BN, int CL>
 static cudaError_t launch_down(const FfnArgs& a, int n_sm, cudaStream_t stream) {
-  using P = DownProblem<BN>;
+  using P = DownProblem<BN, CL>;
   typename P::Params p{};
-  if (!encode_bf16_2d(&p.tm_act, a.act, a.M, a.C, 64, 128)) return cudaErrorInvalidValue;
+  if (!encode_bf16_2d(&p.tm_act, a.act, a.M, a.C, 64, CL == 1 ? 128 : 64)) return cudaErrorInvalidValue;
   if (!encode_bf16_2d(&p.tm_wdt, a.WdT, a.C, a.d, 64, 64)) return cudaErrorInvalidValue;
   p.idx = a.idx;
   p.hin = a.h;
@@ -330,7 +338,8 @@ static cudaError_t launch_down(const FfnArgs& a, int n_sm, cudaStream_t stream) 
   p.k_tot = a.k_tot;
   p.n_mt = (a.M + 127) / 128;
   p.n_nt = (a.d + BN - 1) / BN;
-  return launch_gemm<P>(p, p.n_mt * p.n_nt, n_sm, stream);
+  p.n_ntc = (p.n_nt + CL - 1) / CL;
+  return launch_gemm<P>(p, p.n_mt * p.n_ntc, n_sm, stream);
 }
 
 // N-tile width of the down GEMM: the one with the least per-SM work
@@ -350,11 +359,14 @@ int down_tile_width(int M, int d, int n_sm) {
   return best;
 }
 
+// One CTA per tile.  (Pairs of N tiles sharing the act tile through cluster
+// multicast, DownProblem<BN, 2>, measured 6-7% slower on the 1.5B and 7B
+// workloads: the paired pipelines wait on each other.)
 cudaError_t launch_ffn_down(const FfnArgs& a, int n_sm, cudaStream_t stream) {
   switch (down_tile_width(a.M, a.d, n_sm)) {
-    case 192: return launch_down<192>(a, n_sm, stream);
-    case 128: return launch_down<128>(a, n_sm, stream);
-    default: return launch_down<256>(a, n_sm, stream);
+    case 192: return launch_down<192, 1>(a, n_sm, stream);
+    case 128: return launch_down<128, 1>(a, n_sm, stream);
+    default: return launch_down<256, 1>(a, n_sm, stream);
   }
 }
 

@@ -24,6 +24,18 @@ __device__ __forceinline__ uint64_t globaltimer_ns() {
   return t;
 }
 
+// ------------------------------------------------------------------ dependent launch
+
+// Programmatic dependent launch: every kernel of this library lets the next
+// kernel on the stream be scheduled as soon as all of its own blocks have
+// started (launch_dependents at entry), and waits for the previous kernel's
+// results to be complete and visible before reading them (wait).  Without
+// the launch attribute both are no-ops.
+__device__ __forceinline__ void griddep_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // ------------------------------------------------------------------ mbarrier
 
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {

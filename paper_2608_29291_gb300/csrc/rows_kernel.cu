@@ -5,6 +5,7 @@
 #include <cuda_bf16.h>
 
 #include "kernels.h"
+#include "ptx.cuh"
 #include "status.cuh"
 
 namespace cer {
@@ -14,6 +15,8 @@ constexpr int kRowThreads = 512;
 __global__ void __launch_bounds__(kRowThreads) gather_rows_kernel(const uint4* __restrict__ h, int N, int d16,
                                                                   const int32_t* __restrict__ idx, int k_tot,
                                                                   int M, uint4* __restrict__ X, int* status) {
+  griddep_wait();
+  griddep_launch_dependents();
   const int lane = threadIdx.x & 31;
   const int wpb = blockDim.x >> 5;
   for (int m = blockIdx.x * wpb + (threadIdx.x >> 5); m < M; m += gridDim.x * wpb) {
@@ -53,6 +56,8 @@ __global__ void __launch_bounds__(kRowThreads) scatter_add_kernel(uint4* __restr
                                                                   const int32_t* __restrict__ idx, int k_tot,
                                                                   int M, const uint4* __restrict__ Y,
                                                                   int* status) {
+  griddep_wait();
+  griddep_launch_dependents();
   const int lane = threadIdx.x & 31;
   const int wpb = blockDim.x >> 5;
   for (int m = blockIdx.x * wpb + (threadIdx.x >> 5); m < M; m += gridDim.x * wpb) {
@@ -86,20 +91,16 @@ cudaError_t launch_gather(const __nv_bfloat16* h, int B, int N, int d, const int
                           __nv_bfloat16* X, int* status, int n_sm, cudaStream_t stream) {
   const int M = B * k_tot;
   if (M == 0 || d == 0) return cudaSuccess;
-  gather_rows_kernel<<<row_grid(M, n_sm), kRowThreads, 0, stream>>>(reinterpret_cast<const uint4*>(h), N, d / 8,
-                                                                    idx, k_tot, M, reinterpret_cast<uint4*>(X),
-                                                                    status);
-  return cudaGetLastError();
+  return launch_k(gather_rows_kernel, dim3(row_grid(M, n_sm)), dim3(kRowThreads), 0, stream, 1,
+                  reinterpret_cast<const uint4*>(h), N, d / 8, idx, k_tot, M, reinterpret_cast<uint4*>(X), status);
 }
 
 cudaError_t launch_scatter_add(__nv_bfloat16* h, int B, int N, int d, const int32_t* idx, int k_tot,
                                const __nv_bfloat16* Y, int* status, int n_sm, cudaStream_t stream) {
   const int M = B * k_tot;
   if (M == 0 || d == 0) return cudaSuccess;
-  scatter_add_kernel<<<row_grid(M, n_sm), kRowThreads, 0, stream>>>(reinterpret_cast<uint4*>(h), N, d / 8, idx,
-                                                                    k_tot, M, reinterpret_cast<const uint4*>(Y),
-                                                                    status);
-  return cudaGetLastError();
+  return launch_k(scatter_add_kernel, dim3(row_grid(M, n_sm)), dim3(kRowThreads), 0, stream, 1,
+                  reinterpret_cast<uint4*>(h), N, d / 8, idx, k_tot, M, reinterpret_cast<const uint4*>(Y), status);
 }
 
 }  // namespace cer

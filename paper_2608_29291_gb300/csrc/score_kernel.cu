@@ -39,6 +39,8 @@ constexpr int kBiasColsPerBlock = 8;
 __global__ void __launch_bounds__(32 * kBiasColsPerBlock) time_bias_kernel(ScoreArgs a,
                                                                            const __grid_constant__ EmbFreqTable ft,
                                                                            float* bias_tab, float* w2_tab) {
+  griddep_wait();
+  griddep_launch_dependents();
   extern __shared__ float emb[];
   const int b = blockIdx.x;
   const int Ht = a.Hc + (a.gen ? a.He : 0);
@@ -128,8 +130,10 @@ struct ScoreProblem {
     CUtensorMap tm_w1;   // core W1 [Hc, d], box 64 x BN
     CUtensorMap tm_w1e;  // expansion W1e as [S*He, d], box 64 x BN
     const float* t;
-    const float* bias_tab;
+    const float* bias_tab;   // [B][Ht], or NULL: columns take b1 (or 0) and w2 directly
     const float* w2_tab;
+    const float* b1;
+    const float* w2;
     float* partial;
     int* status;
     int B, N, d, S, He, Ht;
@@ -175,18 +179,19 @@ struct ScoreProblem {
   __device__ static bool epilogue(const Params& p, int tile, int row, int half, uint32_t taddr, EpiCtx&) {
     int b, rt, chunk;
     decode(p, tile, b, rt, chunk);
-    const float* bias = p.bias_tab + static_cast<size_t>(b) * p.Ht + chunk * BN;
-    const float* w2 = p.w2_tab + static_cast<size_t>(b) * p.Ht + chunk * BN;
+    const float* bias = p.bias_tab ? p.bias_tab + static_cast<size_t>(b) * p.Ht + chunk * BN
+                                   : (p.b1 ? p.b1 + chunk * BN : nullptr);
+    const float* w2 = p.w2_tab ? p.w2_tab + static_cast<size_t>(b) * p.Ht + chunk * BN : p.w2 + chunk * BN;
     float s = 0.f;
 #pragma unroll 1
     for (int c = half * (BN / 64); c < (half + 1) * (BN / 64); ++c) {
       float v[32];
       tmem_ld_32x32(taddr + c * 32, v);
-      const float4* b4 = reinterpret_cast<const float4*>(bias + c * 32);
+      const float4* b4 = bias ? reinterpret_cast<const float4*>(bias + c * 32) : nullptr;
       const float4* w4 = reinterpret_cast<const float4*>(w2 + c * 32);
 #pragma unroll
       for (int q = 0; q < 8; ++q) {
-        const float4 bb = __ldg(b4 + q), ww = __ldg(w4 + q);
+        const float4 bb = b4 ? __ldg(b4 + q) : make_float4(0.f, 0.f, 0.f, 0.f), ww = __ldg(w4 + q);
         s = fmaf(ww.x, gelu_as(v[4 * q + 0] + bb.x), s);
         s = fmaf(ww.y, gelu_as(v[4 * q + 1] + bb.y), s);
         s = fmaf(ww.z, gelu_as(v[4 * q + 2] + bb.z), s);
@@ -203,6 +208,8 @@ struct ScoreProblem {
 
 __global__ void score_reduce_kernel(const float* __restrict__ partial, int n_chunks, size_t total,
                                     float* __restrict__ logits, float* __restrict__ probs) {
+  griddep_wait();
+  griddep_launch_dependents();
   for (size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; i < total;
        i += static_cast<size_t>(gridDim.x) * blockDim.x) {
     float s = partial[i];
@@ -257,6 +264,8 @@ static cudaError_t launch_score_gemm(const ScoreArgs& a, const float* bias_tab, 
   p.t = a.t;
   p.bias_tab = bias_tab;
   p.w2_tab = w2_tab;
+  p.b1 = a.b1;
+  p.w2 = a.w2;
   p.partial = partial;
   p.status = a.status;
   p.B = a.B;
@@ -274,24 +283,33 @@ static cudaError_t launch_score_gemm(const ScoreArgs& a, const float* bias_tab, 
   cudaError_t e = ensure_max_smem(reinterpret_cast<const void*>(umma_gemm_kernel<P>), smem);
   if (e != cudaSuccess) return e;
   const int grid = tiles < n_sm ? tiles : n_sm;
-  umma_gemm_kernel<P><<<grid, gemm_threads<P>(), smem, stream>>>(p);
-  return cudaGetLastError();
+  return launch_k(umma_gemm_kernel<P>, dim3(grid), dim3(gemm_threads<P>()), smem, stream, 1, p);
 }
 
 cudaError_t launch_score(const ScoreArgs& a, const ScoreWorkspace& ws, int n_sm, cudaStream_t stream,
                          int* n_partials) {
-  const int emb_bytes = (a.gen && a.U) ? a.E * static_cast<int>(sizeof(float)) : 0;
-  const int Ht = a.Hc + (a.gen ? a.He : 0);
+  const int bn = pick_chunk_width(a, n_sm);
+  *n_partials = bn ? 2 * (a.Hc + (a.gen ? a.He : 0)) / bn : 0;
+  if (!a.gen) {
+    // Understanding: one core scorer for every sequence, no time input; the
+    // epilogue reads b1 and w2 directly and no bias table is built.
+    switch (bn) {
+      case 256: return launch_score_gemm<256>(a, nullptr, nullptr, ws.partial, n_sm, stream);
+      case 128: return launch_score_gemm<128>(a, nullptr, nullptr, ws.partial, n_sm, stream);
+      case 64: return launch_score_gemm<64>(a, nullptr, nullptr, ws.partial, n_sm, stream);
+      default: return cudaErrorInvalidValue;
+    }
+  }
+  const int emb_bytes = a.U ? a.E * static_cast<int>(sizeof(float)) : 0;
+  const int Ht = a.Hc + a.He;
   EmbFreqTable ft;
   const int half = (a.gen && a.U) ? a.E / 2 : 0;
   for (int j = 0; j < half; ++j) ft.g[j] = std::pow(10000.0, -static_cast<double>(j) / half) / (2.0 * M_PI);
   for (int j = half; j < 512; ++j) ft.g[j] = 0.0;
   const dim3 bias_grid(a.B, (Ht + kBiasColsPerBlock - 1) / kBiasColsPerBlock);
-  time_bias_kernel<<<bias_grid, 32 * kBiasColsPerBlock, emb_bytes, stream>>>(a, ft, ws.bias_tab, ws.w2_tab);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = launch_k(time_bias_kernel, bias_grid, dim3(32 * kBiasColsPerBlock), emb_bytes, stream, 1, a, ft,
+                           ws.bias_tab, ws.w2_tab);
   if (e != cudaSuccess) return e;
-  const int bn = pick_chunk_width(a, n_sm);
-  *n_partials = bn ? 2 * (a.Hc + (a.gen ? a.He : 0)) / bn : 0;
   switch (bn) {
     case 256: return launch_score_gemm<256>(a, ws.bias_tab, ws.w2_tab, ws.partial, n_sm, stream);
     case 128: return launch_score_gemm<128>(a, ws.bias_tab, ws.w2_tab, ws.partial, n_sm, stream);
@@ -306,8 +324,8 @@ cudaError_t launch_score_reduce(const float* partial, int n_chunks, size_t total
   size_t blocks = (total + 255) / 256;
   const size_t cap = static_cast<size_t>(n_sm) * 8;
   if (blocks > cap) blocks = cap;
-  score_reduce_kernel<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(partial, n_chunks, total, logits, probs);
-  return cudaGetLastError();
+  return launch_k(score_reduce_kernel, dim3(static_cast<unsigned>(blocks)), dim3(256), 0, stream, 1, partial,
+                  n_chunks, total, logits, probs);
 }
 
 }  // namespace cer

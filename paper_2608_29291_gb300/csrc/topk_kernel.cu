@@ -13,6 +13,7 @@
 #include <cuda_runtime.h>
 
 #include "kernels.h"
+#include "ptx.cuh"
 #include "status.cuh"
 
 namespace cer {
@@ -55,9 +56,16 @@ __device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t* w
   return r;
 }
 
+// Histogram counts go to kSubHist copies (by warp) to spread the atomic
+// contention of logits that share a few digit values; merged after each pass.
+constexpr int kSubHist = 8;
+
 __global__ void __launch_bounds__(kTopkThreads) topk_kernel(TopkArgs a) {
+  griddep_wait();
+  griddep_launch_dependents();
   extern __shared__ uint32_t keys[];
   __shared__ uint32_t hist[256];
+  __shared__ uint32_t sub[kSubHist][256];
   __shared__ uint32_t warp_tot[32];
   __shared__ uint32_t s_prefix, s_remaining;
   __shared__ int s_nan;
@@ -90,11 +98,19 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(TopkArgs a) {
   if (!keep_all && !keep_none) {
     uint32_t prefix = 0, pmask = 0, remaining = static_cast<uint32_t>(K);
     for (int shift = 24; shift >= 0; shift -= 8) {
-      for (int i = tid; i < 256; i += blockDim.x) hist[i] = 0;
+      for (int i = tid; i < kSubHist * 256; i += blockDim.x) (&sub[0][0])[i] = 0;
       __syncthreads();
+      uint32_t* my = sub[(tid >> 5) % kSubHist];
       for (int i = a.r0 + tid; i < a.r1; i += blockDim.x) {
         const uint32_t k = keys[i];
-        if ((k & pmask) == prefix) atomicAdd(&hist[(k >> shift) & 255u], 1u);
+        if ((k & pmask) == prefix) atomicAdd(&my[(k >> shift) & 255u], 1u);
+      }
+      __syncthreads();
+      for (int i = tid; i < 256; i += blockDim.x) {
+        uint32_t c = 0;
+#pragma unroll
+        for (int q = 0; q < kSubHist; ++q) c += sub[q][i];
+        hist[i] = c;
       }
       __syncthreads();
       if (tid < 32) {
@@ -190,8 +206,7 @@ cudaError_t launch_topk(const TopkArgs& a, cudaStream_t stream) {
   // The limit is raised once per device to the largest N ever accepted.
   cudaError_t e = ensure_max_smem(reinterpret_cast<const void*>(topk_kernel), kTopkMaxN * sizeof(uint32_t));
   if (e != cudaSuccess) return e;
-  topk_kernel<<<a.B, kTopkThreads, smem, stream>>>(a);
-  return cudaGetLastError();
+  return launch_k(topk_kernel, dim3(a.B), dim3(kTopkThreads), smem, stream, 1, a);
 }
 
 }  // namespace cer

@@ -5,6 +5,7 @@
 #include <cuda_bf16.h>
 
 #include "kernels.h"
+#include "ptx.cuh"
 #include "status.cuh"
 
 namespace cer {
@@ -25,11 +26,15 @@ __device__ __forceinline__ int warp_sum_int(int v) {
 // Reading of J_rand: E|A&B| / E|A|B| for uniformly random drop sets of the
 // same sizes a, b among the n routable tokens, E|A&B| = a b / n.  An empty
 // union gives J = 1; J_rand = 1 gives RDA = 1.
-__global__ void __launch_bounds__(kStatThreads) drop_stats_kernel(const uint8_t* __restrict__ mask_t,
+constexpr int kDropThreads = 1024;
+
+__global__ void __launch_bounds__(kDropThreads) drop_stats_kernel(const uint8_t* __restrict__ mask_t,
                                                                    const uint8_t* __restrict__ mask_ref, int N,
                                                                    int r0, int r1, float* jac, float* jrand,
                                                                    float* rda, int32_t* counts) {
-  __shared__ int part[3][kStatThreads / 32];
+  griddep_wait();
+  griddep_launch_dependents();
+  __shared__ int part[3][kDropThreads / 32];
   const int b = blockIdx.x;
   const uint8_t* mt = mask_t + static_cast<size_t>(b) * N;
   const uint8_t* mr = mask_ref + static_cast<size_t>(b) * N;
@@ -52,7 +57,7 @@ __global__ void __launch_bounds__(kStatThreads) drop_stats_kernel(const uint8_t*
   __syncthreads();
   if (threadIdx.x != 0) return;
   na = nb = ni = 0;
-  for (int w = 0; w < kStatThreads / 32; ++w) {
+  for (int w = 0; w < kDropThreads / 32; ++w) {
     na += part[0][w];
     nb += part[1][w];
     ni += part[2][w];
@@ -84,6 +89,8 @@ __global__ void __launch_bounds__(kStatThreads) drop_stats_kernel(const uint8_t*
 __global__ void __launch_bounds__(kStatThreads) row_cosine_kernel(const uint4* __restrict__ h_in,
                                                                    const uint4* __restrict__ h_out, int d8,
                                                                    long rows, float* __restrict__ cosv) {
+  griddep_wait();
+  griddep_launch_dependents();
   const int lane = threadIdx.x & 31;
   const long wpb = blockDim.x >> 5;
   for (long r = blockIdx.x * wpb + (threadIdx.x >> 5); r < rows; r += static_cast<long>(gridDim.x) * wpb) {
@@ -91,6 +98,7 @@ __global__ void __launch_bounds__(kStatThreads) row_cosine_kernel(const uint4* _
     const uint4* o = h_out + r * d8;
     float dot = 0.f, na = 0.f, no = 0.f;
     unsigned diff = 0;
+#pragma unroll 8
     for (int c = lane; c < d8; c += 32) {
       const uint4 va = __ldg(a + c), vo = __ldg(o + c);
       diff |= (va.x ^ vo.x) | (va.y ^ vo.y) | (va.z ^ vo.z) | (va.w ^ vo.w);
@@ -122,20 +130,25 @@ __global__ void __launch_bounds__(kStatThreads) row_cosine_kernel(const uint4* _
   }
 }
 
-// One block per sequence: g = mean_all(cos) - mean_R(cos) in fp64 (fixed
-// summation order), skip = g <= delta (compared in fp64).  Empty R gives g = 0.
+// One block per sequence: g = mean_all(cos) - mean_R(cos), skip = g <= delta.
+// fp32 sums in a fixed tree order (per-thread strided sums, xor-shuffle tree,
+// warps in order): relative error about log2(N) * 2^-24.  FP64 arithmetic is
+// very slow on this part, so it is kept out of this reduction.  Empty R gives
+// g = 0.
 __global__ void __launch_bounds__(kStatThreads) gap_reduce_kernel(const float* __restrict__ cosv,
                                                                    const uint8_t* __restrict__ mask, int N,
                                                                    float delta, float* gap, uint8_t* skip) {
-  __shared__ double part_all[kStatThreads / 32], part_ret[kStatThreads / 32];
+  griddep_wait();
+  griddep_launch_dependents();
+  __shared__ float part_all[kStatThreads / 32], part_ret[kStatThreads / 32];
   __shared__ int part_n[kStatThreads / 32];
   const int b = blockIdx.x;
   const float* c = cosv + static_cast<size_t>(b) * N;
   const uint8_t* m = mask + static_cast<size_t>(b) * N;
-  double s_all = 0.0, s_ret = 0.0;
+  float s_all = 0.f, s_ret = 0.f;
   int n_ret = 0;
   for (int i = threadIdx.x; i < N; i += blockDim.x) {
-    const double v = c[i];
+    const float v = c[i];
     s_all += v;
     if (m[i]) {
       s_ret += v;
@@ -156,16 +169,16 @@ __global__ void __launch_bounds__(kStatThreads) gap_reduce_kernel(const float* _
   }
   __syncthreads();
   if (threadIdx.x != 0) return;
-  s_all = s_ret = 0.0;
+  s_all = s_ret = 0.f;
   n_ret = 0;
   for (int w = 0; w < kStatThreads / 32; ++w) {
     s_all += part_all[w];
     s_ret += part_ret[w];
     n_ret += part_n[w];
   }
-  const double g = (n_ret == 0 || N == 0) ? 0.0 : s_all / N - s_ret / n_ret;
-  gap[b] = static_cast<float>(g);
-  if (skip) skip[b] = g <= static_cast<double>(delta) ? 1 : 0;
+  const float g = (n_ret == 0 || N == 0) ? 0.f : s_all / static_cast<float>(N) - s_ret / static_cast<float>(n_ret);
+  gap[b] = g;
+  if (skip) skip[b] = g <= delta ? 1 : 0;
 }
 
 // ---------------------------------------------------------------- Eq. 8 / 9
@@ -180,6 +193,8 @@ __global__ void __launch_bounds__(kGateThreads) saliency_kernel(const float* __r
                                                                  int M, int I, int C_keep,
                                                                  const float* __restrict__ norms, float* saliency,
                                                                  float* part_ws) {
+  griddep_wait();
+  griddep_launch_dependents();
   __shared__ double red[2][kGateThreads / 32];
   const int c = blockIdx.x * kGateThreads + threadIdx.x;
   double s = 0.0;
@@ -213,6 +228,8 @@ __global__ void __launch_bounds__(kGateThreads) saliency_kernel(const float* __r
 
 // One thread: leakage of Eq. 9 and the pruned-or-full decision.
 __global__ void leakage_kernel(const float* part_ws, int n_blocks, float delta, float* leakage, uint8_t* use_pruned) {
+  griddep_wait();
+  griddep_launch_dependents();
   if (threadIdx.x != 0 || blockIdx.x != 0) return;
   double kept = 0.0, pruned = 0.0;
   for (int b = 0; b < n_blocks; ++b) {
@@ -228,6 +245,8 @@ __global__ void leakage_kernel(const float* part_ws, int n_blocks, float delta, 
 // One warp per row: ||W[r, :]||_2 in fp32 (static per-layer input of Eq. 8).
 __global__ void __launch_bounds__(kStatThreads) row_norm_kernel(const uint4* __restrict__ W, int d8, int rows,
                                                                  float* __restrict__ norms) {
+  griddep_wait();
+  griddep_launch_dependents();
   const int lane = threadIdx.x & 31;
   const int wpb = blockDim.x >> 5;
   for (int r = blockIdx.x * wpb + (threadIdx.x >> 5); r < rows; r += gridDim.x * wpb) {
@@ -253,26 +272,26 @@ cudaError_t launch_ffn_gate(const float* colsum, int n_parts, int M, int I, int 
                             float delta, float* saliency, float* part_ws, float* leakage, uint8_t* use_pruned,
                             cudaStream_t stream) {
   const int blocks = (I + kGateThreads - 1) / kGateThreads;
-  saliency_kernel<<<blocks, kGateThreads, 0, stream>>>(colsum, n_parts, M, I, C_keep, norms, saliency, part_ws);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = launch_k(saliency_kernel, dim3(blocks), dim3(kGateThreads), 0, stream, 1, colsum, n_parts, M, I,
+                           C_keep, norms, saliency, part_ws);
   if (e != cudaSuccess) return e;
-  leakage_kernel<<<1, 32, 0, stream>>>(part_ws, blocks, delta, leakage, use_pruned);
-  return cudaGetLastError();
+  return launch_k(leakage_kernel, dim3(1), dim3(32), 0, stream, 1, static_cast<const float*>(part_ws), blocks, delta,
+                  leakage, use_pruned);
 }
 
 cudaError_t launch_row_norms(const __nv_bfloat16* W, int rows, int d, float* norms, int n_sm, cudaStream_t stream) {
   if (rows == 0) return cudaSuccess;
   int blocks = (rows + 7) / 8;
   if (blocks > n_sm * 8) blocks = n_sm * 8;
-  row_norm_kernel<<<blocks, kStatThreads, 0, stream>>>(reinterpret_cast<const uint4*>(W), d / 8, rows, norms);
-  return cudaGetLastError();
+  return launch_k(row_norm_kernel, dim3(blocks), dim3(kStatThreads), 0, stream, 1, reinterpret_cast<const uint4*>(W),
+                  d / 8, rows, norms);
 }
 
 cudaError_t launch_drop_stats(const uint8_t* mask_t, const uint8_t* mask_ref, int B, int N, int r0, int r1,
                               float* jac, float* jrand, float* rda, int32_t* counts, cudaStream_t stream) {
   if (B == 0) return cudaSuccess;
-  drop_stats_kernel<<<B, kStatThreads, 0, stream>>>(mask_t, mask_ref, N, r0, r1, jac, jrand, rda, counts);
-  return cudaGetLastError();
+  return launch_k(drop_stats_kernel, dim3(B), dim3(kDropThreads), 0, stream, 1, mask_t, mask_ref, N, r0, r1, jac,
+                  jrand, rda, counts);
 }
 
 cudaError_t launch_redundancy_gap(const __nv_bfloat16* h_in, const __nv_bfloat16* h_out, const uint8_t* mask,
@@ -284,13 +303,13 @@ cudaError_t launch_redundancy_gap(const __nv_bfloat16* h_in, const __nv_bfloat16
     long blocks = (rows + 7) / 8;
     const long cap = static_cast<long>(n_sm) * 8;
     if (blocks > cap) blocks = cap;
-    row_cosine_kernel<<<static_cast<unsigned>(blocks), kStatThreads, 0, stream>>>(
-        reinterpret_cast<const uint4*>(h_in), reinterpret_cast<const uint4*>(h_out), d / 8, rows, cos_ws);
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = launch_k(row_cosine_kernel, dim3(static_cast<unsigned>(blocks)), dim3(kStatThreads), 0, stream,
+                             1, reinterpret_cast<const uint4*>(h_in), reinterpret_cast<const uint4*>(h_out), d / 8,
+                             rows, cos_ws);
     if (e != cudaSuccess) return e;
   }
-  gap_reduce_kernel<<<B, kStatThreads, 0, stream>>>(cos_ws, mask, N, delta, gap, skip);
-  return cudaGetLastError();
+  return launch_k(gap_reduce_kernel, dim3(B), dim3(kStatThreads), 0, stream, 1, static_cast<const float*>(cos_ws),
+                  mask, N, delta, gap, skip);
 }
 
 }  // namespace cer

@@ -153,6 +153,8 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1) umma_gemm_kernel(const _
   }
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  griddep_wait();                 // inputs written by the previous kernel are visible
+  griddep_launch_dependents();
 
   const int ntiles = P::num_tiles(p);
   const int nkb = P::num_kb(p);

@@ -1,7 +1,7 @@
 """GPU parity of the UCS statistics (Sec. 3.4) against the oracle: drop-set
 counts exact and J / J_rand / RDA bit-exact (both sides form them in fp64 from
-the same integers); the redundancy gap within 2e-5 absolute (fp32 cosines,
-fp64 means), its skip decision equal away from the threshold."""
+the same integers); the redundancy gap within 2e-5 absolute (fp32 cosines and
+means), its skip decision equal away from the threshold."""
 import numpy as np
 import pytest
 import torch
