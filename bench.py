@@ -425,7 +425,7 @@ def run_gpu(args, info):
         "warmup": args.warmup, "ms_per_step": slow_ms, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": workload_config(w, True),
-        "roofline": {"kernel": "ffn gate/up GEMM (tcgen05, fused row gather + SwiGLU)", "bound": "tensor",
+        "roofline": {"kernel": "ffn gate/up GEMM (tcgen05 pair MMA, SwiGLU epilogue)", "bound": "tensor",
                      "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
                      "peak_source": f"bf16_tflops (burst) of {peak_kind}",
                      "algorithmic_flops_per_launch": gateup_flops,

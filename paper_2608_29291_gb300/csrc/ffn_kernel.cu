@@ -35,17 +35,19 @@ __device__ __forceinline__ float silu_mul(float g, float u) {
 
 // ---------------------------------------------------------------- gate/up
 
+// Two CTAs of a cluster take adjacent 128-row tiles of the same 128 channels
+// as one M=256 x N=256 pair MMA: rank 0 holds the gate rows of the weight
+// tile, rank 1 the up rows, and each CTA receives only its own 32 KB per K
+// block (the one-CTA form with the weight tile multicast to both received
+// 48 KB and measured 3-6% slower); the ring has room for six slots.
 template <int EPI_WARPS_>
 struct GateUpProblemT {
   static constexpr int BN = 256;
-  static constexpr int STAGES = 4;
+  static constexpr int MMA_PAIR = 1;
+  static constexpr int STAGES = 6;
   static constexpr int B_MN_MAJOR = 0;
   static constexpr int EPI_WARPS = EPI_WARPS_;
   static constexpr int kGroups = EPI_WARPS / 4;
-  // Two CTAs per cluster take adjacent 128-row tiles of the same 128
-  // channels: rank 0 fetches the gate rows of the B tile, rank 1 the up rows,
-  // each multicast to both, so each CTA reads 32 KB instead of 48 KB of L2
-  // per K block.
   static constexpr int CLUSTER = 2;
   static constexpr uint32_t kBStepBytes = 32;
   static constexpr uint32_t kBoxBytes = 128 * 128;          // 128 rows x 64 bf16
@@ -67,21 +69,20 @@ struct GateUpProblemT {
   // Cluster tile t covers row tiles 2*(t % n_mtp) + {0, 1} and channel tile t / n_mtp.
   __device__ static int num_tiles(const Params& p) { return p.n_mtp * p.n_ct; }
   __device__ static int num_kb(const Params& p) { return p.d / 64; }
-  __device__ static uint32_t stage_bytes(const Params&, int, int) { return kATileBytes + BN * 128; }
+  __device__ static uint32_t stage_bytes(const Params&, int, int) { return 2 * (kATileBytes + 128 * 128); }
   __device__ static void prod_tile(const Params& p, int tile, int rank, ProdState& st) {
     st.c0 = (tile / p.n_mtp) * 128;
     st.m0 = (2 * (tile % p.n_mtp) + rank) * 128;   // rows past M load as zeros
     st.rank = rank;
   }
+  // Pair MMA: N columns 0..127 (gate) come from rank 0's B slot, 128..255 (up)
+  // from rank 1's; every copy counts on the even CTA's barrier.
   __device__ static void prod_kb(const Params& p, const ProdState& st, int, int kb, int lane, uint8_t* a,
-                                 uint8_t* b, uint64_t* bar) {
+                                 uint8_t* b, uint32_t leader_bar) {
     if (lane == 0) {
       const int x = kb * 64;
-      tma_load_2d(a, &p.tm_x, bar, x, st.m0);
-      if (st.rank == 0)
-        tma_load_2d_multicast(b, &p.tm_wg, bar, x, st.c0, 0x3);
-      else
-        tma_load_2d_multicast(b + 128 * 128, &p.tm_wu, bar, x, st.c0, 0x3);
+      tma_load_2d_pair(a, &p.tm_x, leader_bar, x, st.m0);
+      tma_load_2d_pair(b, st.rank == 0 ? &p.tm_wg : &p.tm_wu, leader_bar, x, st.c0);
     }
   }
   __device__ static uint64_t bdesc(uint32_t saddr) { return sdesc_kmajor_sw128(saddr); }
@@ -146,22 +147,28 @@ using GateUpProblem = GateUpProblemT<4>;
 
 // ---------------------------------------------------------------- down
 
-// CL = 2: two CTAs per cluster take adjacent N tiles of the same 128 rows;
-// each loads 64 of the act tile's rows and multicasts them to both.
-template <int BN_, int CL>
+// PAIR_ = 0: one CTA per 128 x BN tile.
+// PAIR_ = 1: two CTAs of a cluster take adjacent 128-row tiles as one M=256 x
+// N=BN pair MMA; each holds its act rows and BN/2 of the B columns, so it
+// streams 16 KB of act and BN*64 bytes of WdT per K block for a 128 x BN
+// output tile.
+template <int BN_, int PAIR_>
 struct DownProblem {
   static constexpr int BN = BN_;
-  static constexpr int ATOMS = BN / 64;
-  static constexpr int STAGES = BN == 256 ? 4 : BN == 192 ? 5 : 6;
+  static constexpr int MMA_PAIR = PAIR_;
+  static constexpr int CLUSTER = PAIR_ ? 2 : 1;
+  static constexpr int CTA_N = PAIR_ ? BN / 2 : BN;   // B columns in one CTA's ring slot
+  static constexpr int ATOMS = CTA_N / 64;
+  static constexpr int STAGES = PAIR_ ? 7 : BN == 256 ? 4 : BN == 192 ? 5 : 6;
   static constexpr int B_MN_MAJOR = 1;
   static constexpr int EPI_WARPS = 8;
-  static constexpr int CLUSTER = CL;
   static constexpr uint32_t kBStepBytes = 2048;     // 16 K-rows = two 1024 B row groups
   static constexpr uint32_t kAtomBytes = 64 * 128;  // 64 K-rows x 64 columns
   static constexpr uint32_t kEpiSmemBytes = 0;
+  static_assert(CTA_N % 64 == 0, "whole 64-column B atoms per CTA");
 
   struct Params {
-    CUtensorMap tm_act;  // act [M, C], box 64 x 128 (64 x 64 with CL = 2)
+    CUtensorMap tm_act;  // act [M, C], box 64 x 128
     CUtensorMap tm_wdt;  // WdT [C, d], box 64 x 64
     const int32_t* idx;          // scatter mode: keep list [B][k_tot]
     const __nv_bfloat16* hin;    // scatter mode: residual input
@@ -169,49 +176,61 @@ struct DownProblem {
     const uint8_t* use_small_k;  // optional device flag: contract only the first C_small channels
     int* status;
     int scatter;
-    int M, d, C, C_small, N, k_tot, n_mt, n_nt, n_ntc;   // n_ntc: N-tile groups of CL
+    int M, d, C, C_small, N, k_tot, n_mt, n_mtp, n_nt;   // n_mtp: row-tile pairs
   };
   struct ProdState {
-    int m0, n0, n_atoms, rank;
+    int m0, n0, n_atoms;
   };
 
-  // Cluster tile t: row tile t % n_mt, N tiles CL * (t / n_mt) + rank.
-  __device__ static int num_tiles(const Params& p) { return p.n_mt * p.n_ntc; }
-  __device__ static int ntile(const Params& p, int tile, int rank) { return CL * (tile / p.n_mt) + rank; }
+  // Tile t: N tile t / R and row tile t % R (pair: rows 2 (t % R) + rank),
+  // R = row tiles (pairs).
+  __device__ static int rows_per_n(const Params& p) { return PAIR_ ? p.n_mtp : p.n_mt; }
+  __device__ static int num_tiles(const Params& p) { return rows_per_n(p) * p.n_nt; }
+  __device__ static int row_tile(const Params& p, int tile, int rank) {
+    const int r = tile % rows_per_n(p);
+    return PAIR_ ? 2 * r + rank : r;
+  }
   __device__ static int num_kb(const Params& p) {
     return (p.use_small_k != nullptr && *p.use_small_k) ? p.C_small / 64 : p.C / 64;
   }
   __device__ static int atoms(const Params& p, int nt) {
-    const int left = (p.d - nt * BN) / 64;    // an N tile past d (odd pair) loads no B
-    return left < 0 ? 0 : left < ATOMS ? left : ATOMS;
+    const int left = (p.d - nt * BN) / 64;
+    return left < ATOMS ? left : ATOMS;
   }
+  // The pair always loads whole atoms (columns past d read as zeros), so both
+  // CTAs' byte counts are known to the even CTA.
   __device__ static uint32_t stage_bytes(const Params& p, int tile, int) {
-    return kATileBytes + atoms(p, ntile(p, tile, static_cast<int>(CL > 1 ? cluster_ctarank() : 0))) * kAtomBytes;
+    if (PAIR_) return 2 * (kATileBytes + ATOMS * kAtomBytes);
+    return kATileBytes + atoms(p, tile / rows_per_n(p)) * kAtomBytes;
   }
   __device__ static void prod_tile(const Params& p, int tile, int rank, ProdState& st) {
-    const int nt = ntile(p, tile, rank);
-    st.n0 = nt * BN;
-    st.m0 = (tile % p.n_mt) * 128;
-    st.n_atoms = atoms(p, nt);
-    st.rank = rank;
+    const int nt = tile / rows_per_n(p);
+    st.m0 = row_tile(p, tile, rank) * 128;   // rows past M load as zeros
+    st.n0 = nt * BN + (PAIR_ ? rank * CTA_N : 0);
+    st.n_atoms = PAIR_ ? ATOMS : atoms(p, nt);
   }
   __device__ static void prod_kb(const Params& p, const ProdState& st, int, int kb, int lane, uint8_t* a,
                                  uint8_t* b, uint64_t* bar) {
     if (lane == 0) {
-      if (CL == 1) {
-        tma_load_2d(a, &p.tm_act, bar, kb * 64, st.m0);
-      } else {
-        tma_load_2d_multicast(a + st.rank * (kATileBytes / 2), &p.tm_act, bar, kb * 64, st.m0 + 64 * st.rank, 0x3);
-      }
+      tma_load_2d(a, &p.tm_act, bar, kb * 64, st.m0);
       for (int at = 0; at < st.n_atoms; ++at) tma_load_2d(b + at * kAtomBytes, &p.tm_wdt, bar, st.n0 + at * 64, kb * 64);
+    }
+  }
+  __device__ static void prod_kb(const Params& p, const ProdState& st, int, int kb, int lane, uint8_t* a,
+                                 uint8_t* b, uint32_t leader_bar) {
+    if (lane == 0) {
+      tma_load_2d_pair(a, &p.tm_act, leader_bar, kb * 64, st.m0);
+#pragma unroll
+      for (int at = 0; at < ATOMS; ++at)
+        tma_load_2d_pair(b + at * kAtomBytes, &p.tm_wdt, leader_bar, st.n0 + at * 64, kb * 64);
     }
   }
   __device__ static uint64_t bdesc(uint32_t saddr) { return sdesc_mnmajor_sw128(saddr, kAtomBytes, 1024); }
 
   __device__ static void epilogue_done(const Params&, int, int) {}
   __device__ static bool epilogue(const Params& p, int tile, int row, int half, uint32_t taddr, EpiCtx& ctx) {
-    const int nt = ntile(p, tile, ctx.rank);
-    const int m = (tile % p.n_mt) * 128 + row;
+    const int nt = tile / rows_per_n(p);
+    const int m = row_tile(p, tile, ctx.rank) * 128 + row;
     bool valid = m < p.M;
     size_t dst_row = 0;
     if (valid) {
@@ -318,11 +337,11 @@ cudaError_t launch_ffn_gateup(const FfnArgs& a, int n_sm, cudaStream_t stream) {
   return launch_gemm<GateUpProblem>(p, p.n_mtp * p.n_ct, n_sm, stream);
 }
 
-template <int BN, int CL>
+template <int BN, int PAIR>
 static cudaError_t launch_down(const FfnArgs& a, int n_sm, cudaStream_t stream) {
-  using P = DownProblem<BN, CL>;
+  using P = DownProblem<BN, PAIR>;
   typename P::Params p{};
-  if (!encode_bf16_2d(&p.tm_act, a.act, a.M, a.C, 64, CL == 1 ? 128 : 64)) return cudaErrorInvalidValue;
+  if (!encode_bf16_2d(&p.tm_act, a.act, a.M, a.C, 64, 128)) return cudaErrorInvalidValue;
   if (!encode_bf16_2d(&p.tm_wdt, a.WdT, a.C, a.d, 64, 64)) return cudaErrorInvalidValue;
   p.idx = a.idx;
   p.hin = a.h;
@@ -337,15 +356,19 @@ static cudaError_t launch_down(const FfnArgs& a, int n_sm, cudaStream_t stream) 
   p.N = a.N;
   p.k_tot = a.k_tot;
   p.n_mt = (a.M + 127) / 128;
+  p.n_mtp = (p.n_mt + 1) / 2;
   p.n_nt = (a.d + BN - 1) / BN;
-  p.n_ntc = (p.n_nt + CL - 1) / CL;
-  return launch_gemm<P>(p, p.n_mt * p.n_ntc, n_sm, stream);
+  return launch_gemm<P>(p, (PAIR ? p.n_mtp : p.n_mt) * p.n_nt, n_sm, stream);
 }
 
-// N-tile width of the down GEMM: the one with the least per-SM work
-// (waves x width), the wider on a tie.
+// Tile shape of the down GEMM.  With at least two row tiles: 256-row pair
+// tiles 256 columns wide (the act and WdT streams per flop are what bound
+// this contraction; the one-CTA 128 x 192 tile measured about 1.3x slower
+// even where it fills every SM).  Otherwise one CTA per 128 x BN tile, BN the
+// width with the least per-SM work (waves x width), the wider on a tie.
 int down_tile_width(int M, int d, int n_sm) {
   const long n_mt = (M + 127) / 128;
+  if (n_mt >= 2) return 0;
   int best = 256;
   long best_cost = -1;
   for (int bn : {256, 192, 128}) {
@@ -359,14 +382,12 @@ int down_tile_width(int M, int d, int n_sm) {
   return best;
 }
 
-// One CTA per tile.  (Pairs of N tiles sharing the act tile through cluster
-// multicast, DownProblem<BN, 2>, measured 6-7% slower on the 1.5B and 7B
-// workloads: the paired pipelines wait on each other.)
 cudaError_t launch_ffn_down(const FfnArgs& a, int n_sm, cudaStream_t stream) {
   switch (down_tile_width(a.M, a.d, n_sm)) {
-    case 192: return launch_down<192, 1>(a, n_sm, stream);
-    case 128: return launch_down<128, 1>(a, n_sm, stream);
-    default: return launch_down<256, 1>(a, n_sm, stream);
+    case 0: return launch_down<256, 1>(a, n_sm, stream);
+    case 192: return launch_down<192, 0>(a, n_sm, stream);
+    case 128: return launch_down<128, 0>(a, n_sm, stream);
+    default: return launch_down<256, 0>(a, n_sm, stream);
   }
 }
 

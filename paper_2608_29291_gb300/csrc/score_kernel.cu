@@ -122,6 +122,7 @@ struct ScoreProblem {
   static constexpr int B_MN_MAJOR = 0;
   static constexpr int EPI_WARPS = 8;
   static constexpr int CLUSTER = 1;
+  static constexpr int MMA_PAIR = 0;
   static constexpr uint32_t kBStepBytes = 32;
   static constexpr uint32_t kEpiSmemBytes = 0;
 

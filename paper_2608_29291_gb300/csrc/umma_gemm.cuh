@@ -19,15 +19,28 @@
 // one cluster tile (two adjacent 128-row tiles sharing a B tile): each loads
 // half of B and multicasts it to both, each MMA commit frees the ring slot
 // in both CTAs, and cluster barriers bracket start-up and teardown so no CTA
-// exits while its peer may still write into its shared memory.  Every wait is bounded (ptx.cuh); on a timeout the CTA unwinds,
-// waits briefly for its own copies and MMAs, frees TMEM and exits.
+// exits while its peer may still write into its shared memory.
+//
+// With MMA_PAIR == 1 (CLUSTER == 2) the cluster runs one M=256 x N=BN pair MMA
+// per K step instead (tcgen05 cta_group::2): each CTA loads its 128 A rows
+// and its half of the B tile into its own ring, all of the pair's copies are
+// counted on the even CTA's ring barrier, the even CTA's warp 1 issues the
+// MMAs and its commits free the ring slot and publish the accumulator in both
+// CTAs, and each epilogue warp frees its accumulator buffer with one arrival
+// on the even CTA's barrier.  Each SM then streams 128 x 64 of A plus
+// BN/2 x 64 of B per K step instead of the whole B tile.
+//
+// Every wait is bounded (ptx.cuh); on a timeout the CTA unwinds, waits
+// briefly for its own copies and MMAs, frees TMEM and exits.
 //
 // A problem class P supplies:
-//   BN, STAGES, B_MN_MAJOR, EPI_WARPS, CLUSTER, kBStepBytes,
+//   BN, STAGES, B_MN_MAJOR, EPI_WARPS, CLUSTER, MMA_PAIR, kBStepBytes,
 //   Params (with `int* status`), num_tiles(p) (cluster tiles),
 //   num_kb(p), prod_tile(p, tile, rank, state),
-//   prod_kb(p, state, tile, kb, lane, a_smem, b_smem, bar),
-//   stage_bytes(p, tile, kb), bdesc(saddr),
+//   prod_kb(p, state, tile, kb, lane, a_smem, b_smem, bar) (with MMA_PAIR,
+//   `bar` is the cluster address of the even CTA's ring barrier),
+//   stage_bytes(p, tile, kb) (with MMA_PAIR, the bytes of both CTAs),
+//   bdesc(saddr),
 //   kEpiSmemBytes (shared memory reserved for the epilogue, may be 0),
 //   epilogue(p, tile, row, half, taddr, ctx) -> false to abort (ctx.rank is
 //   the CTA's rank in its cluster): columns
@@ -54,9 +67,21 @@ struct TmemCols {
   static constexpr uint32_t value = need <= 32 ? 32 : need <= 64 ? 64 : need <= 128 ? 128 : need <= 256 ? 256 : 512;
 };
 
+// Bytes of one ring slot's B tile in one CTA (half of it with a pair MMA).
+template <class P>
+__host__ __device__ constexpr uint32_t b_stage_bytes() {
+  return static_cast<uint32_t>(P::MMA_PAIR ? P::BN / 2 : P::BN) * 128u;
+}
+
 template <class P>
 constexpr size_t gemm_smem_bytes() {
-  return 1024 + static_cast<size_t>(P::STAGES) * (kATileBytes + P::BN * 128) + P::kEpiSmemBytes + 256;
+  return 1024 + static_cast<size_t>(P::STAGES) * (kATileBytes + b_stage_bytes<P>()) + P::kEpiSmemBytes + 256;
+}
+
+// Sleep about `ns` nanoseconds (bounded; used only while unwinding).
+__device__ __forceinline__ void unwind_pause(uint64_t ns) {
+  const uint64_t t0 = globaltimer_ns();
+  while (globaltimer_ns() - t0 < ns) __nanosleep(1000);
 }
 
 // A short, abort-independent wait used only while unwinding.
@@ -99,12 +124,14 @@ template <class P>
 __global__ void __launch_bounds__(gemm_threads<P>(), 1) umma_gemm_kernel(const __grid_constant__ typename P::Params p) {
   static_assert(P::EPI_WARPS == 4 || P::EPI_WARPS == 8, "epilogue is one or two groups of four warps");
   static_assert(P::CLUSTER == 1 || P::CLUSTER == 2, "clusters of one or two CTAs");
+  constexpr bool PAIR = P::MMA_PAIR != 0;
+  static_assert(!PAIR || P::CLUSTER == 2, "a pair MMA runs on a 2-CTA cluster");
   constexpr uint16_t kPairMask = 0x3;
   constexpr int BN = P::BN;
   constexpr int STAGES = P::STAGES;
-  constexpr uint32_t B_BYTES = BN * 128;
+  constexpr uint32_t B_BYTES = b_stage_bytes<P>();
   constexpr uint32_t TMEM_COLS = TmemCols<BN>::value;
-  constexpr uint32_t IDESC = idesc_bf16(128, BN, P::B_MN_MAJOR);
+  constexpr uint32_t IDESC = idesc_bf16(PAIR ? 256 : 128, BN, P::B_MN_MAJOR);
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -129,11 +156,13 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1) umma_gemm_kernel(const _
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], P::CLUSTER);   // one MMA commit from each CTA of the cluster
+      // One MMA commit from each CTA of the cluster (from the even CTA alone with a pair MMA).
+      mbar_init(&empty[s], PAIR ? 1 : P::CLUSTER);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull[a], 1);
-      mbar_init(&tempty[a], 32 * P::EPI_WARPS);
+      // Every epilogue thread (with a pair MMA: every epilogue warp of both CTAs).
+      mbar_init(&tempty[a], PAIR ? 2 * P::EPI_WARPS : 32 * P::EPI_WARPS);
     }
     mbar_init(drain, 1);
     mbar_init(&half_bar[0], 128);
@@ -142,8 +171,13 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1) umma_gemm_kernel(const _
     fence_mbar_init();
   }
   if (warp == 1) {
-    tmem_alloc(tmem_slot, TMEM_COLS);
-    tmem_relinquish();
+    if (PAIR) {
+      tmem_alloc_pair(tmem_slot, TMEM_COLS);   // together with warp 1 of the peer CTA
+      tmem_relinquish_pair();
+    } else {
+      tmem_alloc(tmem_slot, TMEM_COLS);
+      tmem_relinquish();
+    }
   }
   tc_fence_before();
   if (P::CLUSTER > 1) {
@@ -166,6 +200,8 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1) umma_gemm_kernel(const _
     uint32_t phase = 0;
     long issued = 0;
     bool ok = true;
+    // With a pair MMA the even CTA's ring barriers count both CTAs' copies.
+    const uint32_t leader_full = PAIR ? mapa_shared(smem_u32(full), 0) : 0u;
     for (int tile = cluster_id; tile < ntiles && ok; tile += n_clusters) {
       P::prod_tile(p, tile, rank, st);
       for (int kb = 0; kb < nkb; ++kb) {
@@ -173,10 +209,17 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1) umma_gemm_kernel(const _
           ok = false;
           break;
         }
-        const uint32_t bytes = P::stage_bytes(p, tile, kb);
-        if (lane == 0) mbar_arrive_expect_tx(&full[stage], bytes);
+        if (!PAIR || rank == 0) {
+          const uint32_t bytes = P::stage_bytes(p, tile, kb);
+          if (lane == 0) mbar_arrive_expect_tx(&full[stage], bytes);
+        }
         __syncwarp();
-        P::prod_kb(p, st, tile, kb, lane, a_ring + stage * kATileBytes, b_ring + stage * B_BYTES, &full[stage]);
+        if constexpr (PAIR) {
+          P::prod_kb(p, st, tile, kb, lane, a_ring + stage * kATileBytes, b_ring + stage * B_BYTES,
+                     leader_full + static_cast<uint32_t>(stage) * 8u);
+        } else {
+          P::prod_kb(p, st, tile, kb, lane, a_ring + stage * kATileBytes, b_ring + stage * B_BYTES, &full[stage]);
+        }
         ++issued;
         if (++stage == STAGES) {
           stage = 0;
@@ -185,11 +228,16 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1) umma_gemm_kernel(const _
       }
     }
     if (!ok && lane == 0) {
-      // Let the copies already issued land before the CTA's memory goes away.
-      for (long n = issued - 1; n >= 0 && n >= issued - STAGES; --n)
-        drain_wait(&full[n % STAGES], static_cast<uint32_t>((n / STAGES) & 1));
+      // Let the copies already issued land before the CTA's memory goes away
+      // (the odd CTA of a pair cannot see the barrier its copies count on).
+      if (PAIR && rank != 0) {
+        unwind_pause(1000000ull);
+      } else {
+        for (long n = issued - 1; n >= 0 && n >= issued - STAGES; --n)
+          drain_wait(&full[n % STAGES], static_cast<uint32_t>((n / STAGES) & 1));
+      }
     }
-  } else if (warp == 1) {
+  } else if (warp == 1 && (!PAIR || rank == 0)) {
     // ---------------------------------------------------------------- MMA issuer
     int stage = 0;
     uint32_t phase = 0;
@@ -215,10 +263,16 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1) umma_gemm_kernel(const _
           const uint32_t b_base = smem_u32(b_ring + stage * B_BYTES);
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
-            umma_bf16(d_tmem, sdesc_kmajor_sw128(a_base + k * 32), P::bdesc(b_base + k * P::kBStepBytes), IDESC,
-                      (kb | k) != 0 ? 1u : 0u);
+            const uint64_t adesc = sdesc_kmajor_sw128(a_base + k * 32);
+            const uint64_t bdesc = P::bdesc(b_base + k * P::kBStepBytes);
+            if (PAIR)
+              umma_bf16_pair(d_tmem, adesc, bdesc, IDESC, (kb | k) != 0 ? 1u : 0u);
+            else
+              umma_bf16(d_tmem, adesc, bdesc, IDESC, (kb | k) != 0 ? 1u : 0u);
           }
-          if (P::CLUSTER > 1)
+          if (PAIR)
+            umma_commit_pair_multicast(&empty[stage], kPairMask);
+          else if (P::CLUSTER > 1)
             umma_commit_multicast(&empty[stage], kPairMask);   // frees the slot in both CTAs
           else
             umma_commit(&empty[stage]);
@@ -231,7 +285,12 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1) umma_gemm_kernel(const _
         }
       }
       if (!ok) break;
-      if (lane == 0) umma_commit(&tfull[acc]);
+      if (lane == 0) {
+        if (PAIR)
+          umma_commit_pair_multicast(&tfull[acc], kPairMask);   // both CTAs' epilogues
+        else
+          umma_commit(&tfull[acc]);
+      }
       __syncwarp();
       if (++acc == 2) {
         acc = 0;
@@ -239,15 +298,19 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1) umma_gemm_kernel(const _
       }
     }
     if (!ok && lane == 0 && issued_any) {
-      umma_commit(drain);
+      if (PAIR)
+        umma_commit_pair(drain);
+      else
+        umma_commit(drain);
       drain_wait(drain, 0);
     }
-  } else {
+  } else if (warp >= 2) {
     // ---------------------------------------------------------------- epilogue
     const int q = warp & 3;            // TMEM lane quadrant this warp may access
     const int row = q * 32 + lane;     // accumulator row = TMEM lane
     const int half = (warp - 2) >> 2;  // which half of the accumulator columns
     EpiCtx ctx{epi_smem, rank, &half_bar[half], 0u, abort_flag, p.status};
+    const uint32_t leader_tempty = PAIR ? mapa_shared(smem_u32(tempty), 0) : 0u;
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int tile = cluster_id; tile < ntiles; tile += n_clusters) {
@@ -256,7 +319,12 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1) umma_gemm_kernel(const _
       const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BN);
       const bool ok = P::epilogue(p, tile, row, half, taddr, ctx);
       tc_fence_before();
-      mbar_arrive(&tempty[acc]);
+      if (PAIR) {
+        __syncwarp();
+        if (lane == 0) mbar_arrive_cluster(leader_tempty + static_cast<uint32_t>(acc) * 8u);
+      } else {
+        mbar_arrive(&tempty[acc]);
+      }
       if (!ok) break;
       if (++acc == 2) {
         acc = 0;
@@ -274,7 +342,10 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1) umma_gemm_kernel(const _
   }
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, TMEM_COLS);
+    if (PAIR)
+      tmem_dealloc_pair(tmem_base, TMEM_COLS);   // together with warp 1 of the peer CTA
+    else
+      tmem_dealloc(tmem_base, TMEM_COLS);
   }
 }
 
