@@ -154,7 +154,9 @@ cer_status cer_gather(const void* h, int B, int N, int d, const int32_t* idx, in
  * Two tcgen05 GEMMs (bf16 operands, fp32 accumulation in TMEM) over dense
  * TMA tiles; with chan != NULL the kept weight rows are first copied into the
  * workspace (3*C*d*2 bytes moved twice per call).  The SwiGLU activation
- * passes through the workspace as bf16 [M, C].
+ * passes through the workspace as bf16 [M, C]; for M > 0 the workspace also
+ * holds 24 MiB + 8 KiB in which the two GEMMs split output tiles by
+ * contraction block across SM pairs and add the fp32 partial sums.
  * Workspace: cer_routed_ffn_workspace_size(M, d, C, chan != NULL).         */
 cer_status cer_routed_ffn(const void* X, int M, int d,
                           const void* Wg, const void* Wu, const void* WdT, int I,

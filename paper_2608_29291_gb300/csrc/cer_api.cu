@@ -83,6 +83,18 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 size_t round256(size_t x) { return (x + 255) & ~size_t(255); }
 
+// The GEMMs' stream-K region (partial accumulators, then flags), placed right
+// after the act buffer of every FFN workspace.
+size_t ffn_stream_k_bytes(long long M) {
+  return M > 0 ? cer::kStreamKPartialBytes + cer::kStreamKFlagBytes : 0;
+}
+void carve_stream_k(char** ws, long long M, cer::FfnArgs* a) {
+  if (M <= 0) return;
+  a->sk_partial = reinterpret_cast<float*>(*ws);
+  a->sk_flags = reinterpret_cast<unsigned long long*>(*ws + cer::kStreamKPartialBytes);
+  *ws += ffn_stream_k_bytes(M);
+}
+
 #define CER_REQUIRE(cond, status, ...) \
   do {                                 \
     if (!(cond)) return fail(status, __VA_ARGS__); \
@@ -423,7 +435,7 @@ cer_status cer_pack_ffn_weights(const void* Wg, const void* Wu, const void* WdT,
 
 size_t cer_routed_ffn_workspace_size(int M, int d, int C, int with_chan) {
   if (M < 0 || d < 0 || C < 0) return 0;
-  size_t ws = round256(static_cast<size_t>(M) * C * 2);
+  size_t ws = round256(static_cast<size_t>(M) * C * 2) + ffn_stream_k_bytes(M);
   if (with_chan) ws += 3 * round256(static_cast<size_t>(C) * d * 2);
   return ws;
 }
@@ -482,6 +494,7 @@ cer_status cer_routed_ffn(const void* X, int M, int d, const void* Wg, const voi
   cer::FfnArgs a{};
   a.act = reinterpret_cast<__nv_bfloat16*>(ws);
   ws += round256(static_cast<size_t>(M) * C * 2);
+  carve_stream_k(&ws, M, &a);
   const __nv_bfloat16* w[3];
   if ((s = ffn_weight_slices(Wg, Wu, WdT, I, d, chan, C, &ws, w, dev, stream)) != CER_OK) return s;
   a.X = static_cast<const __nv_bfloat16*>(X);
@@ -633,6 +646,8 @@ cer_status routed_block_impl(void* h, void* out, int B, int N, int d, const cer_
   ws += round256(static_cast<size_t>(M64) * d * 2);
   __nv_bfloat16* act = reinterpret_cast<__nv_bfloat16*>(ws);
   ws += round256(static_cast<size_t>(M64) * C * 2);
+  cer::FfnArgs fa{};
+  carve_stream_k(&ws, M64, &fa);
   char* gate_ws = ws + (chan ? 3 * round256(static_cast<size_t>(C) * d * 2) : 0);
 
   // S1: scorer GEMM -> partial sums
@@ -669,7 +684,6 @@ cer_status routed_block_impl(void* h, void* out, int B, int N, int d, const cer_
   if ((e = mark(3)) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
 
   // S4: gate/up GEMM with the SwiGLU epilogue
-  cer::FfnArgs fa{};
   fa.X = X;
   fa.M = static_cast<int>(M64);
   fa.d = d;
@@ -788,6 +802,7 @@ cer_status cer_routed_ffn_gated(const void* X, int M, int d, const void* Wg, con
   cer::FfnArgs a{};
   a.act = reinterpret_cast<__nv_bfloat16*>(ws);
   ws += round256(static_cast<size_t>(M) * I * 2);
+  carve_stream_k(&ws, M, &a);
   a.X = static_cast<const __nv_bfloat16*>(X);
   a.M = M;
   a.d = d;

@@ -284,7 +284,7 @@ static cudaError_t launch_score_gemm(const ScoreArgs& a, const float* bias_tab, 
   cudaError_t e = ensure_max_smem(reinterpret_cast<const void*>(umma_gemm_kernel<P>), smem);
   if (e != cudaSuccess) return e;
   const int grid = tiles < n_sm ? tiles : n_sm;
-  return launch_k(umma_gemm_kernel<P>, dim3(grid), dim3(gemm_threads<P>()), smem, stream, 1, p);
+  return launch_k(umma_gemm_kernel<P>, dim3(grid), dim3(gemm_threads<P>()), smem, stream, 1, p, StreamK{});
 }
 
 cudaError_t launch_score(const ScoreArgs& a, const ScoreWorkspace& ws, int n_sm, cudaStream_t stream,

@@ -13,22 +13,43 @@
 //              TMEM (lane = tile row; with 8 warps, warps 2-5 take the first
 //              half of the columns and warps 6-9 the second) and apply the
 //              problem's fused epilogue.
-// The accumulator is double-buffered in TMEM so the epilogue of tile i
-// overlaps the MMAs of tile i+1.  Tiles are visited with a stride of the
-// number of clusters.  With CLUSTER == 2 the two CTAs of a cluster work on
-// one cluster tile (two adjacent 128-row tiles sharing a B tile): each loads
-// half of B and multicasts it to both, each MMA commit frees the ring slot
-// in both CTAs, and cluster barriers bracket start-up and teardown so no CTA
-// exits while its peer may still write into its shared memory.
+// The accumulator is double-buffered in TMEM so the epilogue of one tile
+// overlaps the MMAs of the next.
 //
-// With MMA_PAIR == 1 (CLUSTER == 2) the cluster runs one M=256 x N=BN pair MMA
-// per K step instead (tcgen05 cta_group::2): each CTA loads its 128 A rows
-// and its half of the B tile into its own ring, all of the pair's copies are
-// counted on the even CTA's ring barrier, the even CTA's warp 1 issues the
-// MMAs and its commits free the ring slot and publish the accumulator in both
-// CTAs, and each epilogue warp frees its accumulator buffer with one arrival
-// on the even CTA's barrier.  Each SM then streams 128 x 64 of A plus
-// BN/2 x 64 of B per K step instead of the whole B tile.
+// With MMA_PAIR == 1 (CLUSTER == 2) the two CTAs of a cluster run one
+// M=256 x N=BN pair MMA per K step (tcgen05 cta_group::2): each CTA loads its
+// 128 A rows and its half of the B tile into its own ring, all of the pair's
+// copies are counted on the even CTA's ring barrier, the even CTA's warp 1
+// issues the MMAs and its commits free the ring slot and publish the
+// accumulator in both CTAs, and each epilogue warp frees its accumulator
+// buffer with one arrival on the even CTA's barrier.  Each SM then streams
+// 128 x 64 of A plus BN/2 x 64 of B per K step.  Cluster barriers bracket
+// start-up and teardown so no CTA exits while its peer may still use it.
+//
+// Work split.  A cluster is a "slot"; the grid holds as many slots as can be
+// resident at once.  Tiles [0, dp_tiles) go round-robin to the slots whole.
+// The K blocks of the remaining tiles (stream-K) are cut into one contiguous
+// run per slot, so every slot gets the same number of K blocks however the
+// tile count divides.  A run splits into segments at tile boundaries:
+//   - a segment that starts at K block 0 belongs to the tile's owner, which
+//     runs the problem's epilogue once the tile is complete;
+//   - a segment that starts later (only a run's first segment can) is a
+//     contribution: its fp32 accumulator goes to the slot's region of the
+//     partial buffer and the slot publishes a flag.
+// The owner of a split tile waits (bounded) for the flags of the following
+// slots whose runs start inside the tile, adds their partials into its TMEM
+// accumulator, clears the flags and calls the epilogue as for a whole tile.
+// Contributions are made at the start of a run and consumed at the end of
+// another, so the owner rarely waits; every slot of the grid is resident.
+// The owner's segment ends its run, so by the time its accumulator is full
+// the ring is idle: each partial comes in with one bulk copy per epilogue
+// half.  Partials are stored per (slot, CTA, half) as 128 rows of the half's
+// columns with the 16-byte chunks of row r permuted by r % 8, so that the
+// owner's threads, one row each, read shared memory without bank conflicts.
+//
+// When every slot is busy these contractions are bound by L2 bandwidth (the
+// K-block rate per slot drops as slots are added), so splitting only pays
+// where a last wave would leave most slots idle; see stream_k_dp_tiles.
 //
 // Every wait is bounded (ptx.cuh); on a timeout the CTA unwinds, waits
 // briefly for its own copies and MMAs, frees TMEM and exits.
@@ -51,6 +72,7 @@
 //   epilogue_done(p, row, half): once, after the last tile.
 #pragma once
 
+#include "kernels.h"
 #include "ptx.cuh"
 
 namespace cer {
@@ -78,11 +100,67 @@ constexpr size_t gemm_smem_bytes() {
   return 1024 + static_cast<size_t>(P::STAGES) * (kATileBytes + b_stage_bytes<P>()) + P::kEpiSmemBytes + 256;
 }
 
-// Sleep about `ns` nanoseconds (bounded; used only while unwinding).
-__device__ __forceinline__ void unwind_pause(uint64_t ns) {
-  const uint64_t t0 = globaltimer_ns();
-  while (globaltimer_ns() - t0 < ns) __nanosleep(1000);
+// Stream-K split of a launch (see above).  partial == nullptr: every tile
+// whole, round-robin over the slots.
+struct StreamK {
+  float* partial;               // [slots][CLUSTER][128][BN] fp32, one contribution per slot
+  unsigned long long* flags;    // [slots][CLUSTER][EPI_WARPS / 4]; 0 or a launch token
+  unsigned long long token;     // non-zero value a contributor publishes
+  int dp_tiles;                 // tiles handed out whole
+};
+
+// First stream-K unit (K block) of slot s of S over U units.
+__host__ __device__ __forceinline__ long long sk_first_unit(long long U, int s, int S) {
+  return U * s / S;
 }
+
+// Tiles handed out whole when `tiles` tiles of `nkb` K blocks run on `slots`
+// slots.  `tiles` (no split) unless the tiles fill at least one wave and the
+// last wave would be at most half full, for contractions of at least 64 K
+// blocks (the partial sums cost about as much as a few K blocks); then the
+// last full wave and the remainder are split, every run covering at least one
+// tile, so a tile has at most two contributors.
+inline int stream_k_dp_tiles(int tiles, int nkb, int slots) {
+  if (slots <= 1 || nkb < 64) return tiles;
+  const int q = tiles / slots;
+  const int r = tiles % slots;
+  if (q == 0 || r == 0 || 2 * r > slots) return tiles;
+  return (q - 1) * slots;
+}
+
+// The segments a slot works through, in order: its whole tiles, then its
+// stream-K run cut at tile boundaries.  Producer, MMA issuer and epilogue
+// each walk their own copy.
+struct SegCursor {
+  int n_slots, nkb, dp_tiles, next_dp;
+  long long u, u_end;
+
+  __device__ SegCursor(int slot, int n_slots_, int ntiles, int nkb_, int dp_tiles_)
+      : n_slots(n_slots_), nkb(nkb_), dp_tiles(dp_tiles_), next_dp(slot) {
+    const long long U = static_cast<long long>(ntiles - dp_tiles_) * nkb_;
+    u = sk_first_unit(U, slot, n_slots_);
+    u_end = sk_first_unit(U, slot + 1, n_slots_);
+  }
+  __device__ bool next(int& tile, int& kb0, int& kb1) {
+    if (next_dp < dp_tiles) {
+      tile = next_dp;
+      kb0 = 0;
+      kb1 = nkb;
+      next_dp += n_slots;
+      return true;
+    }
+    if (u < u_end) {
+      const long long t = u / nkb;
+      tile = dp_tiles + static_cast<int>(t);
+      kb0 = static_cast<int>(u - t * nkb);
+      const long long end = u_end - t * nkb;
+      kb1 = end < nkb ? static_cast<int>(end) : nkb;
+      u += kb1 - kb0;
+      return true;
+    }
+    return false;
+  }
+};
 
 // A short, abort-independent wait used only while unwinding.
 __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
@@ -90,6 +168,12 @@ __device__ __forceinline__ void drain_wait(uint64_t* bar, uint32_t parity) {
   while (!mbar_try_wait(bar, parity)) {
     if (globaltimer_ns() - t0 > 100000000ull) return;
   }
+}
+
+// Sleep about `ns` nanoseconds (bounded; used only while unwinding).
+__device__ __forceinline__ void unwind_pause(uint64_t ns) {
+  const uint64_t t0 = globaltimer_ns();
+  while (globaltimer_ns() - t0 < ns) __nanosleep(1000);
 }
 
 // Lane 0 waits, the whole warp takes its verdict: keeps every branch after a
@@ -120,15 +204,34 @@ struct EpiCtx {
   }
 };
 
+// Wait until a stream-K flag holds `token` (bounded like every wait).
+__device__ __forceinline__ bool flag_wait(const unsigned long long* flag, unsigned long long token,
+                                          volatile int* abort_flag, int* status) {
+  if (ld_acquire_u64(flag) == token) return true;
+  const uint64_t t0 = globaltimer_ns();
+  while (true) {
+    if (ld_acquire_u64(flag) == token) return true;
+    if (*abort_flag) return false;
+    if (globaltimer_ns() - t0 > kWaitLimitNs) {
+      *abort_flag = 1;
+      record_status(status, CER_DEV_TIMEOUT);
+      return false;
+    }
+    __nanosleep(64);
+  }
+}
+
 template <class P>
-__global__ void __launch_bounds__(gemm_threads<P>(), 1) umma_gemm_kernel(const __grid_constant__ typename P::Params p) {
+__global__ void __launch_bounds__(gemm_threads<P>(), 1)
+    umma_gemm_kernel(const __grid_constant__ typename P::Params p, const __grid_constant__ StreamK sk) {
   static_assert(P::EPI_WARPS == 4 || P::EPI_WARPS == 8, "epilogue is one or two groups of four warps");
-  static_assert(P::CLUSTER == 1 || P::CLUSTER == 2, "clusters of one or two CTAs");
   constexpr bool PAIR = P::MMA_PAIR != 0;
-  static_assert(!PAIR || P::CLUSTER == 2, "a pair MMA runs on a 2-CTA cluster");
+  static_assert(P::CLUSTER == (PAIR ? 2 : 1), "a pair MMA runs on a 2-CTA cluster, anything else on one CTA");
   constexpr uint16_t kPairMask = 0x3;
   constexpr int BN = P::BN;
   constexpr int STAGES = P::STAGES;
+  constexpr int HALVES = P::EPI_WARPS / 4;
+  constexpr int HALF_COLS = BN / HALVES;
   constexpr uint32_t B_BYTES = b_stage_bytes<P>();
   constexpr uint32_t TMEM_COLS = TmemCols<BN>::value;
   constexpr uint32_t IDESC = idesc_bf16(PAIR ? 256 : 128, BN, P::B_MN_MAJOR);
@@ -144,20 +247,20 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1) umma_gemm_kernel(const _
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tempty + 2;
   uint64_t* half_bar = drain + 1;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(half_bar + 2);
+  uint64_t* sk_bar = half_bar + 2;   // the owner's partial copies, one per epilogue half
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sk_bar + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int rank = P::CLUSTER > 1 ? static_cast<int>(cluster_ctarank()) : 0;
-  const int cluster_id = blockIdx.x / P::CLUSTER;
-  const int n_clusters = gridDim.x / P::CLUSTER;
+  const int rank = PAIR ? static_cast<int>(cluster_ctarank()) : 0;
+  const int slot = blockIdx.x / P::CLUSTER;
+  const int n_slots = gridDim.x / P::CLUSTER;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full[s], 1);
-      // One MMA commit from each CTA of the cluster (from the even CTA alone with a pair MMA).
-      mbar_init(&empty[s], PAIR ? 1 : P::CLUSTER);
+      mbar_init(&empty[s], 1);   // one MMA commit (the even CTA's, with a pair MMA)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull[a], 1);
@@ -167,6 +270,8 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1) umma_gemm_kernel(const _
     mbar_init(drain, 1);
     mbar_init(&half_bar[0], 128);
     mbar_init(&half_bar[1], 128);
+    mbar_init(&sk_bar[0], 1);
+    mbar_init(&sk_bar[1], 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -180,8 +285,8 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1) umma_gemm_kernel(const _
     }
   }
   tc_fence_before();
-  if (P::CLUSTER > 1) {
-    cluster_sync();      // the peer's barriers exist before any multicast reaches them
+  if (PAIR) {
+    cluster_sync();      // the peer's barriers exist before any copy or commit reaches them
   } else {
     __syncthreads();
   }
@@ -192,19 +297,22 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1) umma_gemm_kernel(const _
 
   const int ntiles = P::num_tiles(p);
   const int nkb = P::num_kb(p);
+  const int dp_tiles = sk.partial != nullptr && sk.dp_tiles < ntiles ? sk.dp_tiles : ntiles;
 
   if (warp == 0) {
     // ---------------------------------------------------------------- producer
     typename P::ProdState st;
+    SegCursor cur(slot, n_slots, ntiles, nkb, dp_tiles);
     int stage = 0;
     uint32_t phase = 0;
     long issued = 0;
     bool ok = true;
     // With a pair MMA the even CTA's ring barriers count both CTAs' copies.
     const uint32_t leader_full = PAIR ? mapa_shared(smem_u32(full), 0) : 0u;
-    for (int tile = cluster_id; tile < ntiles && ok; tile += n_clusters) {
+    int tile, kb0, kb1;
+    while (ok && cur.next(tile, kb0, kb1)) {
       P::prod_tile(p, tile, rank, st);
-      for (int kb = 0; kb < nkb; ++kb) {
+      for (int kb = kb0; kb < kb1; ++kb) {
         if (!warp_wait(&empty[stage], phase ^ 1, abort_flag, p.status)) {
           ok = false;
           break;
@@ -239,20 +347,22 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1) umma_gemm_kernel(const _
     }
   } else if (warp == 1 && (!PAIR || rank == 0)) {
     // ---------------------------------------------------------------- MMA issuer
+    SegCursor cur(slot, n_slots, ntiles, nkb, dp_tiles);
     int stage = 0;
     uint32_t phase = 0;
     int acc = 0;
     uint32_t acc_phase = 0;
     bool ok = true;
     bool issued_any = false;
-    for (int tile = cluster_id; tile < ntiles && ok; tile += n_clusters) {
+    int tile, kb0, kb1;
+    while (ok && cur.next(tile, kb0, kb1)) {
       if (!warp_wait(&tempty[acc], acc_phase ^ 1, abort_flag, p.status)) {
         ok = false;
         break;
       }
       tc_fence_after();
       const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
-      for (int kb = 0; kb < nkb; ++kb) {
+      for (int kb = kb0; kb < kb1; ++kb) {
         if (!warp_wait(&full[stage], phase, abort_flag, p.status)) {
           ok = false;
           break;
@@ -265,15 +375,14 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1) umma_gemm_kernel(const _
           for (int k = 0; k < 4; ++k) {
             const uint64_t adesc = sdesc_kmajor_sw128(a_base + k * 32);
             const uint64_t bdesc = P::bdesc(b_base + k * P::kBStepBytes);
+            const uint32_t accumulate = ((kb - kb0) | k) != 0 ? 1u : 0u;
             if (PAIR)
-              umma_bf16_pair(d_tmem, adesc, bdesc, IDESC, (kb | k) != 0 ? 1u : 0u);
+              umma_bf16_pair(d_tmem, adesc, bdesc, IDESC, accumulate);
             else
-              umma_bf16(d_tmem, adesc, bdesc, IDESC, (kb | k) != 0 ? 1u : 0u);
+              umma_bf16(d_tmem, adesc, bdesc, IDESC, accumulate);
           }
           if (PAIR)
-            umma_commit_pair_multicast(&empty[stage], kPairMask);
-          else if (P::CLUSTER > 1)
-            umma_commit_multicast(&empty[stage], kPairMask);   // frees the slot in both CTAs
+            umma_commit_pair_multicast(&empty[stage], kPairMask);   // frees the slot in both CTAs
           else
             umma_commit(&empty[stage]);
           issued_any = true;
@@ -311,13 +420,81 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1) umma_gemm_kernel(const _
     const int half = (warp - 2) >> 2;  // which half of the accumulator columns
     EpiCtx ctx{epi_smem, rank, &half_bar[half], 0u, abort_flag, p.status};
     const uint32_t leader_tempty = PAIR ? mapa_shared(smem_u32(tempty), 0) : 0u;
+    const long long sk_units = static_cast<long long>(ntiles - dp_tiles) * nkb;
+    uint32_t sk_phase = 0;
+    SegCursor cur(slot, n_slots, ntiles, nkb, dp_tiles);
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int tile = cluster_id; tile < ntiles; tile += n_clusters) {
+    int tile, kb0, kb1;
+    while (cur.next(tile, kb0, kb1)) {
       if (!warp_wait(&tfull[acc], acc_phase, abort_flag, p.status)) break;
       tc_fence_after();
       const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(acc * BN);
-      const bool ok = P::epilogue(p, tile, row, half, taddr, ctx);
+      bool ok = true;
+      if (kb0 > 0) {
+        // A contribution: this half's columns of the row go to the slot's
+        // partial region (chunks permuted by row), then the half publishes
+        // its flag.
+        float4* dst = reinterpret_cast<float4*>(sk.partial) +
+                      (static_cast<size_t>((slot * P::CLUSTER + rank) * HALVES + half) * 128 + row) * (HALF_COLS / 4);
+#pragma unroll 1
+        for (int c = 0; c < HALF_COLS; c += 32) {
+          float v[32];
+          tmem_ld_32x32(taddr + half * HALF_COLS + c, v);
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            __stcg(dst + ((c / 4 + j) ^ (row & 7)), make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]));
+        }
+        __threadfence();
+        ok = ctx.sync();
+        if (ok && row == 0) st_release_u64(&sk.flags[(slot * P::CLUSTER + rank) * HALVES + half], sk.token);
+      } else {
+        if (kb1 < nkb) {
+          // The owner of a split tile: the runs of the following slots that
+          // start inside this tile hold the rest of its K blocks.  Each
+          // partial is copied into the (idle) ring, then added into TMEM.
+          const long long tile_end = static_cast<long long>(tile - dp_tiles + 1) * nkb;
+          constexpr uint32_t kHalfBytes = 128u * HALF_COLS * 4u;
+          static_assert(HALVES * kHalfBytes <= STAGES * (kATileBytes + B_BYTES), "partials fit in the ring");
+          static_assert(kHalfBytes % 16384 == 0, "copied in 16 KB pieces");
+          const float4* stage = reinterpret_cast<const float4*>(a_ring + half * kHalfBytes) + row * (HALF_COLS / 4);
+          for (int s2 = slot + 1; ok && s2 < n_slots && sk_first_unit(sk_units, s2, n_slots) < tile_end; ++s2) {
+            unsigned long long* flag = &sk.flags[(s2 * P::CLUSTER + rank) * HALVES + half];
+            if (row == 0) {
+              ok = flag_wait(flag, sk.token, abort_flag, p.status);
+              if (ok) {
+                fence_proxy_async_global();
+                const char* src = reinterpret_cast<const char*>(sk.partial) +
+                                  static_cast<size_t>((s2 * P::CLUSTER + rank) * HALVES + half) * kHalfBytes;
+                mbar_arrive_expect_tx(&sk_bar[half], kHalfBytes);
+                for (uint32_t off = 0; off < kHalfBytes; off += 16384)
+                  bulk_load(a_ring + half * kHalfBytes + off, src + off, 16384, &sk_bar[half]);
+              }
+            }
+            ok = ctx.sync() && !*abort_flag;
+            if (ok) ok = mbar_wait(&sk_bar[half], sk_phase, abort_flag, p.status);
+            sk_phase ^= 1;
+            if (!ok) break;
+#pragma unroll 1
+            for (int c = 0; c < HALF_COLS; c += 32) {
+              float v[32];
+              tmem_ld_32x32(taddr + half * HALF_COLS + c, v);
+#pragma unroll
+              for (int j = 0; j < 8; ++j) {
+                const float4 w = stage[(c / 4 + j) ^ (row & 7)];
+                v[4 * j] += w.x;
+                v[4 * j + 1] += w.y;
+                v[4 * j + 2] += w.z;
+                v[4 * j + 3] += w.w;
+              }
+              tmem_st_32x32(taddr + half * HALF_COLS + c, v);
+            }
+            ok = ctx.sync();   // the stage is read before the next copy overwrites it
+            if (ok && row == 0) st_relaxed_u64(flag, 0ull);
+          }
+        }
+        if (ok) ok = P::epilogue(p, tile, row, half, taddr, ctx);
+      }
       tc_fence_before();
       if (PAIR) {
         __syncwarp();
@@ -335,8 +512,8 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1) umma_gemm_kernel(const _
   }
 
   tc_fence_before();
-  if (P::CLUSTER > 1) {
-    cluster_sync();      // the peer no longer multicasts into this CTA
+  if (PAIR) {
+    cluster_sync();      // the peer no longer copies into, commits to or arrives on this CTA
   } else {
     __syncthreads();
   }

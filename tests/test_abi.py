@@ -52,8 +52,11 @@ def test_workspace_sizes(lib):
     assert lib.cer_score_workspace_size(1, 256, 64, 64, 1) == 2 * 512 + 4 * 256 * 4
     assert lib.cer_score_workspace_size(1, 10, 100, 0, 0) == 0          # hidden not a multiple of 64
     # FFN: act [M, C] bf16, plus three [C, d] slices when a channel list is packed per call
-    assert lib.cer_routed_ffn_workspace_size(2348, 1536, 6720, 0) == _r256(2348 * 6720 * 2)
-    assert lib.cer_routed_ffn_workspace_size(2348, 1536, 6720, 1) == _r256(2348 * 6720 * 2) + 3 * _r256(6720 * 1536 * 2)
+    sk = (24 << 20) + 8192     # stream-K partial accumulators and flags of the GEMMs
+    assert lib.cer_routed_ffn_workspace_size(2348, 1536, 6720, 0) == _r256(2348 * 6720 * 2) + sk
+    assert lib.cer_routed_ffn_workspace_size(2348, 1536, 6720, 1) == _r256(2348 * 6720 * 2) + sk + \
+        3 * _r256(6720 * 1536 * 2)
+    assert lib.cer_routed_ffn_workspace_size(0, 1536, 6720, 0) == 0
     M = 4 * (292 + 1024 - 729)
     for wc in (0, 1):
         ws = lib.cer_routed_block_workspace_size(4, 1024, 1536, 256, 0, 0, 0, 729, 292, 6720, wc)
