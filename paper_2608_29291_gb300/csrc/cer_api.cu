@@ -90,8 +90,8 @@ size_t ffn_stream_k_bytes(long long M) {
 }
 void carve_stream_k(char** ws, long long M, cer::FfnArgs* a) {
   if (M <= 0) return;
-  a->sk_partial = reinterpret_cast<float*>(*ws);
-  a->sk_flags = reinterpret_cast<unsigned long long*>(*ws + cer::kStreamKPartialBytes);
+  a->sk.partial = reinterpret_cast<float*>(*ws);
+  a->sk.flags = reinterpret_cast<unsigned long long*>(*ws + cer::kStreamKPartialBytes);
   *ws += ffn_stream_k_bytes(M);
 }
 

@@ -21,8 +21,6 @@
 //   distinct, so no atomics; dropped rows are never touched.
 #include <cuda_bf16.h>
 
-#include <atomic>
-
 #include "kernels.h"
 #include "umma_gemm.cuh"
 
@@ -88,6 +86,12 @@ struct GateUpProblemT {
     }
   }
   __device__ static uint64_t bdesc(uint32_t saddr) { return sdesc_kmajor_sw128(saddr); }
+  __device__ static void prefetch(const Params& p) {
+    tma_prefetch_desc(&p.tm_x);
+    tma_prefetch_desc(&p.tm_wg);
+    tma_prefetch_desc(&p.tm_wu);
+    tma_prefetch_desc(&p.tm_act);
+  }
 
   // Group `grp` (four warps, 128 threads, one accumulator row each) produces
   // the 64-channel boxes grp*2/kGroups .. of the tile's 128 channels.
@@ -228,6 +232,10 @@ struct DownProblem {
     }
   }
   __device__ static uint64_t bdesc(uint32_t saddr) { return sdesc_mnmajor_sw128(saddr, kAtomBytes, 1024); }
+  __device__ static void prefetch(const Params& p) {
+    tma_prefetch_desc(&p.tm_act);
+    tma_prefetch_desc(&p.tm_wdt);
+  }
 
   __device__ static void epilogue_done(const Params&, int, int) {}
   __device__ static bool epilogue(const Params& p, int tile, int row, int half, uint32_t taddr, EpiCtx& ctx) {
@@ -282,74 +290,6 @@ struct DownProblem {
 
 // ---------------------------------------------------------------- launchers
 
-// A launch's stream-K token: never 0, and hashed (SplitMix64 finaliser) so
-// that whatever a fresh workspace holds is not taken for a published flag.
-static unsigned long long next_stream_k_token() {
-  static std::atomic<unsigned long long> counter{0};
-  unsigned long long z = counter.fetch_add(1) + 0x9E3779B97F4A7C15ull;
-  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
-  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
-  z ^= z >> 31;
-  return z | 1ull;
-}
-
-// `tiles` counts cluster tiles of `nkb` K blocks (the fewest the kernel may
-// take, for a contraction length decided on the device).  The persistent
-// grid holds as many slots (clusters) as can be resident at once; with a
-// stream-K workspace in `a`, the tiles that do not fill whole waves are split
-// by K block over all of them.
-template <class P>
-static cudaError_t launch_gemm(const typename P::Params& p, int tiles, int nkb, const FfnArgs* a, int n_sm,
-                               cudaStream_t stream) {
-  if (tiles == 0) return cudaSuccess;
-  const size_t smem = gemm_smem_bytes<P>();
-  cudaError_t e = ensure_max_smem(reinterpret_cast<const void*>(umma_gemm_kernel<P>), smem);
-  if (e != cudaSuccess) return e;
-  int slots = n_sm;
-  if (P::CLUSTER > 1) {
-    // Clusters must fit inside GPC boundaries: ask how many can be resident.
-    static int resident[64] = {0};
-    int dev = 0;
-    cudaGetDevice(&dev);
-    int& max_clusters = resident[dev & 63];
-    if (max_clusters == 0) {
-      cudaLaunchConfig_t cfg = {};
-      cfg.gridDim = dim3(n_sm / P::CLUSTER * P::CLUSTER, 1, 1);
-      cfg.blockDim = dim3(gemm_threads<P>(), 1, 1);
-      cfg.dynamicSmemBytes = smem;
-      cfg.stream = stream;
-      cudaLaunchAttribute attr[1];
-      attr[0].id = cudaLaunchAttributeClusterDimension;
-      attr[0].val.clusterDim.x = P::CLUSTER;
-      attr[0].val.clusterDim.y = 1;
-      attr[0].val.clusterDim.z = 1;
-      cfg.attrs = attr;
-      cfg.numAttrs = 1;
-      int n = 0;
-      e = cudaOccupancyMaxActiveClusters(&n, umma_gemm_kernel<P>, &cfg);
-      if (e != cudaSuccess) return e;
-      max_clusters = n > 0 ? n : 1;
-    }
-    slots = max_clusters;
-  }
-  StreamK sk{};
-  int n_slots = tiles < slots ? tiles : slots;
-  if (a != nullptr && a->sk_partial != nullptr && a->sk_flags != nullptr && nkb > 0) {
-    const int dp = stream_k_dp_tiles(tiles, nkb, slots);
-    const size_t partial = static_cast<size_t>(slots) * P::CLUSTER * 128 * P::BN * sizeof(float);
-    const size_t flags = static_cast<size_t>(slots) * P::CLUSTER * (P::EPI_WARPS / 4) * sizeof(unsigned long long);
-    if (dp < tiles && partial <= kStreamKPartialBytes && flags <= kStreamKFlagBytes) {
-      sk.partial = a->sk_partial;
-      sk.flags = a->sk_flags;
-      sk.token = next_stream_k_token();
-      sk.dp_tiles = dp;
-      n_slots = slots;
-    }
-  }
-  return launch_k(umma_gemm_kernel<P>, dim3(n_slots * P::CLUSTER), dim3(gemm_threads<P>()), smem, stream, P::CLUSTER,
-                  p, sk);
-}
-
 cudaError_t launch_ffn_gateup(const FfnArgs& a, int n_sm, cudaStream_t stream) {
   GateUpProblem::Params p{};
   if (!encode_bf16_2d(&p.tm_x, a.X, a.M, a.d, 64, 128)) return cudaErrorInvalidValue;
@@ -364,7 +304,7 @@ cudaError_t launch_ffn_gateup(const FfnArgs& a, int n_sm, cudaStream_t stream) {
   p.n_mt = (a.M + 127) / 128;
   p.n_mtp = (p.n_mt + 1) / 2;
   p.n_ct = (a.C + 127) / 128;
-  return launch_gemm<GateUpProblem>(p, p.n_mtp * p.n_ct, a.d / 64, &a, n_sm, stream);
+  return launch_gemm<GateUpProblem>(p, p.n_mtp * p.n_ct, a.d / 64, &a.sk, n_sm, stream);
 }
 
 template <int BN, int PAIR>
@@ -389,7 +329,7 @@ static cudaError_t launch_down(const FfnArgs& a, int n_sm, cudaStream_t stream) 
   p.n_mtp = (p.n_mt + 1) / 2;
   p.n_nt = (a.d + BN - 1) / BN;
   const int nkb = (a.use_small_k != nullptr ? a.C_small : a.C) / 64;
-  return launch_gemm<P>(p, (PAIR ? p.n_mtp : p.n_mt) * p.n_nt, nkb, &a, n_sm, stream);
+  return launch_gemm<P>(p, (PAIR ? p.n_mtp : p.n_mt) * p.n_nt, nkb, &a.sk, n_sm, stream);
 }
 
 // Tile shape of the down GEMM.  With at least two row tiles: 256-row pair

@@ -52,6 +52,19 @@ cer_status internal_fail(cer_status status, const char* fmt, ...);
 // launch) once per device.
 cudaError_t ensure_max_smem(const void* func, size_t bytes);
 
+// Bytes of the GEMMs' stream-K partial buffer and of its flags (a launch uses
+// at most this much; see umma_gemm.cuh).
+constexpr size_t kStreamKPartialBytes = size_t(24) << 20;
+constexpr size_t kStreamKFlagBytes = 8192;
+
+// A stream-K region of a workspace (both NULL: tiles are never split).  The
+// kernels that use it run one after another on a stream and leave every flag
+// cleared, so one region serves the scorer and both FFN GEMMs of a block.
+struct StreamKArea {
+  float* partial;               // kStreamKPartialBytes
+  unsigned long long* flags;    // kStreamKFlagBytes
+};
+
 // ------------------------------------------------------------------ S1 score
 struct ScoreArgs {
   const __nv_bfloat16* h;
@@ -115,11 +128,6 @@ cudaError_t launch_scatter_add(__nv_bfloat16* h, int B, int N, int d, const int3
                                const __nv_bfloat16* Y, int* status, int n_sm, cudaStream_t stream);
 
 // ------------------------------------------------------------------ S4 FFN
-// Bytes of the GEMMs' stream-K partial buffer and of its flags (a launch uses
-// at most this much; see umma_gemm.cuh).
-constexpr size_t kStreamKPartialBytes = size_t(24) << 20;
-constexpr size_t kStreamKFlagBytes = 8192;
-
 struct FfnArgs {
   const __nv_bfloat16* X;     // packed kept rows [M, d]
   int M, d, C;
@@ -140,10 +148,7 @@ struct FfnArgs {
   float* colsum;
   const uint8_t* use_small_k;
   int C_small;
-  // Stream-K workspace (optional): kStreamKPartialBytes of fp32 partial
-  // accumulators and kStreamKFlagBytes of flags, shared by both GEMMs.
-  float* sk_partial;
-  unsigned long long* sk_flags;
+  StreamKArea sk;   // optional
   int* status;
 };
 cudaError_t launch_ffn_gateup(const FfnArgs& a, int n_sm, cudaStream_t stream);

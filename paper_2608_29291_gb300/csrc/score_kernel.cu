@@ -118,11 +118,11 @@ __device__ __forceinline__ float gelu_as(float x) {
 template <int BN_>
 struct ScoreProblem {
   static constexpr int BN = BN_;
+  static constexpr int MMA_PAIR = 0;
+  static constexpr int CLUSTER = 1;
   static constexpr int STAGES = BN == 256 ? 4 : BN == 128 ? 6 : 8;
   static constexpr int B_MN_MAJOR = 0;
   static constexpr int EPI_WARPS = 8;
-  static constexpr int CLUSTER = 1;
-  static constexpr int MMA_PAIR = 0;
   static constexpr uint32_t kBStepBytes = 32;
   static constexpr uint32_t kEpiSmemBytes = 0;
 
@@ -152,7 +152,7 @@ struct ScoreProblem {
     rt = rest % p.n_rt;
     b = rest / p.n_rt;
   }
-  __device__ static void prod_tile(const Params& p, int tile, int lane, ProdState& st) {
+  __device__ static void prod_tile(const Params& p, int tile, int, ProdState& st) {
     decode(p, tile, st.b, st.rt, st.chunk);
     if (st.chunk < p.n_core) {
       st.wrow = st.chunk * BN;
@@ -168,13 +168,15 @@ struct ScoreProblem {
                                  uint8_t* b, uint64_t* bar) {
     if (lane == 0) {
       tma_load_2d(a, &p.tm_h, bar, kb * 64, st.b * p.N + st.rt * 128);
-      if (st.chunk < p.n_core)
-        tma_load_2d(b, &p.tm_w1, bar, kb * 64, st.wrow);
-      else
-        tma_load_2d(b, &p.tm_w1e, bar, kb * 64, st.wrow);
+      tma_load_2d(b, st.chunk < p.n_core ? &p.tm_w1 : &p.tm_w1e, bar, kb * 64, st.wrow);
     }
   }
   __device__ static uint64_t bdesc(uint32_t saddr) { return sdesc_kmajor_sw128(saddr); }
+  __device__ static void prefetch(const Params& p) {
+    tma_prefetch_desc(&p.tm_h);
+    tma_prefetch_desc(&p.tm_w1);
+    tma_prefetch_desc(&p.tm_w1e);
+  }
 
   __device__ static void epilogue_done(const Params&, int, int) {}
   __device__ static bool epilogue(const Params& p, int tile, int row, int half, uint32_t taddr, EpiCtx&) {
@@ -278,29 +280,26 @@ static cudaError_t launch_score_gemm(const ScoreArgs& a, const float* bias_tab, 
   p.n_rt = (a.N + 127) / 128;
   p.n_core = a.Hc / BN;
   p.n_chunks = Ht / BN;
-  const int tiles = a.B * p.n_rt * p.n_chunks;
-  if (tiles == 0) return cudaSuccess;
-  const size_t smem = gemm_smem_bytes<P>();
-  cudaError_t e = ensure_max_smem(reinterpret_cast<const void*>(umma_gemm_kernel<P>), smem);
-  if (e != cudaSuccess) return e;
-  const int grid = tiles < n_sm ? tiles : n_sm;
-  return launch_k(umma_gemm_kernel<P>, dim3(grid), dim3(gemm_threads<P>()), smem, stream, 1, p, StreamK{});
+  return launch_gemm<P>(p, a.B * p.n_rt * p.n_chunks, a.d / 64, nullptr, n_sm, stream);
+}
+
+// Understanding reads b1 and w2 directly (bias/w2 tables NULL); generation
+// first builds the per-sequence tables.
+static cudaError_t launch_score_chunks(const ScoreArgs& a, const float* bias_tab, const float* w2_tab,
+                                       float* partial, int n_sm, cudaStream_t stream, int* n_partials) {
+  const int bn = pick_chunk_width(a, n_sm);
+  *n_partials = bn ? 2 * (a.Hc + (a.gen ? a.He : 0)) / bn : 0;
+  switch (bn) {
+    case 256: return launch_score_gemm<256>(a, bias_tab, w2_tab, partial, n_sm, stream);
+    case 128: return launch_score_gemm<128>(a, bias_tab, w2_tab, partial, n_sm, stream);
+    case 64: return launch_score_gemm<64>(a, bias_tab, w2_tab, partial, n_sm, stream);
+    default: return cudaErrorInvalidValue;
+  }
 }
 
 cudaError_t launch_score(const ScoreArgs& a, const ScoreWorkspace& ws, int n_sm, cudaStream_t stream,
                          int* n_partials) {
-  const int bn = pick_chunk_width(a, n_sm);
-  *n_partials = bn ? 2 * (a.Hc + (a.gen ? a.He : 0)) / bn : 0;
-  if (!a.gen) {
-    // Understanding: one core scorer for every sequence, no time input; the
-    // epilogue reads b1 and w2 directly and no bias table is built.
-    switch (bn) {
-      case 256: return launch_score_gemm<256>(a, nullptr, nullptr, ws.partial, n_sm, stream);
-      case 128: return launch_score_gemm<128>(a, nullptr, nullptr, ws.partial, n_sm, stream);
-      case 64: return launch_score_gemm<64>(a, nullptr, nullptr, ws.partial, n_sm, stream);
-      default: return cudaErrorInvalidValue;
-    }
-  }
+  if (!a.gen) return launch_score_chunks(a, nullptr, nullptr, ws.partial, n_sm, stream, n_partials);
   const int emb_bytes = a.U ? a.E * static_cast<int>(sizeof(float)) : 0;
   const int Ht = a.Hc + a.He;
   EmbFreqTable ft;
@@ -311,12 +310,7 @@ cudaError_t launch_score(const ScoreArgs& a, const ScoreWorkspace& ws, int n_sm,
   cudaError_t e = launch_k(time_bias_kernel, bias_grid, dim3(32 * kBiasColsPerBlock), emb_bytes, stream, 1, a, ft,
                            ws.bias_tab, ws.w2_tab);
   if (e != cudaSuccess) return e;
-  switch (bn) {
-    case 256: return launch_score_gemm<256>(a, ws.bias_tab, ws.w2_tab, ws.partial, n_sm, stream);
-    case 128: return launch_score_gemm<128>(a, ws.bias_tab, ws.w2_tab, ws.partial, n_sm, stream);
-    case 64: return launch_score_gemm<64>(a, ws.bias_tab, ws.w2_tab, ws.partial, n_sm, stream);
-    default: return cudaErrorInvalidValue;
-  }
+  return launch_score_chunks(a, ws.bias_tab, ws.w2_tab, ws.partial, n_sm, stream, n_partials);
 }
 
 cudaError_t launch_score_reduce(const float* partial, int n_chunks, size_t total, float* logits, float* probs,

@@ -61,7 +61,7 @@
 //   prod_kb(p, state, tile, kb, lane, a_smem, b_smem, bar) (with MMA_PAIR,
 //   `bar` is the cluster address of the even CTA's ring barrier),
 //   stage_bytes(p, tile, kb) (with MMA_PAIR, the bytes of both CTAs),
-//   bdesc(saddr),
+//   bdesc(saddr), prefetch(p) (prefetches the tensor maps' descriptors),
 //   kEpiSmemBytes (shared memory reserved for the epilogue, may be 0),
 //   epilogue(p, tile, row, half, taddr, ctx) -> false to abort (ctx.rank is
 //   the CTA's rank in its cluster): columns
@@ -71,6 +71,8 @@
 //   bounded barrier over the 128 threads of the half;
 //   epilogue_done(p, row, half): once, after the last tile.
 #pragma once
+
+#include <atomic>
 
 #include "kernels.h"
 #include "ptx.cuh"
@@ -114,18 +116,28 @@ __host__ __device__ __forceinline__ long long sk_first_unit(long long U, int s, 
   return U * s / S;
 }
 
-// Tiles handed out whole when `tiles` tiles of `nkb` K blocks run on `slots`
-// slots.  `tiles` (no split) unless the tiles fill at least one wave and the
-// last wave would be at most half full, for contractions of at least 64 K
-// blocks (the partial sums cost about as much as a few K blocks); then the
-// last full wave and the remainder are split, every run covering at least one
-// tile, so a tile has at most two contributors.
-inline int stream_k_dp_tiles(int tiles, int nkb, int slots) {
-  if (slots <= 1 || nkb < 64) return tiles;
+// Host side: how a launch splits its tiles.  A split pays only where a last
+// wave would leave most slots idle: with every slot busy these contractions
+// are bound by L2 bandwidth (the K-block rate per slot drops as slots are
+// added), so a split elsewhere only adds partial traffic.  It applies when
+// the tiles fill at least one wave, the last wave is at most half full and
+// the contraction has at least 64 K blocks (the partial sums cost about as
+// much as a few K blocks): the last full wave and the remainder are split,
+// every run covering at least one tile (at most two contributors per tile).
+// (Splitting the scorer's short contractions was measured slower: the
+// owners' GELU epilogues then run on a quarter of the SMs.)
+struct SplitPlan {
+  int slots;      // clusters to launch
+  int dp_tiles;   // tiles handed out whole (== tiles: no split)
+};
+
+inline SplitPlan stream_k_plan(int tiles, int nkb, int slots) {
+  const SplitPlan whole{tiles < slots ? tiles : slots, tiles};
+  if (slots <= 1 || nkb < 64) return whole;
   const int q = tiles / slots;
   const int r = tiles % slots;
-  if (q == 0 || r == 0 || 2 * r > slots) return tiles;
-  return (q - 1) * slots;
+  if (q == 0 || r == 0 || 2 * r > slots) return whole;
+  return SplitPlan{slots, (q - 1) * slots};
 }
 
 // The segments a slot works through, in order: its whole tiles, then its
@@ -257,6 +269,7 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1)
   const int slot = blockIdx.x / P::CLUSTER;
   const int n_slots = gridDim.x / P::CLUSTER;
 
+  if (threadIdx.x == 32) P::prefetch(p);   // tensor-map descriptors, ahead of the first copy
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full[s], 1);
@@ -524,6 +537,75 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1)
     else
       tmem_dealloc(tmem_base, TMEM_COLS);
   }
+}
+
+// ---------------------------------------------------------------- host side
+
+// A launch's stream-K token: never 0, and hashed (SplitMix64 finaliser) so
+// that whatever a fresh workspace holds is not taken for a published flag.
+inline unsigned long long next_stream_k_token() {
+  static std::atomic<unsigned long long> counter{0};
+  unsigned long long z = counter.fetch_add(1) + 0x9E3779B97F4A7C15ull;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  z ^= z >> 31;
+  return z | 1ull;
+}
+
+// Launches umma_gemm_kernel<P> over `tiles` cluster tiles of `nkb` K blocks
+// (the fewest the kernel may take, for a contraction length decided on the
+// device).  The persistent grid holds at most as many slots (clusters) as can
+// be resident at once; with a stream-K region the tiles may be split.
+template <class P>
+cudaError_t launch_gemm(const typename P::Params& p, int tiles, int nkb, const StreamKArea* area, int n_sm,
+                        cudaStream_t stream) {
+  if (tiles == 0) return cudaSuccess;
+  const size_t smem = gemm_smem_bytes<P>();
+  cudaError_t e = ensure_max_smem(reinterpret_cast<const void*>(umma_gemm_kernel<P>), smem);
+  if (e != cudaSuccess) return e;
+  int slots = n_sm;
+  if (P::CLUSTER > 1) {
+    // Clusters must fit inside GPC boundaries: ask how many can be resident.
+    static int resident[64] = {0};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    int& max_clusters = resident[dev & 63];
+    if (max_clusters == 0) {
+      cudaLaunchConfig_t cfg = {};
+      cfg.gridDim = dim3(n_sm / P::CLUSTER * P::CLUSTER, 1, 1);
+      cfg.blockDim = dim3(gemm_threads<P>(), 1, 1);
+      cfg.dynamicSmemBytes = smem;
+      cfg.stream = stream;
+      cudaLaunchAttribute attr[1];
+      attr[0].id = cudaLaunchAttributeClusterDimension;
+      attr[0].val.clusterDim.x = P::CLUSTER;
+      attr[0].val.clusterDim.y = 1;
+      attr[0].val.clusterDim.z = 1;
+      cfg.attrs = attr;
+      cfg.numAttrs = 1;
+      int n = 0;
+      e = cudaOccupancyMaxActiveClusters(&n, umma_gemm_kernel<P>, &cfg);
+      if (e != cudaSuccess) return e;
+      max_clusters = n > 0 ? n : 1;
+    }
+    slots = max_clusters;
+  }
+  StreamK sk{};
+  SplitPlan plan{tiles < slots ? tiles : slots, tiles};
+  if (area != nullptr && area->partial != nullptr && area->flags != nullptr) {
+    const SplitPlan split = stream_k_plan(tiles, nkb, slots);
+    const size_t partial = static_cast<size_t>(split.slots) * P::CLUSTER * 128 * P::BN * sizeof(float);
+    const size_t flags = static_cast<size_t>(split.slots) * P::CLUSTER * (P::EPI_WARPS / 4) * sizeof(unsigned long long);
+    if (split.dp_tiles < tiles && partial <= kStreamKPartialBytes && flags <= kStreamKFlagBytes) {
+      plan = split;
+      sk.partial = area->partial;
+      sk.flags = area->flags;
+      sk.token = next_stream_k_token();
+      sk.dp_tiles = split.dp_tiles;
+    }
+  }
+  return launch_k(umma_gemm_kernel<P>, dim3(plan.slots * P::CLUSTER), dim3(gemm_threads<P>()), smem, stream,
+                  P::CLUSTER, p, sk);
 }
 
 }  // namespace cer

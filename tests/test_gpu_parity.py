@@ -285,6 +285,9 @@ def _small(name):
         "segments": dict(n_segments=4, B=4, N=130, r0=0, r1=130, K=65),
         "one_token": dict(B=1, N=1, r0=0, r1=1, K=1),
         "d3584": dict(B=1, N=200, d=3584, I=2048, C=1024, r0=0, r1=200, K=60),
+        # 256-wide scorers (whole 256-column hidden chunks) with ragged row tiles.
+        "wide_scorer_gen": dict(B=3, N=700, d=1024, Hc=256, He=256, r0=50, r1=700, K=200),
+        "wide_scorer_und": dict(task=0, He=0, E=0, Hc=256, B=2, N=1000, d=512, r0=0, r1=900, K=300),
     }
     kw = dict(base)
     kw.update(variants[name])
@@ -292,7 +295,7 @@ def _small(name):
 
 
 @pytest.mark.parametrize("name", ["ragged_gen", "und_text_tail", "k0", "dense_all_kept", "segments", "one_token",
-                                  "d3584"])
+                                  "d3584", "wide_scorer_gen", "wide_scorer_und"])
 @pytest.mark.parametrize("prepacked", [True, False], ids=["packed", "chan"])
 def test_routed_block_small(name, prepacked):
     w = _small(name)
