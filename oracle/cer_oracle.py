@@ -52,6 +52,20 @@ UCS statistics (Sec. 3.4, Unified Computation Scheduling):
   retained set R is every kept token; a zero-norm pair has cosine 1 when the
   vectors are equal, else 0; empty R gives g = 0.
 
+Attention on the packed sequence (Sec. 3.4: the retained tokens are packed
+into a shorter sequence for attention and FFN; for understanding the packed
+keys and values form a compressed KV cache):
+  * rope: rotary position embedding of the Qwen2.5 backbone (App. A.5),
+    rotate-half pairing (j, j + dh/2), theta_j = base^(-2j/dh);
+  * packed_attention: softmax(Q K^T / sqrt(dh)) V per head over one packed
+    sequence, query head h reading key/value head h // (Hq / Hkv).
+  Readings: a packed token keeps its original position (its index in the
+  full sequence) for the rotary embedding; the keep list is ascending, so a
+  causal mask by original position is the causal mask on the packed order;
+  understanding (LLM prefill) is causal, generation attends bidirectionally
+  among the packed tokens (a flag); a query with no admissible key is not
+  possible (every token attends to itself).
+
 Parity status: every function below is pinned by tests/test_oracle_pins.py
 (hand-computed example, brute-force top-k, closed forms, library special cases,
 invariants).  Agreement with what the paper's authors ran is unpinned: the paper
@@ -315,3 +329,49 @@ def ffn_leakage(saliency: np.ndarray, pruned) -> float:
     mask proposes to remove."""
     total = float(np.sum(saliency))
     return float(np.sum(saliency[np.asarray(pruned, dtype=np.int64)])) / total if total > 0 else 0.0
+
+
+# ---------------------------------------------------------------- attention on the packed sequence
+
+def rope_frequencies(dh: int, base: float) -> np.ndarray:
+    """theta_j = base^(-2j/dh), j < dh/2: the rotary frequencies of the Qwen2.5
+    backbone (App. A.5)."""
+    j = np.arange(dh // 2, dtype=np.float64)
+    return float(base) ** (-2.0 * j / dh)
+
+
+def rope(x: np.ndarray, pos: np.ndarray, base: float) -> np.ndarray:
+    """Rotary embedding of x [T, heads, dh] (fp64) at positions pos [T], in the
+    rotate-half pairing: for j < dh/2, with a = p theta_j,
+    x'[j] = x[j] cos a - x[j + dh/2] sin a,  x'[j + dh/2] = x[j + dh/2] cos a + x[j] sin a.
+    Packed tokens keep their original positions (Sec. 3.4 compaction; reading)."""
+    T, H, dh = x.shape
+    ang = np.outer(np.asarray(pos, dtype=np.float64), rope_frequencies(dh, base))
+    c = np.cos(ang)[:, None, :]
+    s = np.sin(ang)[:, None, :]
+    lo, hi = x[..., : dh // 2], x[..., dh // 2:]
+    return np.concatenate([lo * c - hi * s, hi * c + lo * s], axis=-1)
+
+
+def packed_attention(Q: np.ndarray, K: np.ndarray, V: np.ndarray, causal: bool, scale: float | None = None):
+    """Softmax attention over one packed sequence (Sec. 3.4: attention runs on
+    the retained tokens only).  Q [L, Hq, dh], K and V [L, Hkv, dh] in fp64;
+    query head h uses key/value head h // (Hq // Hkv).  causal: packed token i
+    attends to packed tokens j <= i (the packed order is the original order).
+    Returns O [L, Hq, dh]."""
+    L, Hq, dh = Q.shape
+    Hkv = K.shape[1]
+    group = Hq // Hkv
+    if scale is None:
+        scale = 1.0 / math.sqrt(dh)
+    O = np.empty((L, Hq, dh), dtype=np.float64)
+    allowed = np.tril(np.ones((L, L), dtype=bool)) if causal else np.ones((L, L), dtype=bool)
+    for h in range(Hq):
+        kh = h // group
+        S = (Q[:, h, :] @ K[:, kh, :].T) * scale
+        S = np.where(allowed, S, -np.inf)
+        S = S - S.max(axis=1, keepdims=True)
+        P = np.exp(S)
+        P = P / P.sum(axis=1, keepdims=True)
+        O[:, h, :] = P @ V[:, kh, :]
+    return O

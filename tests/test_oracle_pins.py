@@ -552,3 +552,141 @@ def test_zero_leakage_means_pruned_ffn_equals_full_ffn():
     W2 = WdT.copy()
     W2[0] = gen.f32_to_bf16_bits(ora.bf16_to_f64(WdT[0]).astype(np.float32) * 2)
     assert abs(ora.ffn_saliency(X, Wg, Wu, W2)[0] - 2 * sal[0]) < 1e-12 * max(1, sal[0])
+
+
+# ------------------------------------------------------------------ attention on the packed sequence (Sec. 3.4)
+
+def _rope_checks():
+    f = []
+    # dh = 4: the rotate-half pairs are (0, 2) and (1, 3); theta_0 = 1, theta_1 = base^(-1/2).
+    x = np.zeros((1, 1, 4))
+    x[0, 0, 0] = 1.0
+    y = ora.rope(x, np.array([1]), 1e6)
+    if not np.allclose(y[0, 0], [math.cos(1), 0, math.sin(1), 0], atol=1e-15):
+        f.append(f"rope pair (0, 2): {y[0, 0]}")
+    x = np.zeros((1, 1, 4))
+    x[0, 0, 1] = 1.0
+    y = ora.rope(x, np.array([2]), 100.0)          # theta_1 = 0.1, angle 0.2
+    if not np.allclose(y[0, 0], [0, math.cos(0.2), 0, math.sin(0.2)], atol=1e-15):
+        f.append(f"rope pair (1, 3): {y[0, 0]}")
+    rng = np.random.default_rng(3)
+    z = rng.normal(size=(5, 3, 16))
+    if not np.array_equal(ora.rope(z, np.zeros(5), 1e6), z):
+        f.append("rope at position 0 is not the identity")
+    r = ora.rope(z, np.array([0, 7, 300, 4095, 16383]), 1e6)
+    n_in = np.hypot(z[..., :8], z[..., 8:])
+    n_out = np.hypot(r[..., :8], r[..., 8:])
+    if not np.allclose(n_in, n_out, rtol=1e-13):
+        f.append("rope changes the norm of a rotated pair")
+    # Relative position: <rope(q, p + s), rope(k, p' + s)> does not depend on s.
+    q, k = rng.normal(size=(1, 1, 128)), rng.normal(size=(1, 1, 128))
+    dots = [float(np.sum(ora.rope(q, [10 + s], 1e6) * ora.rope(k, [3 + s], 1e6))) for s in (0, 1, 977, 12000)]
+    if max(dots) - min(dots) > 1e-9 * max(1.0, abs(dots[0])):
+        f.append(f"rope dot products depend on the absolute position: {dots}")
+    return f
+
+
+def _attention_checks():
+    f = []
+    e = math.e
+    Q = np.array([[[1.0, 0.0]], [[0.0, 1.0]]])     # L = 2, one head, dh = 2
+    V = np.array([[[1.0, 2.0]], [[3.0, 4.0]]])
+    O = ora.packed_attention(Q, Q.copy(), V, causal=False, scale=1.0)
+    want = np.array([[(e + 3) / (e + 1), (2 * e + 4) / (e + 1)], [(1 + 3 * e) / (e + 1), (2 + 4 * e) / (e + 1)]])
+    if not np.allclose(O[:, 0], want, atol=1e-15):
+        f.append(f"attention hand example (full): {O[:, 0]}")
+    Oc = ora.packed_attention(Q, Q.copy(), V, causal=True, scale=1.0)
+    if not (np.array_equal(Oc[0, 0], [1.0, 2.0]) and np.allclose(Oc[1, 0], want[1], atol=1e-15)):
+        f.append(f"attention hand example (causal): {Oc[:, 0]}")
+    # Equal scores (Q = 0): prefix means of V (causal), the mean of V (full);
+    # query head h reads key/value head h // 2 (4 query heads, 2 kv heads).
+    rng = np.random.default_rng(4)
+    V = rng.normal(size=(6, 2, 8))
+    K = rng.normal(size=(6, 2, 8))
+    Q0 = np.zeros((6, 4, 8))
+    Oc = ora.packed_attention(Q0, K, V, causal=True)
+    Of = ora.packed_attention(Q0, K, V, causal=False)
+    for i in range(6):
+        for h in range(4):
+            if not np.allclose(Oc[i, h], V[: i + 1, h // 2].mean(axis=0), atol=1e-14):
+                f.append(f"causal equal-score row {i} head {h}")
+            if not np.allclose(Of[i, h], V[:, h // 2].mean(axis=0), atol=1e-14):
+                f.append(f"full equal-score row {i} head {h}")
+    O1 = ora.packed_attention(rng.normal(size=(1, 3, 8)), K[:1, :1], V[:1, :1], causal=True)
+    if not np.allclose(O1, np.repeat(V[:1, :1], 3, axis=1), atol=1e-15):
+        f.append("a single key does not return its value")
+    # Independent library routine: torch's scaled_dot_product_attention in fp64.
+    L, Hq, Hkv, dh = 37, 6, 2, 16
+    Q, K, V = rng.normal(size=(L, Hq, dh)), rng.normal(size=(L, Hkv, dh)), rng.normal(size=(L, Hkv, dh))
+    for causal in (False, True):
+        q = torch.tensor(Q).permute(1, 0, 2)[None]
+        k = torch.tensor(K).permute(1, 0, 2).repeat_interleave(Hq // Hkv, dim=0)[None]
+        v = torch.tensor(V).permute(1, 0, 2).repeat_interleave(Hq // Hkv, dim=0)[None]
+        ref = F.scaled_dot_product_attention(q, k, v, is_causal=causal)[0].permute(1, 0, 2).numpy()
+        got = ora.packed_attention(Q, K, V, causal=causal)
+        if not np.allclose(got, ref, atol=1e-12):
+            f.append(f"attention differs from torch sdpa (causal={causal}): {np.abs(got - ref).max()}")
+    return f
+
+
+def test_rope_pins():
+    assert _rope_checks() == []
+
+
+def test_attention_pins():
+    assert _attention_checks() == []
+
+
+def _attention_strict_causal(orig):
+    def f(Q, K, V, causal, scale=None):
+        if not causal:
+            return orig(Q, K, V, causal, scale)
+        L, Hq, dh = Q.shape
+        sc = 1.0 / math.sqrt(dh) if scale is None else scale
+        O = np.zeros_like(Q)
+        for h in range(Hq):
+            kh = h // (Hq // K.shape[1])
+            S = Q[:, h] @ K[:, kh].T * sc
+            S = np.where(np.tril(np.ones((L, L), bool), -1), S, -1e300)   # j < i instead of j <= i
+            P = np.exp(S - S.max(axis=1, keepdims=True))
+            O[:, h] = (P / P.sum(axis=1, keepdims=True)) @ V[:, kh]
+        return O
+    return f
+
+
+def _attention_gqa_modulo(orig):
+    def f(Q, K, V, causal, scale=None):
+        Hq, Hkv = Q.shape[1], K.shape[1]
+        perm = [h % Hkv for h in range(Hq)]          # h % Hkv instead of h // (Hq / Hkv)
+        Kx, Vx = K[:, perm], V[:, perm]
+        return orig(Q, Kx, Vx, causal, scale)
+    return f
+
+
+def _rope_adjacent_pairs(orig):
+    def f(x, pos, base):
+        T, H, dh = x.shape
+        ang = np.outer(np.asarray(pos, np.float64), ora.rope_frequencies(dh, base))
+        c, s = np.cos(ang)[:, None, :], np.sin(ang)[:, None, :]
+        ev, od = x[..., 0::2], x[..., 1::2]
+        y = np.empty_like(x)
+        y[..., 0::2] = ev * c - od * s
+        y[..., 1::2] = od * c + ev * s
+        return y
+    return f
+
+
+ATTENTION_MUTATIONS = {
+    "causal_excludes_self": ("packed_attention", _attention_strict_causal),
+    "gqa_modulo_heads": ("packed_attention", _attention_gqa_modulo),
+    "no_score_scale": ("packed_attention", lambda orig: (lambda Q, K, V, causal, scale=None: orig(Q, K, V, causal, 1.0))),
+    "rope_adjacent_pairs": ("rope", _rope_adjacent_pairs),
+    "rope_sign": ("rope", lambda orig: (lambda x, pos, base: orig(x, -np.asarray(pos, np.float64), base))),
+}
+
+
+@pytest.mark.parametrize("name", sorted(ATTENTION_MUTATIONS))
+def test_attention_pins_catch_planted_mistake(name, monkeypatch):
+    attr, make = ATTENTION_MUTATIONS[name]
+    monkeypatch.setattr(ora, attr, make(getattr(ora, attr)))
+    assert _rope_checks() + _attention_checks(), f"planted mistake {name} went unnoticed"
