@@ -292,6 +292,43 @@ cer_status cer_redundancy_gap(const void* h_in, const void* h_out, const uint8_t
                               void* workspace, size_t workspace_bytes, cudaStream_t stream);
 size_t cer_redundancy_gap_workspace_size(int B, int N);
 
+/* ------------------------------------------------------------------ attention on the packed sequence
+ * Sec. 3.4: the retained tokens are packed into a shorter sequence for
+ * attention and FFN; for understanding, the packed keys and values form the
+ * compressed key-value cache that decoding reuses.  Backbone (App. A.5):
+ * Qwen2.5, head size 128, grouped key/value heads, rotary embedding.
+ *
+ * Packed rows: qkv bf16 [B * L, (Hq + 2 Hkv) * 128] (device, 16-byte
+ * aligned): per row the token's Hq query heads, then Hkv key heads, then Hkv
+ * value heads, 128 values each; L = the packed length of every sequence (the
+ * k_tot of cer_select_topk).  Requires Hq >= 1, Hkv >= 1, Hq % Hkv == 0.
+ *
+ * cer_rope_packed: rotary position embedding of the query and key heads, in
+ * place, each packed row at its original position (a packed token keeps its
+ * index in the full sequence).
+ *   pos   int32 [B * L] device: the rows' original positions, e.g. the keep
+ *         list of cer_select_topk; a negative position is reported as
+ *         CER_ERR_INDEX by cer_sync_status and that row is left unrotated
+ *   base  rotary base (1e6 for Qwen2.5): for j < 64 the pair (j, j + 64) of a
+ *         head is rotated by pos * base^(-2j/128) (rotate-half pairing)
+ * Angles are formed in fp64 turns and reduced exactly before an fp32 sine
+ * and cosine; rotated values are rounded to bf16.
+ *
+ * cer_packed_attention: softmax attention over each packed sequence,
+ *   out[b, i, h] = sum_j softmax_j(q_{b,i,h} . k_{b,j,g} / sqrt(128)) v_{b,j,g},
+ *   g = h / (Hq / Hkv), over the packed tokens j of sequence b (j <= i when
+ *   causal: the keep list is ascending, so this is the causal mask by
+ *   original position).
+ *   qkv   as above (rotated); not modified
+ *   out   bf16 [B * L, Hq * 128] device
+ * Q K^T accumulates in fp32 on the tensor cores; the softmax weights are
+ * rounded to bf16 for their product with V (fp32 accumulation); out is the
+ * normalised fp32 result rounded to bf16.                                    */
+cer_status cer_rope_packed(void* qkv, int B, int L, int Hq, int Hkv, const int32_t* pos, double base,
+                           cudaStream_t stream);
+cer_status cer_packed_attention(const void* qkv, int B, int L, int Hq, int Hkv, int causal, void* out,
+                                cudaStream_t stream);
+
 /* ------------------------------------------------------------------ status
  * cer_sync_status: synchronise `stream`, then return and clear the current
  * device's status word (the first kernel-detected error since the last call),

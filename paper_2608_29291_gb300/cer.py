@@ -31,8 +31,8 @@ EXPORTS = ("cer_score", "cer_score_workspace_size", "cer_score_static", "cer_sel
            "cer_routed_block_workspace_size", "cer_ffn_channel_norms", "cer_routed_ffn_gated",
            "cer_routed_ffn_gated_workspace_size", "cer_routed_block_gated", "cer_routed_block_gated_workspace_size",
            "cer_drop_set_stats", "cer_redundancy_gap",
-           "cer_redundancy_gap_workspace_size", "cer_sync_status", "cer_get_error", "cer_status_string",
-           "cer_version")
+           "cer_redundancy_gap_workspace_size", "cer_rope_packed", "cer_packed_attention", "cer_sync_status",
+           "cer_get_error", "cer_status_string", "cer_version")
 
 
 class CerError(RuntimeError):
@@ -73,6 +73,8 @@ _SIGS = {
     "cer_drop_set_stats": ([_vp, _vp, _i, _i, _i, _i, _vp, _vp, _vp, _vp, _vp], _i),
     "cer_redundancy_gap": ([_vp, _vp, _vp, _i, _i, _i, _f, _vp, _vp, _vp, _sz, _vp], _i),
     "cer_redundancy_gap_workspace_size": ([_i, _i], _sz),
+    "cer_rope_packed": ([_vp, _i, _i, _i, _i, _vp, ctypes.c_double, _vp], _i),
+    "cer_packed_attention": ([_vp, _i, _i, _i, _i, _i, _vp, _vp], _i),
     "cer_sync_status": ([_vp], _i),
     "cer_get_error": ([], ctypes.c_char_p),
     "cer_status_string": ([_i], ctypes.c_char_p),
@@ -294,6 +296,20 @@ def cer_redundancy_gap(h_in, h_out, mask, delta, gap, skip=None, ws=None, stream
         ws = workspace(load().cer_redundancy_gap_workspace_size(B, N), h_in.device)
     _check(load().cer_redundancy_gap(_p(h_in), _p(h_out), _p(mask), B, N, d, float(delta), _p(gap), _p(skip),
                                      _p(ws), ws.numel(), _stream(stream)))
+
+
+def cer_rope_packed(qkv, B, L, Hq, Hkv, pos, base=1e6, stream=None):
+    """Rotary embedding of the packed query and key heads in place (qkv bf16 [B*L, (Hq+2Hkv)*128])."""
+    _check(load().cer_rope_packed(_p(qkv), B, L, Hq, Hkv, _p(pos), float(base), _stream(stream)))
+
+
+def cer_packed_attention(qkv, B, L, Hq, Hkv, causal, out=None, stream=None):
+    """Softmax attention over each packed sequence; returns out bf16 [B*L, Hq*128]."""
+    import torch
+    if out is None:
+        out = torch.empty((B * L, Hq * 128), dtype=torch.bfloat16, device=qkv.device)
+    _check(load().cer_packed_attention(_p(qkv), B, L, Hq, Hkv, int(causal), _p(out), _stream(stream)))
+    return out
 
 
 def cer_sync_status(stream=None) -> None:

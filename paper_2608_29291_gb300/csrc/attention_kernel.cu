@@ -1,0 +1,442 @@
+// attention_kernel.cu -- attention on the packed sequence (Sec. 3.4: the
+// retained tokens are packed into a shorter sequence for attention and FFN;
+// for understanding the packed keys and values are the compressed KV cache),
+// with the rotary position embedding of the Qwen2.5 backbone (App. A.5).
+//
+// Packed rows are laid out as one bf16 matrix qkv [B * L, (Hq + 2 Hkv) * 128]:
+// per row Hq query heads, Hkv key heads, Hkv value heads of 128 values.  A
+// packed token keeps its original position (its index in the full sequence)
+// for the rotary embedding, and the keep list is ascending, so masking by
+// original position is the causal mask on the packed order.
+//
+// rope_kernel: one block per packed row rotates its query and key heads in
+// place (rotate-half pairing (j, j + 64)).
+//
+// packed_attention_kernel: persistent, one CTA per SM, one work item per
+// (query tile of 128 packed tokens, sequence, query head), the tiles with the
+// most key blocks first.  192 threads:
+//   warp 0     TMA: the Q tile once per item (two 64-column boxes, K-major)
+//              and, per key block of 128 tokens, K (K-major) and V (four
+//              64 x 64 MN-major atoms) into a two-slot ring;
+//   warp 1     allocates TMEM (two S buffers of 128 columns, O of 128) and
+//              issues tcgen05.mma: S_j = Q K_j^T into S[j % 2] -- issued one
+//              block ahead, so it overlaps the softmax of block j - 1 -- and
+//              O += P_j V_j once the softmax has written P_j;
+//   warps 2-5  softmax, one query row per thread (its TMEM lane): masked row
+//              maximum in the log2 domain, O rescaled in TMEM only when a
+//              row maximum of the warp moved, P_j = exp2(s - m) written as
+//              bf16 into a 128-byte-swizzled tile (the A operand of P V), the
+//              running sum kept in fp32; at the end O / l goes out as bf16.
+// Every wait is bounded like the GEMM skeleton's (umma_gemm.cuh).
+#include <cuda_bf16.h>
+
+#include "kernels.h"
+#include "umma_gemm.cuh"
+
+namespace cer {
+
+// ------------------------------------------------------------------ rotary embedding
+
+constexpr int kRopeThreads = 128;
+
+// angle a = pos * theta_j is formed in turns, x = pos * g_j with g_j =
+// theta_j / (2 pi) from the host's fp64 table, reduced exactly in fp64
+// (x - rint(x)) and handed to fp32 sincospif: accurate to ~2e-7 for any
+// position, where an fp32 product pos * theta_j would lose the angle.
+__global__ void __launch_bounds__(kRopeThreads)
+    rope_kernel(__nv_bfloat16* qkv, long long rows, int Hq, int Hkv, const int32_t* __restrict__ pos,
+                const __grid_constant__ RopeFreqTable ft, int* status) {
+  griddep_wait();
+  griddep_launch_dependents();
+  __shared__ float cs[kHeadDim / 2], sn[kHeadDim / 2];
+  const int width = (Hq + 2 * Hkv) * kHeadDim;
+  const int pairs = (Hq + Hkv) * (kHeadDim / 2);
+  for (long long row = blockIdx.x; row < rows; row += gridDim.x) {
+    const int p = __ldg(pos + row);
+    __syncthreads();   // the previous row's table is no longer read
+    if (threadIdx.x < kHeadDim / 2) {
+      const double x = static_cast<double>(p) * ft.g[threadIdx.x];
+      const float r = static_cast<float>(x - rint(x));
+      float s, c;
+      sincospif(2.0f * r, &s, &c);
+      cs[threadIdx.x] = c;
+      sn[threadIdx.x] = s;
+    }
+    __syncthreads();
+    if (p < 0) {
+      if (threadIdx.x == 0) record_status(status, CER_DEV_INDEX);
+      continue;
+    }
+    __nv_bfloat16* r = qkv + row * width;
+    for (int t = threadIdx.x; t < pairs; t += blockDim.x) {
+      __nv_bfloat16* hp = r + (t >> 6) * kHeadDim;
+      const int j = t & 63;
+      const float lo = __bfloat162float(hp[j]), hi = __bfloat162float(hp[j + 64]);
+      const float c = cs[j], s = sn[j];
+      hp[j] = __float2bfloat16_rn(fmaf(lo, c, -hi * s));
+      hp[j + 64] = __float2bfloat16_rn(fmaf(hi, c, lo * s));
+    }
+  }
+}
+
+cudaError_t launch_rope(__nv_bfloat16* qkv, long long rows, int Hq, int Hkv, const int32_t* pos,
+                        const RopeFreqTable& ft, int* status, int n_sm, cudaStream_t stream) {
+  if (rows == 0) return cudaSuccess;
+  const long long cap = static_cast<long long>(n_sm) * 16;
+  const unsigned grid = static_cast<unsigned>(rows < cap ? rows : cap);
+  return launch_k(rope_kernel, dim3(grid), dim3(kRopeThreads), 0, stream, 1, qkv, rows, Hq, Hkv, pos, ft, status);
+}
+
+// ------------------------------------------------------------------ attention
+
+struct AttnParams {
+  CUtensorMap tm_qk;   // qkv, box 64 x 128 (Q and K tiles)
+  CUtensorMap tm_v;    // qkv, box 64 x 64 (V atoms)
+  __nv_bfloat16* out;  // [B * L, Hq * 128]
+  int* status;
+  int B, L, Hq, Hkv, causal, n_qt, n_items;
+  float scale_log2;    // log2(e) / sqrt(128)
+};
+
+constexpr int kAttnThreads = 192;
+constexpr uint32_t kBox = 128 * 128;              // 128 rows x 64 bf16
+constexpr uint32_t kQBytes = 2 * kBox;            // Q tile: 128 tokens x 128
+constexpr uint32_t kKVBytes = 4 * kBox;           // K tile (2 boxes) + V (4 atoms of 8 KB)
+constexpr uint32_t kPBytes = 2 * kBox;            // P tile: 128 queries x 128 keys, bf16
+constexpr size_t kAttnSmem = 1024 + kQBytes + 2 * kKVBytes + kPBytes + 256;
+constexpr uint32_t kIdescS = idesc_bf16(128, 128, 0);    // Q (K-major) x K (K-major)
+constexpr uint32_t kIdescPV = idesc_bf16(128, 128, 1);   // P (K-major) x V (MN-major)
+
+struct AttnItem {
+  int b, h, kh, qt, n_kv;
+};
+
+__device__ __forceinline__ AttnItem attn_item(const AttnParams& p, int item) {
+  AttnItem it;
+  const int per_tile = p.B * p.Hq;
+  it.qt = p.n_qt - 1 - item / per_tile;   // the tiles with the most key blocks first
+  const int rest = item % per_tile;
+  it.b = rest / p.Hq;
+  it.h = rest % p.Hq;
+  it.kh = it.h / (p.Hq / p.Hkv);
+  it.n_kv = p.causal ? it.qt + 1 : p.n_qt;
+  return it;
+}
+
+__global__ void __launch_bounds__(kAttnThreads, 1) packed_attention_kernel(const __grid_constant__ AttnParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* q_tile = smem;
+  uint8_t* kv_ring = q_tile + kQBytes;          // slot s: K at +0 (2 boxes), V at +2*kBox (4 atoms)
+  uint8_t* p_tile = kv_ring + 2 * kKVBytes;
+  uint64_t* q_full = reinterpret_cast<uint64_t*>(p_tile + kPBytes);
+  uint64_t* q_empty = q_full + 1;
+  uint64_t* kv_full = q_empty + 1;     // [2]
+  uint64_t* kv_empty = kv_full + 2;    // [2]
+  uint64_t* s_full = kv_empty + 2;     // [2]
+  uint64_t* s_free = s_full + 2;       // [2]
+  uint64_t* p_full = s_free + 2;
+  uint64_t* o_done = p_full + 1;
+  uint64_t* o_free = o_done + 1;
+  uint64_t* drain = o_free + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  if (threadIdx.x == 32) {
+    tma_prefetch_desc(&p.tm_qk);
+    tma_prefetch_desc(&p.tm_v);
+  }
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    mbar_init(q_empty, 1);
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&kv_full[s], 1);
+      mbar_init(&kv_empty[s], 1);
+      mbar_init(&s_full[s], 1);
+      mbar_init(&s_free[s], 4);   // one arrival per softmax warp
+    }
+    mbar_init(p_full, 4);
+    mbar_init(o_done, 1);
+    mbar_init(o_free, 4);
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  griddep_wait();   // qkv written by the previous kernel is visible
+  griddep_launch_dependents();
+
+  if (warp == 0) {
+    // ---------------------------------------------------------------- producer
+    uint32_t g = 0;          // key blocks loaded so far (ring slot g % 2)
+    uint32_t items = 0;
+    bool ok = true;
+    for (int item = blockIdx.x; item < p.n_items && ok; item += gridDim.x, ++items) {
+      const AttnItem it = attn_item(p, item);
+      const int row0 = it.b * p.L;
+      if (!warp_wait(q_empty, (items & 1) ^ 1, abort_flag, p.status)) {
+        ok = false;
+        break;
+      }
+      if (lane == 0) {
+        mbar_arrive_expect_tx(q_full, kQBytes);
+        tma_load_2d(q_tile, &p.tm_qk, q_full, it.h * kHeadDim, row0 + it.qt * 128);
+        tma_load_2d(q_tile + kBox, &p.tm_qk, q_full, it.h * kHeadDim + 64, row0 + it.qt * 128);
+      }
+      __syncwarp();
+      for (int j = 0; j < it.n_kv; ++j, ++g) {
+        const int s = g & 1;
+        if (!warp_wait(&kv_empty[s], ((g >> 1) & 1) ^ 1, abort_flag, p.status)) {
+          ok = false;
+          break;
+        }
+        if (lane == 0) {
+          uint8_t* slot = kv_ring + s * kKVBytes;
+          const int kcol = (p.Hq + it.kh) * kHeadDim;
+          const int vcol = (p.Hq + p.Hkv + it.kh) * kHeadDim;
+          const int kv0 = row0 + j * 128;
+          mbar_arrive_expect_tx(&kv_full[s], kKVBytes);
+          tma_load_2d(slot, &p.tm_qk, &kv_full[s], kcol, kv0);
+          tma_load_2d(slot + kBox, &p.tm_qk, &kv_full[s], kcol + 64, kv0);
+          for (int kh = 0; kh < 2; ++kh)
+            for (int na = 0; na < 2; ++na)
+              tma_load_2d(slot + 2 * kBox + kh * 16384 + na * 8192, &p.tm_v, &kv_full[s], vcol + na * 64,
+                          kv0 + kh * 64);
+        }
+        __syncwarp();
+      }
+    }
+    if (!ok && lane == 0) unwind_pause(1000000ull);
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA issuer
+    uint32_t g = 0;          // key blocks consumed (ring slot g % 2)
+    uint32_t cs = 0;         // S tiles issued (buffer cs % 2)
+    uint32_t cp = 0;         // P tiles consumed
+    uint32_t items = 0;
+    bool ok = true;
+    bool issued_any = false;
+    const uint32_t q_base = smem_u32(q_tile), p_base = smem_u32(p_tile);
+    const uint32_t o_tm = tmem_base + 256;
+    for (int item = blockIdx.x; item < p.n_items && ok; item += gridDim.x, ++items) {
+      const AttnItem it = attn_item(p, item);
+      if (!warp_wait(q_full, items & 1, abort_flag, p.status)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      for (int j = -1; j < it.n_kv && ok; ++j) {
+        // Issue S_{j+1} (one block ahead of the P V product of block j).
+        if (j + 1 < it.n_kv) {
+          const uint32_t gs = g + static_cast<uint32_t>(j + 1);
+          const uint32_t slot = gs & 1;
+          const uint32_t buf = cs & 1;
+          if (!warp_wait(&kv_full[slot], (gs >> 1) & 1, abort_flag, p.status) ||
+              !warp_wait(&s_free[buf], ((cs >> 1) & 1) ^ 1, abort_flag, p.status)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          if (lane == 0) {
+            const uint32_t k_base = smem_u32(kv_ring + slot * kKVBytes);
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+              const uint32_t off = (k >> 2) * kBox + (k & 3) * 32;
+              umma_bf16(tmem_base + buf * 128, sdesc_kmajor_sw128(q_base + off), sdesc_kmajor_sw128(k_base + off),
+                        kIdescS, k > 0 ? 1u : 0u);
+            }
+            umma_commit(&s_full[buf]);
+            if (j + 2 == it.n_kv) umma_commit(q_empty);   // the item's last S: the Q tile may be reloaded
+            issued_any = true;
+          }
+          __syncwarp();
+          ++cs;
+        }
+        if (j < 0) continue;
+        // O += P_j V_j once the softmax has written P_j (and, for the item's
+        // first block, has read out the previous item's O).
+        if (!warp_wait(p_full, cp & 1, abort_flag, p.status)) {
+          ok = false;
+          break;
+        }
+        ++cp;
+        if (j == 0 && !warp_wait(o_free, (items & 1) ^ 1, abort_flag, p.status)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t slot = (g + static_cast<uint32_t>(j)) & 1;
+        if (lane == 0) {
+          const uint32_t v_base = smem_u32(kv_ring + slot * kKVBytes + 2 * kBox);
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            const uint64_t adesc = sdesc_kmajor_sw128(p_base + (k >> 2) * kBox + (k & 3) * 32);
+            const uint64_t bdesc = sdesc_mnmajor_sw128(v_base + (k >> 2) * 16384 + (k & 3) * 2048, 8192, 1024);
+            umma_bf16(o_tm, adesc, bdesc, kIdescPV, (j > 0 || k > 0) ? 1u : 0u);
+          }
+          umma_commit(&kv_empty[slot]);
+          umma_commit(o_done);
+        }
+        __syncwarp();
+      }
+      g += static_cast<uint32_t>(it.n_kv);
+    }
+    if (!ok && lane == 0 && issued_any) {
+      umma_commit(drain);
+      drain_wait(drain, 0);
+    }
+  } else {
+    // ---------------------------------------------------------------- softmax
+    const int qd = warp & 3;            // TMEM lane quadrant
+    const int r = qd * 32 + lane;       // query row of the tile
+    const uint32_t lane_off = static_cast<uint32_t>(qd * 32) << 16;
+    const uint32_t o_tm = tmem_base + lane_off + 256;
+    uint32_t cs = 0, co = 0, items = 0;
+    bool ok = true;
+    for (int item = blockIdx.x; item < p.n_items && ok; item += gridDim.x, ++items) {
+      const AttnItem it = attn_item(p, item);
+      const int qi = it.qt * 128 + r;
+      float m = -INFINITY, l = 0.f;
+      for (int j = 0; j < it.n_kv; ++j, ++cs) {
+        const uint32_t buf = cs & 1;
+        if (!warp_wait(&s_full[buf], (cs >> 1) & 1, abort_flag, p.status)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t s_tm = tmem_base + lane_off + buf * 128;
+        const int kv0 = j * 128;
+        // Keys past the sequence, and (causal) past the query, are masked.
+        const int lim = p.causal ? (qi + 1 < p.L ? qi + 1 : p.L) : p.L;
+        float mx = -INFINITY;
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          float v[32];
+          tmem_ld_32x32(s_tm + c * 32, v);
+#pragma unroll
+          for (int e = 0; e < 32; ++e)
+            if (kv0 + c * 32 + e < lim) mx = fmaxf(mx, v[e] * p.scale_log2);
+        }
+        const float m_new = fmaxf(m, mx);
+        const float alpha = exp2f(m - m_new);   // 0 for the first block
+        if (j > 0) {
+          // P_{j-1} V_{j-1} is complete: the P tile is free and O may be rescaled.
+          if (!warp_wait(o_done, co & 1, abort_flag, p.status)) {
+            ok = false;
+            break;
+          }
+          ++co;
+          tc_fence_after();
+          if (__any_sync(0xffffffffu, alpha != 1.0f)) {
+#pragma unroll 1
+            for (int c = 0; c < 4; ++c) {
+              float v[32];
+              tmem_ld_32x32(o_tm + c * 32, v);
+#pragma unroll
+              for (int e = 0; e < 32; ++e) v[e] *= alpha;
+              tmem_st_32x32(o_tm + c * 32, v);
+            }
+          }
+        }
+        float rs = 0.f;
+#pragma unroll 1
+        for (int c = 0; c < 4; ++c) {
+          float v[32];
+          tmem_ld_32x32(s_tm + c * 32, v);
+          uint32_t pk[16];
+#pragma unroll
+          for (int e = 0; e < 16; ++e) {
+            const int k0 = kv0 + c * 32 + 2 * e;
+            const float p0 = k0 < lim ? exp2f(fmaf(v[2 * e], p.scale_log2, -m_new)) : 0.f;
+            const float p1 = k0 + 1 < lim ? exp2f(fmaf(v[2 * e + 1], p.scale_log2, -m_new)) : 0.f;
+            rs += p0 + p1;
+            pk[e] = pack_bf16x2(p0, p1);
+          }
+          uint8_t* row_base = p_tile + (c >> 1) * kBox + r * 128;
+#pragma unroll
+          for (int vv = 0; vv < 4; ++vv) {
+            const int chunk = ((c & 1) * 4 + vv) ^ (r & 7);   // 128-byte swizzle
+            *reinterpret_cast<uint4*>(row_base + chunk * 16) =
+                make_uint4(pk[4 * vv], pk[4 * vv + 1], pk[4 * vv + 2], pk[4 * vv + 3]);
+          }
+        }
+        tc_fence_before();
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+          mbar_arrive(&s_free[buf]);
+          mbar_arrive(p_full);
+        }
+        l = l * alpha + rs;
+        m = m_new;
+      }
+      if (!ok) break;
+      if (!warp_wait(o_done, co & 1, abort_flag, p.status)) {
+        ok = false;
+        break;
+      }
+      ++co;
+      tc_fence_after();
+      const float inv = 1.0f / l;
+      __nv_bfloat16* dst = p.out + (static_cast<size_t>(it.b) * p.L + qi) * (static_cast<size_t>(p.Hq) * kHeadDim) +
+                           static_cast<size_t>(it.h) * kHeadDim;
+#pragma unroll 1
+      for (int c = 0; c < 4; ++c) {
+        float v[32];
+        tmem_ld_32x32(o_tm + c * 32, v);
+        if (qi < p.L) {
+          uint32_t pk[16];
+#pragma unroll
+          for (int e = 0; e < 16; ++e) pk[e] = pack_bf16x2(v[2 * e] * inv, v[2 * e + 1] * inv);
+          uint4* d4 = reinterpret_cast<uint4*>(dst + c * 32);
+#pragma unroll
+          for (int q = 0; q < 4; ++q) d4[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(o_free);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, 512);
+  }
+}
+
+cudaError_t launch_packed_attention(const __nv_bfloat16* qkv, int B, int L, int Hq, int Hkv, int causal,
+                                    __nv_bfloat16* out, int* status, int n_sm, cudaStream_t stream) {
+  if (B == 0 || L == 0) return cudaSuccess;
+  AttnParams p{};
+  const uint64_t rows = static_cast<uint64_t>(B) * L;
+  const uint64_t width = static_cast<uint64_t>(Hq + 2 * Hkv) * kHeadDim;
+  if (!encode_bf16_2d(&p.tm_qk, qkv, rows, width, 64, 128)) return cudaErrorInvalidValue;
+  if (!encode_bf16_2d(&p.tm_v, qkv, rows, width, 64, 64)) return cudaErrorInvalidValue;
+  p.out = out;
+  p.status = status;
+  p.B = B;
+  p.L = L;
+  p.Hq = Hq;
+  p.Hkv = Hkv;
+  p.causal = causal;
+  p.n_qt = (L + 127) / 128;
+  p.n_items = B * Hq * p.n_qt;
+  p.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kHeadDim));
+  cudaError_t e = ensure_max_smem(reinterpret_cast<const void*>(packed_attention_kernel), kAttnSmem);
+  if (e != cudaSuccess) return e;
+  const int grid = p.n_items < n_sm ? p.n_items : n_sm;
+  return launch_k(packed_attention_kernel, dim3(grid), dim3(kAttnThreads), kAttnSmem, stream, 1, p);
+}
+
+}  // namespace cer

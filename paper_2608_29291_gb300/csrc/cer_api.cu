@@ -5,6 +5,7 @@
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 
+#include <cmath>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
@@ -876,6 +877,60 @@ cer_status cer_redundancy_gap(const void* h_in, const void* h_out, const uint8_t
                                              static_cast<const __nv_bfloat16*>(h_out), mask, B, N, d, delta, gap,
                                              skip, static_cast<float*>(workspace), dev->n_sm, stream);
   if (e != cudaSuccess) return cuda_fail(e, "redundancy-gap launch");
+  return CER_OK;
+}
+
+namespace {
+
+cer_status check_qkv(int B, int L, int Hq, int Hkv) {
+  CER_REQUIRE(B >= 0 && L >= 0, CER_ERR_SHAPE, "B=%d L=%d must be >= 0", B, L);
+  CER_REQUIRE(Hq >= 1 && Hkv >= 1 && Hq % Hkv == 0 && Hq + 2 * Hkv <= 1024, CER_ERR_SHAPE,
+              "Hq=%d, Hkv=%d: need Hq, Hkv >= 1, Hq a multiple of Hkv, Hq + 2 Hkv <= 1024", Hq, Hkv);
+  CER_REQUIRE(static_cast<long long>(B) * L < (1LL << 31), CER_ERR_SHAPE, "B*L=%lld rows exceed 2^31",
+              static_cast<long long>(B) * L);
+  return CER_OK;
+}
+
+}  // namespace
+
+cer_status cer_rope_packed(void* qkv, int B, int L, int Hq, int Hkv, const int32_t* pos, double base,
+                           cudaStream_t stream) {
+  const bool any = static_cast<long long>(B) * L > 0;
+  CER_PTR_IF(qkv, any);
+  CER_PTR_IF(pos, any);
+  CER_ALIGN(qkv);
+  CER_ALIGN(pos);
+  cer_status s = check_qkv(B, L, Hq, Hkv);
+  if (s != CER_OK) return s;
+  CER_REQUIRE(base > 1.0 && std::isfinite(base), CER_ERR_RANGE, "rotary base %g must be finite and > 1", base);
+  DeviceInfo* dev = nullptr;
+  if ((s = device_info(&dev)) != CER_OK) return s;
+  if (!any) return CER_OK;
+  cer::RopeFreqTable ft;
+  for (int j = 0; j < cer::kHeadDim / 2; ++j)
+    ft.g[j] = std::pow(base, -2.0 * j / cer::kHeadDim) / (2.0 * M_PI);
+  cudaError_t e = cer::launch_rope(static_cast<__nv_bfloat16*>(qkv), static_cast<long long>(B) * L, Hq, Hkv, pos,
+                                   ft, dev->status, dev->n_sm, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "rotary embedding launch");
+  return CER_OK;
+}
+
+cer_status cer_packed_attention(const void* qkv, int B, int L, int Hq, int Hkv, int causal, void* out,
+                                cudaStream_t stream) {
+  const bool any = static_cast<long long>(B) * L > 0;
+  CER_PTR_IF(qkv, any);
+  CER_PTR_IF(out, any);
+  CER_ALIGN(qkv);
+  CER_ALIGN(out);
+  cer_status s = check_qkv(B, L, Hq, Hkv);
+  if (s != CER_OK) return s;
+  CER_REQUIRE(causal == 0 || causal == 1, CER_ERR_RANGE, "causal=%d must be 0 or 1", causal);
+  DeviceInfo* dev = nullptr;
+  if ((s = device_info(&dev)) != CER_OK) return s;
+  if (!any) return CER_OK;
+  cudaError_t e = cer::launch_packed_attention(static_cast<const __nv_bfloat16*>(qkv), B, L, Hq, Hkv, causal,
+                                               static_cast<__nv_bfloat16*>(out), dev->status, dev->n_sm, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "packed attention launch");
   return CER_OK;
 }
 

@@ -170,4 +170,25 @@ cudaError_t launch_redundancy_gap(const __nv_bfloat16* h_in, const __nv_bfloat16
                                   int B, int N, int d, float delta, float* gap, uint8_t* skip, float* cos_ws,
                                   int n_sm, cudaStream_t stream);
 
+// ------------------------------------------------------------------ attention on the packed sequence
+// qkv: bf16 [B * L, (Hq + 2 Hkv) * 128]; each row holds the token's Hq query
+// heads, then Hkv key heads, then Hkv value heads (head size 128).
+constexpr int kHeadDim = 128;
+
+// Frequencies of the rotary embedding divided by 2*pi, in fp64:
+// g[j] = base^(-2j/128) / (2*pi), j < 64 (computed on the host).
+struct RopeFreqTable {
+  double g[kHeadDim / 2];
+};
+
+// Rotates the query and key heads of every packed row in place at the row's
+// original position pos[row] (the keep list, [B * L]).
+cudaError_t launch_rope(__nv_bfloat16* qkv, long long rows, int Hq, int Hkv, const int32_t* pos,
+                        const RopeFreqTable& ft, int* status, int n_sm, cudaStream_t stream);
+
+// out [B * L, Hq * 128] = softmax(Q K^T / sqrt(128)) V per sequence and query
+// head over the packed tokens (causal: key index <= query index).
+cudaError_t launch_packed_attention(const __nv_bfloat16* qkv, int B, int L, int Hq, int Hkv, int causal,
+                                    __nv_bfloat16* out, int* status, int n_sm, cudaStream_t stream);
+
 }  // namespace cer

@@ -110,6 +110,20 @@ def test_score_argument_checks(lib):
     assert s(FAKE, 1, 16, 1536, ctypes.pointer(core), None, None, 0, FAKE, None, FAKE, 8, None) == 9        # workspace
 
 
+def test_attention_argument_checks(lib):
+    r, a = lib.cer_rope_packed, lib.cer_packed_attention
+    assert r(FAKE, 1, 8, 3, 2, FAKE, 1e6, None) == 2        # Hq not a multiple of Hkv
+    assert r(FAKE, 1, 8, 4, 0, FAKE, 1e6, None) == 2        # no key/value head
+    assert r(FAKE, 1, 8, 4, 2, None, 1e6, None) == 1        # NULL positions
+    assert r(FAKE, 1, 8, 4, 2, FAKE, 0.5, None) == 4        # rotary base <= 1
+    assert r(FAKE, 1, 8, 4, 2, FAKE, float("inf"), None) == 4
+    assert a(FAKE, 1, 8, 6, 4, 1, FAKE, None) == 2          # Hq not a multiple of Hkv
+    assert a(FAKE, 1, 8, 4, 2, 2, FAKE, None) == 4          # causal not 0 or 1
+    assert a(FAKE, 1, 8, 4, 2, 1, None, None) == 1          # NULL out
+    assert a(FAKE, -1, 8, 4, 2, 1, FAKE, None) == 2         # negative B
+    assert a(ctypes.c_void_p((1 << 20) + 4), 1, 8, 4, 2, 1, FAKE, None) == 3   # misaligned qkv
+
+
 @pytest.mark.skipif(torch.cuda.is_available(), reason="checks the behaviour without a GPU")
 def test_well_formed_call_without_gpu_fails_loudly(lib):
     st = lib.cer_select_topk(FAKE, 1, 8, 0, 8, 4, FAKE, None, None)
