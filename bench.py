@@ -146,6 +146,54 @@ def workload_config(w: gen.Workload, flush: bool) -> dict:
             "inputs": "seeded synthetic (SplitMix64 normals), resident in HBM"}
 
 
+def device_time(torch, stream, flush, fn, reps=20):
+    """Mean device time (ms) of fn's launches after 3 untimed calls, L2
+    flushed before each; a GPU spin before the start event keeps the host's
+    launch overhead out of the interval."""
+    ms = []
+    for i in range(reps + 3):
+        flush.fill_(float(i))
+        torch.cuda._sleep(200000)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        fn()
+        b.record(stream)
+        b.synchronize()
+        if i >= 3:
+            ms.append(a.elapsed_time(b))
+    return float(np.mean(ms))
+
+
+def measure_attention(cer, torch, w, flush, stream, dev, peak_tf, reps=20):
+    """Rotary embedding and attention over the packed sequences (L = k_tot
+    retained tokens per sequence) with the workload's backbone heads: causal
+    for understanding (prefill), bidirectional for generation.  Synthetic
+    packed rows; positions are an ascending keep list."""
+    Hq, Hkv = w.attn_heads()
+    L = w.k_tot
+    causal = 1 if w.task == 0 else 0
+    width = (Hq + 2 * Hkv) * 128
+    bits = gen.bf16_normal(w.seed, "attn_qkv", (w.B * L, width), 1.0)
+    qkv0 = torch.from_numpy(bits.view(np.int16)).view(torch.bfloat16).to(dev)
+    qkv = qkv0.clone()
+    rng = np.random.default_rng(w.seed)
+    pos = np.concatenate([np.sort(rng.choice(w.N, L, replace=False)) for _ in range(w.B)]).astype(np.int32)
+    pos_d = torch.from_numpy(pos).to(dev)
+    out = torch.empty((w.B * L, Hq * 128), dtype=torch.bfloat16, device=dev)
+    t_rope = device_time(torch, stream, flush, lambda: cer.cer_rope_packed(qkv, w.B, L, Hq, Hkv, pos_d, 1e6,
+                                                                          stream=stream), reps)
+    t_attn = device_time(torch, stream, flush, lambda: cer.cer_packed_attention(qkv, w.B, L, Hq, Hkv, causal, out,
+                                                                               stream=stream), reps)
+    cer.cer_sync_status(stream)
+    flops = w.attn_flops(bool(causal))
+    tf = flops / (t_attn * 1e-3) / 1e12
+    rope_bytes = 2.0 * w.B * L * (Hq + Hkv) * 128 * 2 + 4 * w.B * L
+    return {"heads": [Hq, Hkv], "packed_len": L, "causal": bool(causal),
+            "rope_us": t_rope * 1e3, "rope_gbs": rope_bytes / (t_rope * 1e-3) / 1e9,
+            "attention_us": t_attn * 1e3, "attention_flops": flops, "attention_tflops": tf,
+            "attention_frac": tf / peak_tf, "peak_source": "bf16_tflops (burst) of measured"}
+
+
 def measure_ucs(cer, torch, w, h0, h, flush, stream, dev, core, exp, t, Wg, Wu, WdT, ws, inp, reps=20):
     """Time the UCS kernels on the workload's own tensors: the keep masks of two
     block calls (t and t_ref = the same inputs with t + 0.05), the redundancy
@@ -165,24 +213,10 @@ def measure_ucs(cer, torch, w, h0, h, flush, stream, dev, core, exp, t, Wg, Wu, 
     skip = torch.empty(w.B, dtype=torch.uint8, device=dev)
     gws = cer.workspace(cer.load().cer_redundancy_gap_workspace_size(w.B, w.N), dev)
 
-    def timed(fn):
-        """Device time of fn's launches.  A GPU spin before the start event keeps
-        the host's launch overhead out of the interval."""
-        ms = []
-        for i in range(reps + 3):
-            flush.fill_(float(i))
-            torch.cuda._sleep(200000)
-            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            a.record(stream)
-            fn()
-            b.record(stream)
-            b.synchronize()
-            if i >= 3:
-                ms.append(a.elapsed_time(b))
-        return float(np.mean(ms))
-
-    t_drop = timed(lambda: cer.cer_drop_set_stats(masks[0], masks[1], w.r0, w.r1, jac, None, rda, stream=stream))
-    t_gap = timed(lambda: cer.cer_redundancy_gap(h0, h, masks[1], 0.004, gap, skip, ws=gws, stream=stream))
+    t_drop = device_time(torch, stream, flush, lambda: cer.cer_drop_set_stats(masks[0], masks[1], w.r0, w.r1, jac,
+                                                                               None, rda, stream=stream), reps)
+    t_gap = device_time(torch, stream, flush, lambda: cer.cer_redundancy_gap(h0, h, masks[1], 0.004, gap, skip,
+                                                                              ws=gws, stream=stream), reps)
     cer.cer_sync_status(stream)
     gated = {}
     if w.C < w.I and w.I % 64 == 0:
@@ -401,11 +435,14 @@ def run_gpu(args, info):
     # ---- UCS statistics on this step's tensors (Sec. 3.4): drop-set J/RDA of
     # two keep masks, redundancy gap of the block's input and output
     ucs = measure_ucs(cer, torch, w, h0, h, flush, stream, dev, core, exp, t, Wg, Wu, WdT, ws, inp)
+    peaks, peak_kind = load_peaks()
+    # ---- attention on the packed sequence (Sec. 3.4): rotary embedding and
+    # softmax attention over the retained tokens, with the backbone's heads
+    attn = measure_attention(cer, torch, w, flush, stream, dev, float(peaks["bf16_tflops"]))
 
     if not info.is_root:
         return 0
 
-    peaks, peak_kind = load_peaks()
     score_ms, topk_ms, gather_ms, gateup_ms, down_ms = (float(x) for x in stage.mean(axis=0))
     gateup_flops = 4.0 * w.M * w.d * w.C
     achieved = gateup_flops / (gateup_ms * 1e-3) / 1e12
@@ -443,6 +480,7 @@ def run_gpu(args, info):
                 "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
         "ucs": {**ucs, "redundancy_gap_hbm_frac": ucs["redundancy_gap_gbs"] / float(peaks["hbm_gbs"]),
                 "peak_source": f"hbm_gbs of {peak_kind}"},
+        "attention": {**attn, "rope_hbm_frac": attn["rope_gbs"] / float(peaks["hbm_gbs"])},
         "gpu_launches": kernels_per_step(w.task) * args.steps,
         "stage_pass": f"per-stage times from a separate pass of {n_stage} steps with events between kernels",
         "clocks": clocks.summary(),

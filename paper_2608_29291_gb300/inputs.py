@@ -178,6 +178,20 @@ class Workload:
         h = self.Hc + (self.He if self.task == 1 else 0)
         return 2 * self.B * self.N * self.d * h
 
+    def attn_heads(self):
+        """(query heads, key/value heads) of the Qwen2.5 backbone with this
+        width (head size 128): 12/2 for the 1.5B model, 28/4 for the 7B."""
+        known = {1536: (12, 2), 3584: (28, 4)}
+        return known.get(self.d, (max(1, self.d // 128), 1))
+
+    def attn_flops(self, causal: bool) -> int:
+        """Q K^T and P V over the packed sequences (only the admissible pairs
+        when causal)."""
+        Hq, _ = self.attn_heads()
+        L = self.k_tot
+        pairs = L * (L + 1) // 2 if causal else L * L
+        return 4 * self.B * Hq * 128 * pairs
+
 
 def tiny() -> Workload:
     return Workload("tiny_b1_n256_d256", B=1, N=256, d=256, I=1024, C=512, r0=0, r1=256,
