@@ -375,3 +375,30 @@ def packed_attention(Q: np.ndarray, K: np.ndarray, V: np.ndarray, causal: bool, 
         P = P / P.sum(axis=1, keepdims=True)
         O[:, h, :] = P @ V[:, kh, :]
     return O
+
+
+def routed_attention(h, idx, WqkvT, WoT, Hq: int, Hkv: int, causal: bool, base: float) -> dict:
+    """Attention sublayer on the packed sequence (Sec. 3.4): pack R, project to
+    queries, keys and values (Q | K | V = X WqkvT, the projection stored
+    input-major [d, (Hq + 2 Hkv) * 128]), rotate Q and K at the tokens'
+    original positions idx, attend within each packed sequence, project back
+    (Y = A WoT, WoT [Hq * 128, d]) and scatter-add: kept rows become
+    bf16(h + Y), dropped rows bypass.  fp64 throughout, no intermediate
+    rounding.  Returns the packed K and V too (the compressed KV cache)."""
+    B, k_tot = idx.shape
+    X = bf16_to_f64(gather(h, idx))
+    QKV = X @ bf16_to_f64(WqkvT)
+    T = X.shape[0]
+    dh = 128
+    Q = QKV[:, : Hq * dh].reshape(T, Hq, dh)
+    K = QKV[:, Hq * dh: (Hq + Hkv) * dh].reshape(T, Hkv, dh)
+    V = QKV[:, (Hq + Hkv) * dh:].reshape(T, Hkv, dh)
+    pos = np.asarray(idx, dtype=np.int64).reshape(-1)
+    Q = rope(Q, pos, base)
+    K = rope(K, pos, base)
+    A = np.empty((T, Hq * dh), dtype=np.float64)
+    for b in range(B):
+        s = slice(b * k_tot, (b + 1) * k_tot)
+        A[s] = packed_attention(Q[s], K[s], V[s], causal).reshape(k_tot, Hq * dh)
+    Y = A @ bf16_to_f64(WoT)
+    return {"Y": Y, "out": scatter_add(h, idx, Y), "K": K, "V": V, "A": A}

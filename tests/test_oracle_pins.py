@@ -690,3 +690,46 @@ def test_attention_pins_catch_planted_mistake(name, monkeypatch):
     attr, make = ATTENTION_MUTATIONS[name]
     monkeypatch.setattr(ora, attr, make(getattr(ora, attr)))
     assert _rope_checks() + _attention_checks(), f"planted mistake {name} went unnoticed"
+
+
+def test_routed_attention_composition():
+    """The sublayer against torch as a second opinion (projections, rotary
+    embedding from its closed form, sdpa with grouped heads), a zero output
+    projection leaving h bit-identical, and dropped rows bypassing."""
+    rng = np.random.default_rng(8)
+    B, N, d, Hq, Hkv = 2, 40, 64, 4, 2
+    h = _bits(np.round(rng.normal(size=(B, N, d)) * 8) / 8 + 0.0)   # + 0.0: no negative zeros (-0 + 0 = +0)
+    idx = np.stack([np.sort(rng.choice(N, 13, replace=False)) for _ in range(B)]).astype(np.int32)
+    WqkvT = gen.bf16_normal(3, "wqkv", (d, (Hq + 2 * Hkv) * 128), d ** -.5)
+    WoT = gen.bf16_normal(3, "wo", (Hq * 128, d), (Hq * 128) ** -.5)
+    for causal in (True, False):
+        res = ora.routed_attention(h, idx, WqkvT, WoT, Hq, Hkv, causal, 1e6)
+        X = torch.tensor(ora.bf16_to_f64(ora.gather(h, idx)))
+        qkv = X @ torch.tensor(ora.bf16_to_f64(WqkvT))
+        T = qkv.shape[0]
+        q = qkv[:, : Hq * 128].reshape(T, Hq, 128)
+        k = qkv[:, Hq * 128: (Hq + Hkv) * 128].reshape(T, Hkv, 128)
+        v = qkv[:, (Hq + Hkv) * 128:].reshape(T, Hkv, 128)
+        pos = torch.tensor(idx.reshape(-1), dtype=torch.float64)
+        inv = 1e6 ** (-torch.arange(0, 128, 2, dtype=torch.float64) / 128)
+        ang = pos[:, None] * inv[None]
+        cos, sin = torch.cos(ang).repeat(1, 2)[:, None], torch.sin(ang).repeat(1, 2)[:, None]
+
+        def rot(x):
+            return x * cos + torch.cat([-x[..., 64:], x[..., :64]], dim=-1) * sin
+        q, k = rot(q), rot(k)
+        outs = []
+        for b in range(B):
+            s = slice(b * 13, (b + 1) * 13)
+            qq = q[s].permute(1, 0, 2)[None]
+            kk = k[s].permute(1, 0, 2).repeat_interleave(Hq // Hkv, dim=0)[None]
+            vv = v[s].permute(1, 0, 2).repeat_interleave(Hq // Hkv, dim=0)[None]
+            outs.append(F.scaled_dot_product_attention(qq, kk, vv, is_causal=causal)[0].permute(1, 0, 2).reshape(13, -1))
+        Y = torch.cat(outs) @ torch.tensor(ora.bf16_to_f64(WoT))
+        assert np.allclose(res["Y"], Y.numpy(), atol=1e-10), np.abs(res["Y"] - Y.numpy()).max()
+    zero = ora.routed_attention(h, idx, WqkvT, np.zeros_like(WoT), Hq, Hkv, True, 1e6)
+    assert np.array_equal(zero["out"], h)
+    kept = np.zeros((B, N), bool)
+    for b in range(B):
+        kept[b, idx[b]] = True
+    assert np.array_equal(res["out"][~kept], h[~kept])
