@@ -184,14 +184,31 @@ def measure_attention(cer, torch, w, flush, stream, dev, peak_tf, reps=20):
                                                                           stream=stream), reps)
     t_attn = device_time(torch, stream, flush, lambda: cer.cer_packed_attention(qkv, w.B, L, Hq, Hkv, causal, out,
                                                                                stream=stream), reps)
+    # The whole sublayer from the residual stream: pack, QKV projection, rotary
+    # embedding, attention, output projection with the scatter-add.
+    h = torch.from_numpy(gen.bf16_normal(w.seed, "attn_h", (w.B, w.N, w.d), 1.0).view(np.int16)).view(
+        torch.bfloat16).to(dev)
+    hout = torch.empty_like(h)
+    WqkvT = torch.from_numpy(gen.bf16_normal(w.seed, "wqkv", (w.d, width), w.d ** -0.5).view(np.int16)).view(
+        torch.bfloat16).to(dev)
+    WoT = torch.from_numpy(gen.bf16_normal(w.seed, "wo", (Hq * 128, w.d), (Hq * 128) ** -0.5).view(np.int16)).view(
+        torch.bfloat16).to(dev)
+    idx = pos_d.view(w.B, L)
+    aws = cer.workspace(cer.load().cer_routed_attention_workspace_size(w.B, L, w.d, Hq, Hkv), dev)
+    t_layer = device_time(torch, stream, flush, lambda: cer.cer_routed_attention(
+        h, idx, WqkvT, WoT, Hq, Hkv, causal, out=hout, ws=aws, stream=stream), reps)
     cer.cer_sync_status(stream)
+    proj_flops = 2.0 * w.B * L * w.d * (width + Hq * 128)
     flops = w.attn_flops(bool(causal))
     tf = flops / (t_attn * 1e-3) / 1e12
     rope_bytes = 2.0 * w.B * L * (Hq + Hkv) * 128 * 2 + 4 * w.B * L
     return {"heads": [Hq, Hkv], "packed_len": L, "causal": bool(causal),
             "rope_us": t_rope * 1e3, "rope_gbs": rope_bytes / (t_rope * 1e-3) / 1e9,
             "attention_us": t_attn * 1e3, "attention_flops": flops, "attention_tflops": tf,
-            "attention_frac": tf / peak_tf, "peak_source": "bf16_tflops (burst) of measured"}
+            "attention_frac": tf / peak_tf, "peak_source": "bf16_tflops (burst) of measured",
+            "sublayer_us": t_layer * 1e3, "sublayer_tflops": (proj_flops + flops) / (t_layer * 1e-3) / 1e12,
+            "sublayer": "gather, QKV projection, rotary embedding, attention, output projection + scatter-add "
+                        "(out of place)"}
 
 
 def measure_ucs(cer, torch, w, h0, h, flush, stream, dev, core, exp, t, Wg, Wu, WdT, ws, inp, reps=20):

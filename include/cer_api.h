@@ -329,6 +329,31 @@ cer_status cer_rope_packed(void* qkv, int B, int L, int Hq, int Hkv, const int32
 cer_status cer_packed_attention(const void* qkv, int B, int L, int Hq, int Hkv, int causal, void* out,
                                 cudaStream_t stream);
 
+/* cer_routed_attention: the attention sublayer on the packed sequence,
+ *   X = h[b, idx[b, :]] (packed, [B * L, d]),
+ *   qkv = X WqkvT, rotated at the original positions idx (as cer_rope_packed),
+ *   A = cer_packed_attention(qkv),
+ *   out[b, idx[b, j]] = bf16(h[b, idx[b, j]] + (A WoT)[b * L + j]); other rows
+ *   bypass (bit-identical; copied when out != h).
+ *   h      bf16 [B, N, d] device; out NULL or == h: in place
+ *   idx    int32 [B, L] device: ascending keep list per sequence (e.g. from
+ *          cer_select_topk); out-of-range entries are reported as
+ *          CER_ERR_INDEX by cer_sync_status and their rows skipped
+ *   WqkvT  bf16 [d, (Hq + 2 Hkv) * 128] device: the QKV projection stored
+ *          input-major (column j of W_qkv's transpose per output feature)
+ *   WoT    bf16 [Hq * 128, d] device: the output projection, input-major
+ *   qkv    NULL, or bf16 [B * L, (Hq + 2 Hkv) * 128] device: receives the
+ *          rotated packed rows; their key and value heads are the compressed
+ *          KV cache of the sublayer
+ * Requires d a multiple of 64 in [64, 16384] and the head conditions above.
+ * The projections accumulate in fp32 on the tensor cores (tcgen05 pair
+ * MMA) and round to bf16, like the FFN.
+ * Workspace: cer_routed_attention_workspace_size(B, L, d, Hq, Hkv).       */
+cer_status cer_routed_attention(void* h, void* out, int B, int N, int d, const int32_t* idx, int L,
+                                const void* WqkvT, const void* WoT, int Hq, int Hkv, int causal, double base,
+                                void* qkv, void* workspace, size_t workspace_bytes, cudaStream_t stream);
+size_t cer_routed_attention_workspace_size(int B, int L, int d, int Hq, int Hkv);
+
 /* ------------------------------------------------------------------ status
  * cer_sync_status: synchronise `stream`, then return and clear the current
  * device's status word (the first kernel-detected error since the last call),

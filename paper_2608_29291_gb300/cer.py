@@ -31,7 +31,8 @@ EXPORTS = ("cer_score", "cer_score_workspace_size", "cer_score_static", "cer_sel
            "cer_routed_block_workspace_size", "cer_ffn_channel_norms", "cer_routed_ffn_gated",
            "cer_routed_ffn_gated_workspace_size", "cer_routed_block_gated", "cer_routed_block_gated_workspace_size",
            "cer_drop_set_stats", "cer_redundancy_gap",
-           "cer_redundancy_gap_workspace_size", "cer_rope_packed", "cer_packed_attention", "cer_sync_status",
+           "cer_redundancy_gap_workspace_size", "cer_rope_packed", "cer_packed_attention",
+           "cer_routed_attention", "cer_routed_attention_workspace_size", "cer_sync_status",
            "cer_get_error", "cer_status_string", "cer_version")
 
 
@@ -75,6 +76,9 @@ _SIGS = {
     "cer_redundancy_gap_workspace_size": ([_i, _i], _sz),
     "cer_rope_packed": ([_vp, _i, _i, _i, _i, _vp, ctypes.c_double, _vp], _i),
     "cer_packed_attention": ([_vp, _i, _i, _i, _i, _i, _vp, _vp], _i),
+    "cer_routed_attention": ([_vp, _vp, _i, _i, _i, _vp, _i, _vp, _vp, _i, _i, _i, ctypes.c_double, _vp, _vp,
+                              _sz, _vp], _i),
+    "cer_routed_attention_workspace_size": ([_i, _i, _i, _i, _i], _sz),
     "cer_sync_status": ([_vp], _i),
     "cer_get_error": ([], ctypes.c_char_p),
     "cer_status_string": ([_i], ctypes.c_char_p),
@@ -310,6 +314,18 @@ def cer_packed_attention(qkv, B, L, Hq, Hkv, causal, out=None, stream=None):
         out = torch.empty((B * L, Hq * 128), dtype=torch.bfloat16, device=qkv.device)
     _check(load().cer_packed_attention(_p(qkv), B, L, Hq, Hkv, int(causal), _p(out), _stream(stream)))
     return out
+
+
+def cer_routed_attention(h, idx, WqkvT, WoT, Hq, Hkv, causal, base=1e6, out=None, qkv=None, ws=None,
+                         stream=None):
+    """Attention sublayer on the packed sequence; h [B, N, d] updated in place unless out is given."""
+    B, N, d = h.shape
+    L = idx.shape[1]
+    if ws is None:
+        ws = workspace(load().cer_routed_attention_workspace_size(B, L, d, Hq, Hkv), h.device)
+    _check(load().cer_routed_attention(_p(h), _p(out), B, N, d, _p(idx), L, _p(WqkvT), _p(WoT), Hq, Hkv,
+                                       int(causal), float(base), _p(qkv), _p(ws), ws.numel(), _stream(stream)))
+    return h if out is None else out
 
 
 def cer_sync_status(stream=None) -> None:

@@ -934,4 +934,109 @@ cer_status cer_packed_attention(const void* qkv, int B, int L, int Hq, int Hkv, 
   return CER_OK;
 }
 
+size_t cer_routed_attention_workspace_size(int B, int L, int d, int Hq, int Hkv) {
+  if (B < 0 || L < 0 || d < 0 || Hq < 1 || Hkv < 1) return 0;
+  const long long M = static_cast<long long>(B) * L;
+  const size_t width = static_cast<size_t>(Hq + 2 * Hkv) * cer::kHeadDim;
+  return round256(static_cast<size_t>(M) * d * 2) + round256(static_cast<size_t>(M) * width * 2) +
+         round256(static_cast<size_t>(M) * Hq * cer::kHeadDim * 2) + ffn_stream_k_bytes(M);
+}
+
+cer_status cer_routed_attention(void* h, void* out, int B, int N, int d, const int32_t* idx, int L,
+                                const void* WqkvT, const void* WoT, int Hq, int Hkv, int causal, double base,
+                                void* qkv, void* workspace, size_t workspace_bytes, cudaStream_t stream) {
+  const long long M64 = static_cast<long long>(B) * L;
+  const bool any_h = static_cast<long long>(B) * N > 0;
+  CER_PTR_IF(h, any_h);
+  CER_PTR_IF(idx, M64 > 0);
+  CER_PTR(WqkvT);
+  CER_PTR(WoT);
+  CER_ALIGN(h);
+  CER_ALIGN(out);
+  CER_ALIGN(idx);
+  CER_ALIGN(WqkvT);
+  CER_ALIGN(WoT);
+  CER_ALIGN(qkv);
+  CER_ALIGN(workspace);
+  cer_status s = check_qkv(B, L, Hq, Hkv);
+  if (s != CER_OK) return s;
+  CER_REQUIRE(N >= 0 && L <= N, CER_ERR_SHAPE, "L=%d must be in [0, N=%d]", L, N);
+  CER_REQUIRE(d >= 64 && d <= 16384 && d % 64 == 0, CER_ERR_SHAPE, "d=%d must be a multiple of 64 in [64, 16384]", d);
+  CER_REQUIRE(causal == 0 || causal == 1, CER_ERR_RANGE, "causal=%d must be 0 or 1", causal);
+  CER_REQUIRE(base > 1.0 && std::isfinite(base), CER_ERR_RANGE, "rotary base %g must be finite and > 1", base);
+  const size_t need = cer_routed_attention_workspace_size(B, L, d, Hq, Hkv);
+  CER_REQUIRE(M64 == 0 || (workspace != nullptr && workspace_bytes >= need), CER_ERR_WORKSPACE,
+              "workspace of %zu bytes needed, %zu given", need, workspace_bytes);
+  const bool in_place = (out == nullptr || out == h);
+  const size_t hbytes = static_cast<size_t>(B) * N * d * 2;
+  if (!in_place) {
+    CER_PTR_IF(out, any_h);
+    const char* a0 = static_cast<const char*>(h);
+    const char* b0 = static_cast<const char*>(out);
+    CER_REQUIRE(b0 + hbytes <= a0 || a0 + hbytes <= b0, CER_ERR_RANGE, "out overlaps h without being equal to it");
+  }
+  DeviceInfo* dev = nullptr;
+  if ((s = device_info(&dev)) != CER_OK) return s;
+  void* dst = in_place ? h : out;
+  cudaError_t e;
+  if (!in_place && hbytes) {
+    e = cudaMemcpyAsync(out, h, hbytes, cudaMemcpyDeviceToDevice, stream);   // bypass rows
+    if (e != cudaSuccess) return cuda_fail(e, "bypass copy");
+  }
+  if (M64 == 0) return CER_OK;
+  const int M = static_cast<int>(M64);
+  const int width = (Hq + 2 * Hkv) * cer::kHeadDim;
+  char* ws = static_cast<char*>(workspace);
+  __nv_bfloat16* X = reinterpret_cast<__nv_bfloat16*>(ws);
+  ws += round256(static_cast<size_t>(M) * d * 2);
+  __nv_bfloat16* qkv_ws = reinterpret_cast<__nv_bfloat16*>(ws);
+  ws += round256(static_cast<size_t>(M) * width * 2);
+  __nv_bfloat16* attn = reinterpret_cast<__nv_bfloat16*>(ws);
+  ws += round256(static_cast<size_t>(M) * Hq * cer::kHeadDim * 2);
+  cer::FfnArgs proj{};
+  carve_stream_k(&ws, M, &proj);
+  __nv_bfloat16* qkv_rows = qkv ? static_cast<__nv_bfloat16*>(qkv) : qkv_ws;
+
+  // pack R
+  e = cer::launch_gather(static_cast<const __nv_bfloat16*>(h), B, N, d, idx, L, X, dev->status, dev->n_sm, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "gather launch");
+  // qkv = X WqkvT: the down-projection GEMM in plain-output mode (K = d, N = width)
+  cer::FfnArgs q = proj;
+  q.act = X;
+  q.M = M;
+  q.C = d;
+  q.d = width;
+  q.WdT = static_cast<const __nv_bfloat16*>(WqkvT);
+  q.Y = qkv_rows;
+  q.scatter = 0;
+  q.status = dev->status;
+  e = cer::launch_ffn_down(q, dev->n_sm, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "QKV projection launch");
+  // rotary embedding at the original positions, then attention on the packed rows
+  cer::RopeFreqTable ft;
+  for (int j = 0; j < cer::kHeadDim / 2; ++j)
+    ft.g[j] = std::pow(base, -2.0 * j / cer::kHeadDim) / (2.0 * M_PI);
+  e = cer::launch_rope(qkv_rows, M, Hq, Hkv, idx, ft, dev->status, dev->n_sm, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "rotary embedding launch");
+  e = cer::launch_packed_attention(qkv_rows, B, L, Hq, Hkv, causal, attn, dev->status, dev->n_sm, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "packed attention launch");
+  // out[b, idx] = bf16(h + A WoT): the down-projection GEMM with its fused unpack
+  cer::FfnArgs o = proj;
+  o.act = attn;
+  o.M = M;
+  o.C = Hq * cer::kHeadDim;
+  o.d = d;
+  o.WdT = static_cast<const __nv_bfloat16*>(WoT);
+  o.h = static_cast<const __nv_bfloat16*>(h);
+  o.out = static_cast<__nv_bfloat16*>(dst);
+  o.idx = idx;
+  o.N = N;
+  o.k_tot = L;
+  o.scatter = 1;
+  o.status = dev->status;
+  e = cer::launch_ffn_down(o, dev->n_sm, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "output projection launch");
+  return CER_OK;
+}
+
 }  // extern "C"

@@ -122,6 +122,15 @@ def test_attention_argument_checks(lib):
     assert a(FAKE, 1, 8, 4, 2, 1, None, None) == 1          # NULL out
     assert a(FAKE, -1, 8, 4, 2, 1, FAKE, None) == 2         # negative B
     assert a(ctypes.c_void_p((1 << 20) + 4), 1, 8, 4, 2, 1, FAKE, None) == 3   # misaligned qkv
+    ra, big = lib.cer_routed_attention, 1 << 30
+    assert ra(FAKE, None, 1, 16, 100, FAKE, 8, FAKE, FAKE, 4, 2, 1, 1e6, None, FAKE, big, None) == 2   # d % 64
+    assert ra(FAKE, None, 1, 16, 128, FAKE, 20, FAKE, FAKE, 4, 2, 1, 1e6, None, FAKE, big, None) == 2  # L > N
+    assert ra(FAKE, None, 1, 16, 128, FAKE, 8, None, FAKE, 4, 2, 1, 1e6, None, FAKE, big, None) == 1   # NULL WqkvT
+    assert ra(FAKE, None, 1, 16, 128, FAKE, 8, FAKE, FAKE, 4, 2, 1, 1e6, None, FAKE, 64, None) == 9    # workspace
+    W = (4 + 2 * 2) * 128
+    assert lib.cer_routed_attention_workspace_size(2, 10, 128, 4, 2) == \
+        _r256(20 * 128 * 2) + _r256(20 * W * 2) + _r256(20 * 512 * 2) + (24 << 20) + 8192
+    assert lib.cer_routed_attention_workspace_size(2, 0, 128, 4, 2) == 0
 
 
 @pytest.mark.skipif(torch.cuda.is_available(), reason="checks the behaviour without a GPU")

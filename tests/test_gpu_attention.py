@@ -16,7 +16,7 @@ import torch
 from oracle import cer_oracle as ora
 from paper_2608_29291_gb300 import cer
 from paper_2608_29291_gb300 import inputs as gen
-from tests.gpu_helpers import bf16_dev, bits_host, i32_dev, ulp_bf16
+from tests.gpu_helpers import bf16_dev, bits_host, i32_dev, out_err_ok, ulp_bf16
 
 pytestmark = pytest.mark.gpu
 DH = 128
@@ -161,3 +161,47 @@ def test_empty_inputs_are_no_ops():
     cer.cer_packed_attention(torch.empty(0, device="cuda", dtype=torch.bfloat16), 3, 0, 2, 1, 1,
                              out=torch.empty(0, device="cuda", dtype=torch.bfloat16))
     cer.cer_sync_status()
+
+
+# ------------------------------------------------------------------ the attention sublayer
+
+BLOCK_TOL = 2e-2     # the routed block's output tolerance: 2e-2 * RMS + half a bf16 ulp
+
+
+def _sublayer_inputs(seed, B, N, d, L, Hq, Hkv):
+    h = gen.bf16_normal(seed, "h", (B, N, d), 1.0)
+    rng = np.random.default_rng(seed)
+    idx = np.stack([np.sort(rng.choice(N, L, replace=False)) for _ in range(B)]).astype(np.int32)
+    WqkvT = gen.bf16_normal(seed, "wqkv", (d, (Hq + 2 * Hkv) * DH), d ** -0.5)
+    WoT = gen.bf16_normal(seed, "wo", (Hq * DH, d), (Hq * DH) ** -0.5)
+    return h, idx, WqkvT, WoT
+
+
+@pytest.mark.parametrize("B,N,d,L,Hq,Hkv,causal,inplace", [
+    (2, 300, 256, 100, 4, 2, 1, True), (1, 200, 512, 200, 2, 1, 0, False), (3, 130, 128, 1, 1, 1, 1, True),
+    (2, 700, 768, 333, 6, 3, 0, True), (1, 1024, 1536, 587, 12, 2, 1, True)])
+def test_routed_attention_matches_oracle(B, N, d, L, Hq, Hkv, causal, inplace):
+    h, idx, WqkvT, WoT = _sublayer_inputs(B * 131 + L, B, N, d, L, Hq, Hkv)
+    hd = bf16_dev(h)
+    out = None if inplace else torch.empty_like(hd)
+    qkv = torch.empty((B * L, (Hq + 2 * Hkv) * DH), dtype=torch.bfloat16, device="cuda")
+    cer.cer_routed_attention(hd, i32_dev(idx), bf16_dev(WqkvT), bf16_dev(WoT), Hq, Hkv, causal, out=out, qkv=qkv)
+    cer.cer_sync_status()
+    got = bits_host(hd if inplace else out)
+    if not inplace:
+        assert np.array_equal(bits_host(hd), h)                           # h untouched
+    res = ora.routed_attention(h, idx, WqkvT, WoT, Hq, Hkv, bool(causal), 1e6)
+    kept = np.zeros((B, N), bool)
+    for b in range(B):
+        kept[b, idx[b]] = True
+    assert np.array_equal(got[~kept], h[~kept])                           # dropped rows bypass
+    exact = ora.bf16_to_f64(h).copy()
+    for b in range(B):
+        exact[b, idx[b]] += res["Y"][b * L:(b + 1) * L]
+    ok, excess = out_err_ok(ora.bf16_to_f64(got[kept]), exact[kept], BLOCK_TOL)
+    assert ok, excess
+    # the compressed KV cache: the rotated key and value heads of the packed rows
+    cache = ora.bf16_to_f64(bits_host(qkv))[:, Hq * DH:].reshape(B * L, 2 * Hkv, DH)
+    want = np.concatenate([res["K"], res["V"]], axis=1)
+    ok, excess = out_err_ok(cache, want, BLOCK_TOL)
+    assert ok, excess
