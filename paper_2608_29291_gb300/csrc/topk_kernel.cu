@@ -77,10 +77,19 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(TopkArgs a) {
   if (tid == 0) s_nan = 0;
   __syncthreads();
 
-  // 1. logits (reduced from partial sums in chunk order) -> keys
+  // 1. logits (reduced from partial sums in chunk order) -> keys; the
+  // partial rows are read eight at a time so their loads overlap.
   for (int i = tid; i < N; i += blockDim.x) {
-    float v = a.src[base + i];
-    for (int c = 1; c < a.n_chunks; ++c) v += a.src[static_cast<size_t>(c) * a.chunk_stride + base + i];
+    float v = 0.f;
+    for (int c0 = 0; c0 < a.n_chunks; c0 += 8) {
+      float part[8];
+#pragma unroll
+      for (int c = 0; c < 8; ++c)
+        part[c] = c0 + c < a.n_chunks ? __ldg(a.src + static_cast<size_t>(c0 + c) * a.chunk_stride + base + i) : 0.f;
+#pragma unroll
+      for (int c = 0; c < 8; ++c)
+        if (c0 + c < a.n_chunks) v = (c0 + c == 0) ? part[c] : v + part[c];
+    }
     if (a.logits_out) a.logits_out[base + i] = v;
     if (a.probs_out) a.probs_out[base + i] = 1.0f / (1.0f + expf(-v));
     if (i >= a.r0 && i < a.r1 && v != v) s_nan = 1;
@@ -97,9 +106,12 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(TopkArgs a) {
   // 2. radix select of the K-th largest routable key
   if (!keep_all && !keep_none) {
     uint32_t prefix = 0, pmask = 0, remaining = static_cast<uint32_t>(K);
+    for (int i = tid; i < kSubHist * 256; i += blockDim.x) (&sub[0][0])[i] = 0;
+    __syncthreads();
+    // Three barriers per pass: the merge also clears the sub-histograms for
+    // the next pass, and s_prefix is rewritten only two barriers after every
+    // thread has read it.
     for (int shift = 24; shift >= 0; shift -= 8) {
-      for (int i = tid; i < kSubHist * 256; i += blockDim.x) (&sub[0][0])[i] = 0;
-      __syncthreads();
       uint32_t* my = sub[(tid >> 5) % kSubHist];
       for (int i = a.r0 + tid; i < a.r1; i += blockDim.x) {
         const uint32_t k = keys[i];
@@ -109,7 +121,10 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(TopkArgs a) {
       for (int i = tid; i < 256; i += blockDim.x) {
         uint32_t c = 0;
 #pragma unroll
-        for (int q = 0; q < kSubHist; ++q) c += sub[q][i];
+        for (int q = 0; q < kSubHist; ++q) {
+          c += sub[q][i];
+          sub[q][i] = 0;
+        }
         hist[i] = c;
       }
       __syncthreads();
@@ -142,7 +157,6 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(TopkArgs a) {
       prefix = s_prefix;
       remaining = s_remaining;
       pmask |= 255u << shift;
-      __syncthreads();
     }
     thr = prefix;
     need_eq = remaining;
