@@ -60,34 +60,45 @@ __global__ void __launch_bounds__(kRopeThreads)
   const long long warps = static_cast<long long>(gridDim.x) * (kRopeThreads / 32);
   for (long long row = blockIdx.x * (kRopeThreads / 32) + (threadIdx.x >> 5); row < rows; row += warps) {
     const int p = __ldg(pos + row);
-    if (p < 0) {
-      if (lane == 0) record_status(status, CER_DEV_INDEX);
-      continue;
-    }
-    float c[8], s[8];
-#pragma unroll
-    for (int e = 0; e < 8; ++e) {
-      const double x = static_cast<double>(p) * ft.g[j0 + e];
-      sincospif(2.0f * static_cast<float>(x - rint(x)), &s[e], &c[e]);
-    }
     __nv_bfloat16* r = qkv + row * width;
-    for (int h = lane >> 3; h < heads; h += 4) {
-      uint4* lo4 = reinterpret_cast<uint4*>(r + h * kHeadDim + j0);
-      uint4* hi4 = reinterpret_cast<uint4*>(r + h * kHeadDim + 64 + j0);
-      uint4 lo = *lo4, hi = *hi4;
-      uint32_t* lw = reinterpret_cast<uint32_t*>(&lo);
-      uint32_t* hw = reinterpret_cast<uint32_t*>(&hi);
+    // Heads lane/8, lane/8 + 4, ... in batches of four: a batch's loads are
+    // issued before the angles (and the previous batch's stores) are needed.
+    for (int h0 = lane >> 3; h0 < heads; h0 += 16) {
+      uint4 lo[4], hi[4];
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const float2 a = __bfloat1622float2(*reinterpret_cast<__nv_bfloat162*>(&lw[e]));
-        const float2 b = __bfloat1622float2(*reinterpret_cast<__nv_bfloat162*>(&hw[e]));
-        const int k = 2 * e;
-        lw[e] = pack_bf16x2(fmaf(a.x, c[k], -b.x * s[k]), fmaf(a.y, c[k + 1], -b.y * s[k + 1]));
-        hw[e] = pack_bf16x2(fmaf(b.x, c[k], a.x * s[k]), fmaf(b.y, c[k + 1], a.y * s[k + 1]));
+      for (int i = 0; i < 4; ++i) {
+        const int h = h0 + 4 * i;
+        if (h < heads) {
+          lo[i] = *reinterpret_cast<const uint4*>(r + h * kHeadDim + j0);
+          hi[i] = *reinterpret_cast<const uint4*>(r + h * kHeadDim + 64 + j0);
+        }
       }
-      *lo4 = lo;
-      *hi4 = hi;
+      if (p < 0) break;
+      float c[8], s[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        const double x = static_cast<double>(p) * ft.g[j0 + e];
+        sincospif(2.0f * static_cast<float>(x - rint(x)), &s[e], &c[e]);
+      }
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int h = h0 + 4 * i;
+        if (h >= heads) break;
+        uint32_t* lw = reinterpret_cast<uint32_t*>(&lo[i]);
+        uint32_t* hw = reinterpret_cast<uint32_t*>(&hi[i]);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float2 a = __bfloat1622float2(*reinterpret_cast<__nv_bfloat162*>(&lw[e]));
+          const float2 b = __bfloat1622float2(*reinterpret_cast<__nv_bfloat162*>(&hw[e]));
+          const int k = 2 * e;
+          lw[e] = pack_bf16x2(fmaf(a.x, c[k], -b.x * s[k]), fmaf(a.y, c[k + 1], -b.y * s[k + 1]));
+          hw[e] = pack_bf16x2(fmaf(b.x, c[k], a.x * s[k]), fmaf(b.y, c[k + 1], a.y * s[k + 1]));
+        }
+        *reinterpret_cast<uint4*>(r + h * kHeadDim + j0) = lo[i];
+        *reinterpret_cast<uint4*>(r + h * kHeadDim + 64 + j0) = hi[i];
+      }
     }
+    if (p < 0 && lane == 0) record_status(status, CER_DEV_INDEX);
   }
 }
 
