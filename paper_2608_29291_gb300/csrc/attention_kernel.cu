@@ -14,22 +14,20 @@
 //
 // packed_attention_kernel: persistent, one CTA per SM, one work item per
 // (query tile of 128 packed tokens, sequence, query head), the tiles with the
-// most key blocks first.  192 threads:
-//   warp 0     TMA: the Q tile once per item (two 64-column boxes, K-major)
-//              and, per key block of 128 tokens, K (K-major, a three-slot
-//              ring freed as soon as S is computed) and V (four 64 x 64
-//              MN-major atoms, a two-slot ring), each K one block ahead of
-//              its V;
-//   warp 1     allocates TMEM (two S buffers of 128 columns, O of 128) and
-//              issues tcgen05.mma: S_j = Q K_j^T into S[j % 2] -- issued one
-//              block ahead, so it overlaps the softmax of block j - 1 -- and
-//              O += P_j V_j once the softmax has written P_j;
-//   warps 2-5  softmax, one query row per thread (its TMEM lane), the whole
-//              S row in one 128-column TMEM load: masked row maximum in the
-//              log2 domain, kept until a block's exceeds it by more than 8,
-//              so O is rescaled in TMEM rarely; P_j = exp2(s - m) written as
-//              bf16 into a 128-byte-swizzled tile (the A operand of P V), the
-//              running sum kept in fp32; at the end O / l goes out as bf16.
+// most key blocks first.  352 threads:
+//   warp 0     TMA: the Q tile once per item and K blocks of 128 keys
+//              (K-major, a three-slot ring), streaming ahead of V;
+//   warp 10    TMA: V blocks (two MN-major 64 x 128 boxes, a two-slot ring);
+//   warp 1     allocates TMEM (three S buffers of 128 columns, O of 128) and
+//              issues tcgen05.mma: S_j = Q K_j^T two blocks ahead of the
+//              softmax, and O += P_j V_j with P_j read from tensor memory;
+//   warps 2-9  softmax, two warps per TMEM lane quadrant splitting the key
+//              columns: masked row maximum in the log2 domain (exchanged
+//              between the two halves through shared memory), kept until a
+//              block's exceeds it by more than 8, so O is rescaled rarely;
+//              P_j = exp2(s - m) packed to bf16 over the S buffer it came
+//              from, the running sum kept in fp32; at the end O / l goes
+//              out as bf16.
 // Every wait is bounded like the GEMM skeleton's (umma_gemm.cuh).
 #include <cuda_bf16.h>
 
@@ -116,38 +114,41 @@ cudaError_t launch_rope(__nv_bfloat16* qkv, long long rows, int Hq, int Hkv, con
 // ------------------------------------------------------------------ attention
 
 struct AttnParams {
-  CUtensorMap tm_qk;   // qkv, box 64 x 128 (Q and K tiles)
-  CUtensorMap tm_v;    // qkv, box 64 x 64 (V atoms)
+  CUtensorMap tm_qkv;  // qkv, box 64 columns x 128 rows (Q, K and V tiles)
   __nv_bfloat16* out;  // [B * L, Hq * 128]
   int* status;
-  int B, L, Hq, Hkv, causal, n_qt, n_items;
+  int B, L, Hq, Hkv, causal, group, n_qt, n_items;
   float scale_log2;    // log2(e) / sqrt(128)
 };
 
-constexpr int kAttnThreads = 192;
+constexpr int kAttnThreads = 352;                 // Q/K producer, MMA, eight softmax warps, V producer
 constexpr uint32_t kBox = 128 * 128;              // 128 rows x 64 bf16
-constexpr uint32_t kQBytes = 2 * kBox;            // Q tile: 128 tokens x 128
-constexpr uint32_t kKBytes = 2 * kBox;            // K tile: 128 keys x 128 (two K-major boxes)
-constexpr uint32_t kVBytes = 2 * kBox;            // V tile: four 64 x 64 MN-major atoms
-constexpr uint32_t kPBytes = 2 * kBox;            // P tile: 128 queries x 128 keys, bf16
-constexpr int kKSlots = 3;                        // K is freed as soon as S is computed: one block more in flight
+constexpr uint32_t kQBytes = 2 * kBox;            // Q tile: 128 tokens x 128 (two K-major boxes)
+constexpr uint32_t kKBytes = 2 * kBox;            // K block: 128 keys x 128 (two K-major boxes)
+constexpr uint32_t kVBytes = 2 * kBox;            // V block: two MN-major boxes (dims 0-63, 64-127) of 128 keys
+constexpr int kKSlots = 3;
 constexpr int kVSlots = 2;
-constexpr size_t kAttnSmem = 1024 + kQBytes + kKSlots * kKBytes + kVSlots * kVBytes + kPBytes + 256;
+constexpr int kSBufs = 3;                         // S buffers in tensor memory
+constexpr uint32_t kXchBytes = 2 * 2 * 128 * 4;   // row-maximum exchange: [parity][half][row]
+constexpr size_t kAttnSmem = 1024 + kQBytes + kKSlots * kKBytes + kVSlots * kVBytes + kXchBytes + 512;
 constexpr uint32_t kIdescS = idesc_bf16(128, 128, 0);    // Q (K-major) x K (K-major)
-constexpr uint32_t kIdescPV = idesc_bf16(128, 128, 1);   // P (K-major) x V (MN-major)
+constexpr uint32_t kIdescPV = idesc_bf16(128, 128, 1);   // P (tensor memory) x V (MN-major)
 
+// A work item: one 128-query tile of one sequence and query head.
 struct AttnItem {
   int b, h, kh, qt, n_kv;
 };
 
+// Tiles with the most key blocks first; a key/value head's query heads on
+// neighbouring items, so their K and V blocks are read from L2.
 __device__ __forceinline__ AttnItem attn_item(const AttnParams& p, int item) {
   AttnItem it;
   const int per_tile = p.B * p.Hq;
-  it.qt = p.n_qt - 1 - item / per_tile;   // the tiles with the most key blocks first
+  it.qt = p.n_qt - 1 - item / per_tile;
   const int rest = item % per_tile;
   it.b = rest / p.Hq;
   it.h = rest % p.Hq;
-  it.kh = it.h / (p.Hq / p.Hkv);
+  it.kh = it.h / p.group;
   it.n_kv = p.causal ? it.qt + 1 : p.n_qt;
   return it;
 }
@@ -160,34 +161,67 @@ __device__ __forceinline__ float exp2_fast(float x) {
   return y;
 }
 
+// 32 lanes x 64 columns of fp32 in one load, the wait in the same asm statement.
+__device__ __forceinline__ void tmem_ld_32x32_x64(uint32_t taddr, uint32_t (&r)[64]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x64.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+      "%15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32, %33, %34, %35, "
+      "%36, %37, %38, %39, %40, %41, %42, %43, %44, %45, %46, %47, %48, %49, %50, %51, %52, %53, %54, %55, %56, "
+      "%57, %58, %59, %60, %61, %62, %63}, [%64];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]),
+        "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]), "=r"(r[37]), "=r"(r[38]), "=r"(r[39]),
+        "=r"(r[40]), "=r"(r[41]), "=r"(r[42]), "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]),
+        "=r"(r[48]), "=r"(r[49]), "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]), "=r"(r[55]),
+        "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]), "=r"(r[61]), "=r"(r[62]), "=r"(r[63])
+      : "r"(taddr)
+      : "memory");
+}
+
+// Tensor memory, 512 columns: three S buffers at [0,128), [128,256),
+// [256,384) and O at [384,512).  Key blocks, counted over all of a CTA's
+// items (gb), rotate through the S buffers; P(gb) (bf16, two keys per
+// column) overwrites the first 64 columns of S(gb)'s buffer once the softmax
+// has read S(gb), and is the A operand of O += P(gb) V.  S(gb + 3) reuses the
+// buffer after that product has completed -- by then long done, as S(gb + 3)
+// is issued after P(gb + 1) V.  So the MMA warp issues P(j) V and S(j + 2)
+// back to back as soon as P(j) is written, and S(j + 1) and S(j + 2) are
+// computed while the softmax works on block j.
+//
+// Softmax: warps 2-9, two per TMEM lane quadrant: warp half hf takes key
+// columns [64 hf, 64 hf + 64) of its 32 query rows.  The two halves exchange
+// their row maxima through shared memory once per block (an mbarrier of two
+// arrivals per quadrant, bounded like every wait) and their row sums once
+// per item.
 __global__ void __launch_bounds__(kAttnThreads, 1) packed_attention_kernel(const __grid_constant__ AttnParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* q_tile = smem;
   uint8_t* k_ring = q_tile + kQBytes;
-  uint8_t* v_ring = k_ring + kKSlots * kKBytes;   // slot s: atom (key half kh, dim half na) at kh*16K + na*8K
-  uint8_t* p_tile = v_ring + kVSlots * kVBytes;
-  uint64_t* q_full = reinterpret_cast<uint64_t*>(p_tile + kPBytes);
+  uint8_t* v_ring = k_ring + kKSlots * kKBytes;   // slot s: dims 64 na .. 64 na + 63 of 128 keys at na*16K
+  float* xch_val = reinterpret_cast<float*>(v_ring + kVSlots * kVBytes);   // [parity][half][row]
+  uint64_t* q_full = reinterpret_cast<uint64_t*>(reinterpret_cast<uint8_t*>(xch_val) + kXchBytes);
   uint64_t* q_empty = q_full + 1;
   uint64_t* k_full = q_empty + 1;          // [kKSlots]
   uint64_t* k_empty = k_full + kKSlots;    // [kKSlots]
   uint64_t* v_full = k_empty + kKSlots;    // [kVSlots]
   uint64_t* v_empty = v_full + kVSlots;    // [kVSlots]
-  uint64_t* s_full = v_empty + kVSlots;    // [2]
-  uint64_t* s_free = s_full + 2;           // [2]
-  uint64_t* p_full = s_free + 2;
-  uint64_t* o_done = p_full + 1;
+  uint64_t* s_full = v_empty + kVSlots;    // [kSBufs]
+  uint64_t* p_full = s_full + kSBufs;      // [kSBufs]
+  uint64_t* pv_done = p_full + kSBufs;     // [kSBufs]: P(gb) V complete
+  uint64_t* o_done = pv_done + kSBufs;     // an item's last P V product
   uint64_t* o_free = o_done + 1;
-  uint64_t* drain = o_free + 1;
+  uint64_t* xch = o_free + 1;              // [4]: per lane quadrant
+  uint64_t* drain = xch + 4;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  if (threadIdx.x == 32) {
-    tma_prefetch_desc(&p.tm_qk);
-    tma_prefetch_desc(&p.tm_v);
-  }
+  if (threadIdx.x == 32) tma_prefetch_desc(&p.tm_qkv);
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
     mbar_init(q_empty, 1);
@@ -199,13 +233,14 @@ __global__ void __launch_bounds__(kAttnThreads, 1) packed_attention_kernel(const
       mbar_init(&v_full[s], 1);
       mbar_init(&v_empty[s], 1);
     }
-    for (int s = 0; s < 2; ++s) {
-      mbar_init(&s_full[s], 1);
-      mbar_init(&s_free[s], 4);   // one arrival per softmax warp
+    for (int i = 0; i < kSBufs; ++i) {
+      mbar_init(&s_full[i], 1);
+      mbar_init(&p_full[i], 8);   // one arrival per softmax warp
+      mbar_init(&pv_done[i], 1);
     }
-    mbar_init(p_full, 4);
     mbar_init(o_done, 1);
-    mbar_init(o_free, 4);
+    mbar_init(o_free, 8);
+    for (int i = 0; i < 4; ++i) mbar_init(&xch[i], 2);
     mbar_init(drain, 1);
     *abort_flag = 0;
     fence_mbar_init();
@@ -222,28 +257,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1) packed_attention_kernel(const
   griddep_launch_dependents();
 
   if (warp == 0) {
-    // ---------------------------------------------------------------- producer
-    // Key block j's K goes out one block ahead of its V: K_j, then V_{j-1}
-    // (carried across items), so the keys for S_{j+1} are in flight while
-    // P_j V_j waits.
-    uint32_t gk = 0, gv = 0, items = 0;
+    // ---------------------------------------------------------------- Q and K producer
+    // K streams ahead, limited only by its own ring: S(j) needs just K_j.
+    uint32_t gk = 0, items = 0;
     bool ok = true;
-    bool pend = false;
-    int pend_row = 0, pend_col = 0;
-    auto load_v = [&](int row, int col) -> bool {
-      const uint32_t s = gv % kVSlots;
-      if (!warp_wait(&v_empty[s], ((gv / kVSlots) & 1) ^ 1, abort_flag, p.status)) return false;
-      if (lane == 0) {
-        uint8_t* slot = v_ring + s * kVBytes;
-        mbar_arrive_expect_tx(&v_full[s], kVBytes);
-        for (int kh = 0; kh < 2; ++kh)
-          for (int na = 0; na < 2; ++na)
-            tma_load_2d(slot + kh * 16384 + na * 8192, &p.tm_v, &v_full[s], col + na * 64, row + kh * 64);
-      }
-      __syncwarp();
-      ++gv;
-      return true;
-    };
     for (int item = blockIdx.x; item < p.n_items && ok; item += gridDim.x, ++items) {
       const AttnItem it = attn_item(p, item);
       const int row0 = it.b * p.L;
@@ -252,234 +269,301 @@ __global__ void __launch_bounds__(kAttnThreads, 1) packed_attention_kernel(const
         break;
       }
       if (lane == 0) {
+        const int qrow = row0 + it.qt * 128;
         mbar_arrive_expect_tx(q_full, kQBytes);
-        tma_load_2d(q_tile, &p.tm_qk, q_full, it.h * kHeadDim, row0 + it.qt * 128);
-        tma_load_2d(q_tile + kBox, &p.tm_qk, q_full, it.h * kHeadDim + 64, row0 + it.qt * 128);
+        tma_load_2d(q_tile, &p.tm_qkv, q_full, it.h * kHeadDim, qrow);
+        tma_load_2d(q_tile + kBox, &p.tm_qkv, q_full, it.h * kHeadDim + 64, qrow);
       }
       __syncwarp();
       const int kcol = (p.Hq + it.kh) * kHeadDim;
-      const int vcol = (p.Hq + p.Hkv + it.kh) * kHeadDim;
-      for (int j = 0; j < it.n_kv; ++j) {
-        const uint32_t s = gk % kKSlots;
-        if (!warp_wait(&k_empty[s], ((gk / kKSlots) & 1) ^ 1, abort_flag, p.status)) {
+      for (int j = 0; j < it.n_kv && ok; ++j) {
+        const uint32_t ks = gk % kKSlots;
+        if (!warp_wait(&k_empty[ks], ((gk / kKSlots) & 1) ^ 1, abort_flag, p.status)) {
           ok = false;
           break;
         }
         if (lane == 0) {
-          uint8_t* slot = k_ring + s * kKBytes;
-          mbar_arrive_expect_tx(&k_full[s], kKBytes);
-          tma_load_2d(slot, &p.tm_qk, &k_full[s], kcol, row0 + j * 128);
-          tma_load_2d(slot + kBox, &p.tm_qk, &k_full[s], kcol + 64, row0 + j * 128);
+          uint8_t* slot = k_ring + ks * kKBytes;
+          mbar_arrive_expect_tx(&k_full[ks], kKBytes);
+          tma_load_2d(slot, &p.tm_qkv, &k_full[ks], kcol, row0 + j * 128);
+          tma_load_2d(slot + kBox, &p.tm_qkv, &k_full[ks], kcol + 64, row0 + j * 128);
         }
         __syncwarp();
         ++gk;
-        if (pend && !load_v(pend_row, pend_col)) {
-          ok = false;
-          break;
-        }
-        pend = true;
-        pend_row = row0 + j * 128;
-        pend_col = vcol;
       }
     }
-    if (ok && pend) ok = load_v(pend_row, pend_col);
     if (!ok && lane == 0) unwind_pause(1000000ull);
-  } else if (warp == 1) {
-    // ---------------------------------------------------------------- MMA issuer
-    uint32_t gk = 0, gv = 0;   // K / V blocks consumed
-    uint32_t cs = 0;           // S tiles issued (buffer cs % 2)
-    uint32_t cp = 0;           // P tiles consumed
-    uint32_t items = 0;
+  } else if (warp == 10) {
+    // ---------------------------------------------------------------- V producer
+    uint32_t gv = 0;
     bool ok = true;
-    bool issued_any = false;
-    const uint32_t q_base = smem_u32(q_tile), p_base = smem_u32(p_tile);
-    const uint32_t o_tm = tmem_base + 256;
-    for (int item = blockIdx.x; item < p.n_items && ok; item += gridDim.x, ++items) {
+    for (int item = blockIdx.x; item < p.n_items && ok; item += gridDim.x) {
       const AttnItem it = attn_item(p, item);
-      if (!warp_wait(q_full, items & 1, abort_flag, p.status)) {
-        ok = false;
-        break;
-      }
-      tc_fence_after();
-      for (int j = -1; j < it.n_kv && ok; ++j) {
-        // S_{j+1} = Q K_{j+1}^T, one block ahead of P_j V_j.
-        if (j + 1 < it.n_kv) {
-          const uint32_t ks = gk % kKSlots;
-          const uint32_t buf = cs & 1;
-          if (!warp_wait(&k_full[ks], (gk / kKSlots) & 1, abort_flag, p.status) ||
-              !warp_wait(&s_free[buf], ((cs >> 1) & 1) ^ 1, abort_flag, p.status)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          if (lane == 0) {
-            const uint32_t k_base = smem_u32(k_ring + ks * kKBytes);
-#pragma unroll
-            for (int k = 0; k < 8; ++k) {
-              const uint32_t off = (k >> 2) * kBox + (k & 3) * 32;
-              umma_bf16(tmem_base + buf * 128, sdesc_kmajor_sw128(q_base + off), sdesc_kmajor_sw128(k_base + off),
-                        kIdescS, k > 0 ? 1u : 0u);
-            }
-            umma_commit(&s_full[buf]);
-            umma_commit(&k_empty[ks]);
-            if (j + 2 == it.n_kv) umma_commit(q_empty);   // the item's last S: the Q tile may be reloaded
-            issued_any = true;
-          }
-          __syncwarp();
-          ++gk;
-          ++cs;
-        }
-        if (j < 0) continue;
-        // O += P_j V_j once the softmax has written P_j (and, for the item's
-        // first block, has read out the previous item's O).
-        if (!warp_wait(p_full, cp & 1, abort_flag, p.status)) {
-          ok = false;
-          break;
-        }
-        ++cp;
+      const int row0 = it.b * p.L;
+      const int vcol = (p.Hq + p.Hkv + it.kh) * kHeadDim;
+      for (int j = 0; j < it.n_kv && ok; ++j) {
         const uint32_t vs = gv % kVSlots;
-        if ((j == 0 && !warp_wait(o_free, (items & 1) ^ 1, abort_flag, p.status)) ||
-            !warp_wait(&v_full[vs], (gv / kVSlots) & 1, abort_flag, p.status)) {
+        if (!warp_wait(&v_empty[vs], ((gv / kVSlots) & 1) ^ 1, abort_flag, p.status)) {
           ok = false;
           break;
         }
-        tc_fence_after();
         if (lane == 0) {
-          const uint32_t v_base = smem_u32(v_ring + vs * kVBytes);
-#pragma unroll
-          for (int k = 0; k < 8; ++k) {
-            const uint64_t adesc = sdesc_kmajor_sw128(p_base + (k >> 2) * kBox + (k & 3) * 32);
-            const uint64_t bdesc = sdesc_mnmajor_sw128(v_base + (k >> 2) * 16384 + (k & 3) * 2048, 8192, 1024);
-            umma_bf16(o_tm, adesc, bdesc, kIdescPV, (j > 0 || k > 0) ? 1u : 0u);
-          }
-          umma_commit(&v_empty[vs]);
-          umma_commit(o_done);
+          uint8_t* slot = v_ring + vs * kVBytes;
+          mbar_arrive_expect_tx(&v_full[vs], kVBytes);
+          tma_load_2d(slot, &p.tm_qkv, &v_full[vs], vcol, row0 + j * 128);
+          tma_load_2d(slot + kBox, &p.tm_qkv, &v_full[vs], vcol + 64, row0 + j * 128);
         }
         __syncwarp();
         ++gv;
       }
     }
+    if (!ok && lane == 0) unwind_pause(1000000ull);
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA issuer
+    // Per item: S(0), S(1); then per key block j: S(j + 2), P(j) V_j.
+    uint32_t gk = 0, gv = 0, items = 0, g = 0, o_taken = 0;
+    bool ok = true;
+    bool issued_any = false;
+    // S(gb) = Q K^T from K slot ks, once P(gb - 3) V (the buffer's previous
+    // reader) has completed.  That wait cannot meet a barrier two phases
+    // ahead: P(gb) V needs S(gb).
+    auto issue_s = [&](uint32_t ks, uint32_t gb) -> bool {
+      const uint32_t buf = gb % kSBufs;
+      if (gb >= kSBufs &&
+          !warp_wait(&pv_done[buf], ((gb - kSBufs) / kSBufs) & 1, abort_flag, p.status))
+        return false;
+      tc_fence_after();
+      if (lane == 0) {
+        const uint32_t q_base = smem_u32(q_tile);
+        const uint32_t k_base = smem_u32(k_ring + ks * kKBytes);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          const uint32_t off = (k >> 2) * kBox + (k & 3) * 32;
+          umma_bf16(tmem_base + buf * 128, sdesc_kmajor_sw128(q_base + off), sdesc_kmajor_sw128(k_base + off),
+                    kIdescS, k > 0 ? 1u : 0u);
+        }
+        umma_commit(&s_full[buf]);
+        issued_any = true;
+      }
+      __syncwarp();
+      return true;
+    };
+    // O (+)= P(gb) V from V slot vs; first: the item's first block (also waits
+    // until the previous item's O has been read out); last: its last block.
+    auto issue_pv = [&](uint32_t vs, uint32_t gb, bool first, bool last) -> bool {
+      const uint32_t buf = gb % kSBufs;
+      if (!warp_wait(&p_full[buf], (gb / kSBufs) & 1, abort_flag, p.status)) return false;
+      if (first) {
+        if (!warp_wait(o_free, (o_taken & 1) ^ 1, abort_flag, p.status)) return false;
+        ++o_taken;
+      }
+      tc_fence_after();
+      if (lane == 0) {
+        const uint32_t v_base = smem_u32(v_ring + vs * kVBytes);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          const uint64_t bdesc = sdesc_mnmajor_sw128(v_base + k * 2048, kBox, 1024);
+          umma_bf16_tmem_a(tmem_base + 384, tmem_base + buf * 128 + k * 8, bdesc, kIdescPV,
+                           (!first || k > 0) ? 1u : 0u);
+        }
+        umma_commit(&pv_done[buf]);
+        if (last) umma_commit(o_done);
+        issued_any = true;
+      }
+      __syncwarp();
+      return true;
+    };
+    for (int item = blockIdx.x; item < p.n_items && ok; item += gridDim.x, ++items) {
+      const AttnItem it = attn_item(p, item);
+      const int n = it.n_kv;
+      if (!warp_wait(q_full, items & 1, abort_flag, p.status)) {
+        ok = false;
+        break;
+      }
+      for (int j = 0; j < 2 && j < n; ++j) {
+        const uint32_t ks = gk % kKSlots;
+        if (!warp_wait(&k_full[ks], (gk / kKSlots) & 1, abort_flag, p.status) || !issue_s(ks, g + j)) {
+          ok = false;
+          break;
+        }
+        if (lane == 0) {
+          umma_commit(&k_empty[ks]);
+          if (j + 1 == n) umma_commit(q_empty);
+        }
+        __syncwarp();
+        ++gk;
+      }
+      for (int j = 0; j < n && ok; ++j) {
+        // S(j + 2) first: it needs only K and P(j - 1) V, so it runs while
+        // the softmax still works on block j.
+        if (j + 2 < n) {
+          const uint32_t ks = gk % kKSlots;
+          if (!warp_wait(&k_full[ks], (gk / kKSlots) & 1, abort_flag, p.status) || !issue_s(ks, g + j + 2)) {
+            ok = false;
+            break;
+          }
+          if (lane == 0) {
+            umma_commit(&k_empty[ks]);
+            if (j + 3 == n) umma_commit(q_empty);
+          }
+          __syncwarp();
+          ++gk;
+        }
+        const uint32_t vs = gv % kVSlots;
+        if (!warp_wait(&v_full[vs], (gv / kVSlots) & 1, abort_flag, p.status) ||
+            !issue_pv(vs, g + j, j == 0, j + 1 == n)) {
+          ok = false;
+          break;
+        }
+        if (lane == 0) umma_commit(&v_empty[vs]);
+        __syncwarp();
+        ++gv;
+      }
+      g += n;
+    }
     if (!ok && lane == 0 && issued_any) {
       umma_commit(drain);
       drain_wait(drain, 0);
     }
-  } else {
+  } else if (warp < 10) {
     // ---------------------------------------------------------------- softmax
     const int qd = warp & 3;            // TMEM lane quadrant
+    const int hf = (warp - 2) >> 2;     // key-column half
     const int r = qd * 32 + lane;       // query row of the tile
-    const uint32_t lane_off = static_cast<uint32_t>(qd * 32) << 16;
-    const uint32_t o_tm = tmem_base + lane_off + 256;
+    const uint32_t row_tm = tmem_base + (static_cast<uint32_t>(qd * 32) << 16);
+    const uint32_t o_tm = row_tm + 384 + hf * 64;
     const float sc = p.scale_log2;
-    uint32_t cs = 0, co = 0, items = 0;
+    uint32_t g = 0, done = 0, xp = 0;   // key blocks, items, exchanges so far
     bool ok = true;
-    for (int item = blockIdx.x; item < p.n_items && ok; item += gridDim.x, ++items) {
+    // Swap a value with the other half's warp of this quadrant.
+    auto exchange = [&](float v, float& other) -> bool {
+      float* slot = xch_val + (xp & 1) * 256;
+      slot[hf * 128 + r] = v;
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&xch[qd]);
+      if (!warp_wait(&xch[qd], xp & 1, abort_flag, p.status)) return false;
+      tc_fence_after();
+      other = slot[(hf ^ 1) * 128 + r];
+      ++xp;
+      return true;
+    };
+    for (int item = blockIdx.x; item < p.n_items && ok; item += gridDim.x) {
       const AttnItem it = attn_item(p, item);
       const int qi = it.qt * 128 + r;
       // Keys past the sequence, and (causal) past the query, are masked.
       const int lim = p.causal ? (qi + 1 < p.L ? qi + 1 : p.L) : p.L;
       float m = -INFINITY, l = 0.f;
-      for (int j = 0; j < it.n_kv; ++j, ++cs) {
-        const uint32_t buf = cs & 1;
-        if (!warp_wait(&s_full[buf], (cs >> 1) & 1, abort_flag, p.status)) {
+      for (int j = 0; j < it.n_kv; ++j) {
+        const uint32_t gb = g + j, buf = gb % kSBufs;
+        if (!warp_wait(&s_full[buf], (gb / kSBufs) & 1, abort_flag, p.status)) {
           ok = false;
           break;
         }
         tc_fence_after();
-        const int n_ok = lim - j * 128;   // admissible keys of this block: [0, n_ok)
-        uint32_t sv[128];
-        tmem_ld_32x32_x128(tmem_base + lane_off + buf * 128, sv);   // the whole S row
+        const int n_ok = lim - j * 128 - hf * 64;   // admissible keys of this half: [0, n_ok)
+        uint32_t sv[64];
+        tmem_ld_32x32_x64(row_tm + buf * 128 + hf * 64, sv);
         float mx8[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) mx8[e] = -INFINITY;
-        if (n_ok >= 128) {
+        if (n_ok >= 64) {
 #pragma unroll
-          for (int e = 0; e < 128; ++e) mx8[e & 7] = fmaxf(mx8[e & 7], __uint_as_float(sv[e]));
+          for (int e = 0; e < 64; ++e) mx8[e & 7] = fmaxf(mx8[e & 7], __uint_as_float(sv[e]));
         } else {
 #pragma unroll
-          for (int e = 0; e < 128; ++e)
+          for (int e = 0; e < 64; ++e)
             if (e < n_ok) mx8[e & 7] = fmaxf(mx8[e & 7], __uint_as_float(sv[e]));
         }
-        const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                               fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+        float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                         fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
+        // Both halves have read their S columns before either writes P over them.
+        float mx_other;
+        if (!exchange(mx, mx_other)) {
+          ok = false;
+          break;
+        }
+        mx = fmaxf(mx, mx_other);
         // The running maximum moves only when the block's exceeds it by more
         // than 8 (log2 units): with a stale maximum the weights stay below
         // 2^8, far inside bf16 and fp32, and O is rescaled rarely.  The
-        // result is unchanged: O and l share the same shift.
+        // result is unchanged: O and l share the same shift.  A block with no
+        // admissible key (mx = -inf) leaves it where it is.
         const float mb = mx * sc;
         const float m_new = (mb > m + 8.0f) ? mb : m;   // the first block always takes its maximum
         const float alpha = exp2_fast(m - m_new);       // 0 for the first block, else 1 or < 2^-8
-        if (j > 0) {
-          // P_{j-1} V_{j-1} is complete: the P tile is free and O may be rescaled.
-          if (!warp_wait(o_done, co & 1, abort_flag, p.status)) {
-            ok = false;
-            break;
-          }
-          ++co;
-          tc_fence_after();
-          if (__any_sync(0xffffffffu, alpha != 1.0f)) {
-#pragma unroll 1
-            for (int c = 0; c < 4; ++c) {
-              float ov[32];
-              tmem_ld_32x32(o_tm + c * 32, ov);
-#pragma unroll
-              for (int e = 0; e < 32; ++e) ov[e] *= alpha;
-              tmem_st_32x32(o_tm + c * 32, ov);
-            }
-          }
-        }
-        // P = exp2(s * scale - m) as bf16 into the swizzled A tile of P V.
+        // P = exp2(s * scale - m), packed to bf16 pairs: this half's keys
+        // 64hf + 32hh + (0..31) go to buffer columns 32hf + 16hh + (0..15).
         const float neg = -m_new;
         float rs4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-        for (int c = 0; c < 16; ++c) {   // 16-byte chunks of 8 keys
-          uint32_t pk[4];
+        for (int hh = 0; hh < 2; ++hh) {
+          uint32_t pk[16];
 #pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const int k0 = 8 * c + 2 * e;
+          for (int e = 0; e < 16; ++e) {
+            const int k0 = hh * 32 + 2 * e;
             float p0 = exp2_fast(fmaf(__uint_as_float(sv[k0]), sc, neg));
             float p1 = exp2_fast(fmaf(__uint_as_float(sv[k0 + 1]), sc, neg));
-            if (n_ok < 128) {
+            if (n_ok < 64) {
               p0 = k0 < n_ok ? p0 : 0.f;
               p1 = k0 + 1 < n_ok ? p1 : 0.f;
             }
-            rs4[e] += p0 + p1;
+            rs4[e & 3] += p0 + p1;
             pk[e] = pack_bf16x2(p0, p1);
           }
-          const int chunk = (c & 7) ^ (r & 7);   // 128-byte swizzle within each 64-key box
-          *reinterpret_cast<uint4*>(p_tile + (c >> 3) * kBox + r * 128 + chunk * 16) =
-              make_uint4(pk[0], pk[1], pk[2], pk[3]);
+          tmem_st_32x32_x16_nowait(row_tm + buf * 128 + hf * 32 + hh * 16, pk);
         }
+        // Rescale this half's O columns when the maximum moved, once P(gb - 1)
+        // V has completed (it cannot be two phases ahead: P(gb + 2) V needs
+        // this warp's P(gb + 2)).
+        if (j > 0 && __any_sync(0xffffffffu, alpha != 1.0f)) {
+          const uint32_t pb = gb - 1;
+          if (!warp_wait(&pv_done[pb % kSBufs], (pb / kSBufs) & 1, abort_flag, p.status)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+#pragma unroll 1
+          for (int c = 0; c < 2; ++c) {
+            float ov[32];
+            tmem_ld_32x32(o_tm + c * 32, ov);
+#pragma unroll
+            for (int e = 0; e < 32; ++e) ov[e] *= alpha;
+            tmem_st_32x32(o_tm + c * 32, ov);
+          }
+        }
+        tmem_wait_st();
         tc_fence_before();
-        fence_proxy_async_smem();
         __syncwarp();
-        if (lane == 0) {
-          mbar_arrive(&s_free[buf]);
-          mbar_arrive(p_full);
-        }
+        if (lane == 0) mbar_arrive(&p_full[buf]);
         l = l * alpha + ((rs4[0] + rs4[1]) + (rs4[2] + rs4[3]));
         m = m_new;
       }
       if (!ok) break;
-      if (!warp_wait(o_done, co & 1, abort_flag, p.status)) {
+      g += it.n_kv;
+      float l_other;
+      if (!exchange(l, l_other) || !warp_wait(o_done, done & 1, abort_flag, p.status)) {
         ok = false;
         break;
       }
-      ++co;
+      ++done;
       tc_fence_after();
-      const float inv = 1.0f / l;
-      uint32_t ov[128];
-      tmem_ld_32x32_x128(o_tm, ov);
-      if (qi < p.L) {
-        uint4* d4 = reinterpret_cast<uint4*>(p.out + (static_cast<size_t>(it.b) * p.L + qi) *
-                                                         (static_cast<size_t>(p.Hq) * kHeadDim) +
-                                             static_cast<size_t>(it.h) * kHeadDim);
+      const float inv = 1.0f / (hf == 0 ? l + l_other : l_other + l);
+#pragma unroll 1
+      for (int c = 0; c < 2; ++c) {
+        float ov[32];
+        tmem_ld_32x32(o_tm + c * 32, ov);
+        if (qi < p.L) {
+          uint4* d4 = reinterpret_cast<uint4*>(p.out + (static_cast<size_t>(it.b) * p.L + qi) *
+                                                           (static_cast<size_t>(p.Hq) * kHeadDim) +
+                                               static_cast<size_t>(it.h) * kHeadDim + hf * 64 + c * 32);
 #pragma unroll
-        for (int q = 0; q < 16; ++q) {
-          uint32_t pk[4];
+          for (int q = 0; q < 4; ++q) {
+            uint32_t w4[4];
 #pragma unroll
-          for (int e = 0; e < 4; ++e)
-            pk[e] = pack_bf16x2(__uint_as_float(ov[8 * q + 2 * e]) * inv, __uint_as_float(ov[8 * q + 2 * e + 1]) * inv);
-          d4[q] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+            for (int e = 0; e < 4; ++e) w4[e] = pack_bf16x2(ov[8 * q + 2 * e] * inv, ov[8 * q + 2 * e + 1] * inv);
+            d4[q] = make_uint4(w4[0], w4[1], w4[2], w4[3]);
+          }
         }
       }
       tc_fence_before();
@@ -502,8 +586,7 @@ cudaError_t launch_packed_attention(const __nv_bfloat16* qkv, int B, int L, int 
   AttnParams p{};
   const uint64_t rows = static_cast<uint64_t>(B) * L;
   const uint64_t width = static_cast<uint64_t>(Hq + 2 * Hkv) * kHeadDim;
-  if (!encode_bf16_2d(&p.tm_qk, qkv, rows, width, 64, 128)) return cudaErrorInvalidValue;
-  if (!encode_bf16_2d(&p.tm_v, qkv, rows, width, 64, 64)) return cudaErrorInvalidValue;
+  if (!encode_bf16_2d(&p.tm_qkv, qkv, rows, width, 64, 128)) return cudaErrorInvalidValue;
   p.out = out;
   p.status = status;
   p.B = B;
@@ -511,6 +594,7 @@ cudaError_t launch_packed_attention(const __nv_bfloat16* qkv, int B, int L, int 
   p.Hq = Hq;
   p.Hkv = Hkv;
   p.causal = causal;
+  p.group = Hq / Hkv;
   p.n_qt = (L + 127) / 128;
   p.n_items = B * Hq * p.n_qt;
   p.scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(kHeadDim));
