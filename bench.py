@@ -556,6 +556,100 @@ def run_gpu(args, info):
     return 0
 
 
+SWEEP_POINTS = [(n, r, f) for n in (1024, 4096, 16384) for r in (0.1, 0.5, 0.9) for f in (0.25, 1.0)]
+
+
+def run_sweep(args):
+    """The 7B sweep (B = 1, N in 1K..16K, all routable, generation): one JSON
+    line per (N, token keep ratio, channel keep ratio) point with the whole
+    step time and the FFN stages against their own bound -- the weight stream
+    from HBM for small M, the tensor pipe for large M (the FFN's arithmetic
+    intensity is about M flop per byte)."""
+    import torch
+    from paper_2608_29291_gb300 import cer
+
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    cer.load()
+    peaks, peak_kind = load_peaks()
+    peak_tf = float(peaks["bf16_tflops"])
+    peak_gbs = float(peaks["hbm_gbs"])
+
+    def bf(bits):
+        return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).to(dev)
+
+    def f32(a):
+        return None if a is None else torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(dev)
+
+    base = gen.make_inputs(gen.sweep(max(n for n, _, _ in SWEEP_POINTS), 0.5, 1.0))
+    ffn = (base["Wg"], base["Wu"], base["WdT"])
+    Wg_full, Wu_full, WdT_full = bf(ffn[0]), bf(ffn[1]), bf(ffn[2])
+    flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    for n, r, f in SWEEP_POINTS:
+        w = gen.sweep(n, r, f)
+        inp = gen.make_inputs(w, ffn_weights=ffn)
+        core = cer.Scorer(W1=bf(inp["W1"]), w2=f32(inp["w2"]), b1=f32(inp.get("b1")))
+        exp = cer.Scorer(W1=bf(inp["W1e"]), w2=f32(inp["w2e"]), U=bf(inp["Ue"]) if inp.get("Ue") is not None else None)
+        h = bf(inp["h"])
+        h0 = h.clone()
+        t = f32(inp["t"])
+        if w.C < w.I:
+            Wg, Wu, WdT = cer.pack_ffn_weights(Wg_full, Wu_full, WdT_full, torch.from_numpy(inp["chan"]).to(dev))
+        else:
+            Wg, Wu, WdT = Wg_full, Wu_full, WdT_full
+        ws = cer.workspace(cer.cer_routed_block_workspace_size(w.B, w.N, w.d, w.Hc, w.He, w.task, w.r0, w.r1, w.K,
+                                                               w.C, False), dev)
+
+        def step(stage_events=None):
+            cer.cer_routed_block(h, core, exp, t, w.task, w.r0, w.r1, w.K, Wg, Wu, WdT, None, ws=ws,
+                                 stage_events=stage_events, stream=stream)
+
+        def prepare(i):
+            h.copy_(h0)
+            flush.fill_(float(i))
+            torch.cuda._sleep(200000)
+
+        for i in range(args.warmup):
+            prepare(i)
+            step()
+        cer.cer_sync_status(stream)
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+        for i in range(args.steps):
+            prepare(i)
+            ev[i][0].record(stream)
+            step()
+            ev[i][1].record(stream)
+        torch.cuda.synchronize(dev)
+        step_ms = float(np.mean([a.elapsed_time(b) for a, b in ev]))
+        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(args.steps)]
+        for i in range(args.steps):
+            prepare(i)
+            step(evs[i])
+        torch.cuda.synchronize(dev)
+        cer.cer_sync_status(stream)
+        stage = np.array([[e[j].elapsed_time(e[j + 1]) for j in range(5)] for e in evs]).mean(axis=0)   # ms
+        M = w.B * (w.K + w.N - (w.r1 - w.r0))
+        ffn_s = (stage[3] + stage[4]) * 1e-3
+        flops = 6.0 * M * w.d * w.C
+        wbytes = 6.0 * w.d * w.C
+        t_tensor = flops / (peak_tf * 1e12)
+        t_hbm = (wbytes + 4.0 * M * w.d) / (peak_gbs * 1e9)
+        bound = "tensor" if t_tensor >= t_hbm else "hbm"
+        line = {"sweep_point": w.name, "N": w.N, "K": w.K, "M": M, "C": w.C, "ms_per_step": step_ms,
+                "tokens_per_s": w.B * w.N / (step_ms * 1e-3),
+                "stages_us": {k: round(v * 1e3, 2) for k, v in zip(("score", "topk", "gather", "ffn_gateup",
+                                                                     "ffn_down_scatter"), stage)},
+                "ffn_bound": bound, "ffn_tflops": flops / ffn_s / 1e12,
+                "ffn_weight_gbs": (wbytes + 4.0 * M * w.d) / ffn_s / 1e9,
+                "ffn_frac": (t_tensor if bound == "tensor" else t_hbm) / ffn_s,
+                "peak_source": f"bf16_tflops (burst) / hbm_gbs of {peak_kind}",
+                "steps": args.steps, "warmup": args.warmup, "l2": "flushed between timed steps"}
+        print(json.dumps(line), flush=True)
+        del h, h0, ws, Wg, Wu, WdT
+    return 0
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
@@ -565,10 +659,14 @@ def main(argv=None):
     ap.add_argument("--config", choices=sorted(gen.WORKLOADS), default="und_1p5b")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sweep", action="store_true",
+                    help="time the 7B sweep points (one JSON line each) instead of the bench line")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     info = runtime.rank_info()
+    if args.sweep:
+        return run_sweep(args)
     if args.impl == "reference":
         return run_reference(args, info)
     return run_gpu(args, info)

@@ -116,14 +116,18 @@ __host__ __device__ __forceinline__ long long sk_first_unit(long long U, int s, 
   return U * s / S;
 }
 
-// Host side: how a launch splits its tiles.  A split pays only where a last
-// wave would leave most slots idle: with every slot busy these contractions
-// are bound by L2 bandwidth (the K-block rate per slot drops as slots are
-// added), so a split elsewhere only adds partial traffic.  It applies when
-// the tiles fill at least one wave, the last wave is at most half full and
-// the contraction has at least 64 K blocks (the partial sums cost about as
-// much as a few K blocks): the last full wave and the remainder are split,
-// every run covering at least one tile (at most two contributors per tile).
+// Host side: how a launch splits its tiles.  With every slot busy these
+// contractions are bound by L2 bandwidth (the K-block rate per slot drops as
+// slots are added), so a split that keeps them all busy only adds partial
+// traffic.  Two cases pay:
+//   - a last wave that would leave most slots idle: when the tiles fill at
+//     least one wave, the last wave is at most half full and the contraction
+//     has at least 64 K blocks, the last full wave and the remainder are split,
+//     every run covering at least one tile (at most two contributors a tile);
+//   - fewer tiles than half the slots (a small M): every tile is split over up
+//     to four slots when each run keeps at least 8 K blocks, so the operands
+//     stream into four times as many SMs; runs are then shorter than a tile
+//     and a tile has up to four contributors.
 // (Splitting the scorer's short contractions was measured slower: the
 // owners' GELU epilogues then run on a quarter of the SMs.)
 struct SplitPlan {
@@ -131,12 +135,20 @@ struct SplitPlan {
   int dp_tiles;   // tiles handed out whole (== tiles: no split)
 };
 
+constexpr int kMaxSplit = 4;
+
 inline SplitPlan stream_k_plan(int tiles, int nkb, int slots) {
   const SplitPlan whole{tiles < slots ? tiles : slots, tiles};
-  if (slots <= 1 || nkb < 64) return whole;
+  if (slots <= 1 || tiles <= 0) return whole;
   const int q = tiles / slots;
   const int r = tiles % slots;
-  if (q == 0 || r == 0 || 2 * r > slots) return whole;
+  if (q == 0) {
+    if (2 * tiles > slots) return whole;
+    const int s = tiles * kMaxSplit < slots ? tiles * kMaxSplit : slots;
+    if (static_cast<long long>(tiles) * nkb < 8LL * s) return whole;
+    return SplitPlan{s, 0};
+  }
+  if (nkb < 64 || r == 0 || 2 * r > slots) return whole;
   return SplitPlan{slots, (q - 1) * slots};
 }
 

@@ -177,14 +177,16 @@ def test_score_matches_oracle(name):
 
 # ------------------------------------------------------------------ S4 FFN
 
-# (1000, 1792, ...) runs 28-32 pair tiles on all SM pairs; the last two
-# shapes split tiles by K block across SM pairs (stream-K): the down GEMM of
-# (2000, 2560, ...) and the gate/up GEMM of (256, 4096, ...), the second with
-# a ragged last row tile.
+# Stream-K splits (tiles cut by K block across slots, the owner adding the
+# others' partial sums): a last wave at most half full -- the down GEMM of
+# (2000, 2560, ...), the gate/up GEMM of (200, 4096, ...); fewer tiles than
+# half the slots, each tile over up to four slots -- the down GEMM of
+# (129, 1536, ...) and (200, 4096, ...), the gate/up GEMM of (1000, 1792, ...),
+# and both GEMMs of (100, 3584, ...) (one-CTA down tiles, ragged rows).
 @pytest.mark.parametrize("M,d,I,C,pruned", [(1, 256, 1024, 512, True), (127, 256, 1024, 512, True),
                                             (300, 512, 640, 640, False), (129, 1536, 8960, 6720, True),
                                             (1000, 1792, 1536, 960, True), (2000, 2560, 4096, 4096, False),
-                                            (200, 4096, 10240, 10240, False)])
+                                            (200, 4096, 10240, 10240, False), (100, 3584, 18944, 4736, True)])
 def test_routed_ffn_matches_oracle(M, d, I, C, pruned):
     rng = np.random.default_rng(M + d)
     X = gen.f32_to_bf16_bits(rng.normal(0, 1, (M, d)).astype(np.float32))
