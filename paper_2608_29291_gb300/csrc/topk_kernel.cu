@@ -5,11 +5,12 @@
 // One 1024-thread CTA per sequence keeps the N order-preserving 32-bit keys in
 // shared memory.  A four-pass MSB-first radix select (8-bit digits, shared
 // histograms) finds the K-th largest routable key T and how many tokens equal
-// to T must be taken; two block-wide scans in token order then give every
-// tie its rank (lowest index first) and every kept token its output slot, so
-// the kept list comes out in ascending token order with no sort.  When fed
-// the scorer's partial sums it also reduces them (in chunk order) into the
-// logits.
+// to T must be taken.  Each warp then owns a contiguous run of tokens, read 32
+// at a time (a token per lane, no bank conflicts): ballots rank every tie
+// (lowest index first) and every kept token, and two scans over the warps'
+// counts place them, so the kept list comes out in ascending token order with
+// no sort.  When fed the scorer's partial sums it also reduces them (in chunk
+// order) into the logits.
 #include <cuda_runtime.h>
 
 #include "kernels.h"
@@ -60,6 +61,52 @@ __device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t* w
 // contention of logits that share a few digit values; merged after each pass.
 constexpr int kSubHist = 8;
 
+// Tokens a thread reduces at once in the logits pass (their partial-sum loads
+// are in flight together), and the keep-ballot store of the compaction.
+constexpr int kLoadUnroll = 4;
+constexpr int kMaxSteps = (kTopkMaxN + kTopkThreads - 1) / kTopkThreads;
+
+// Logits from the scorer's partial sums, summed in chunk order, into the
+// order keys: a thread takes U tokens at a time and reads their partial rows
+// eight at a time, so up to 8U loads are in flight.
+template <int U>
+__device__ __forceinline__ void reduce_logits(const TopkArgs& a, size_t base, uint32_t* keys, int* s_nan) {
+  const int N = a.N;
+  for (int i0 = threadIdx.x; i0 < N; i0 += U * blockDim.x) {
+    float v[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) v[u] = 0.f;
+    for (int c0 = 0; c0 < a.n_chunks; c0 += 8) {
+      float part[U][8];
+      // Every load in bounds (token and chunk clamped), so all 8U go out
+      // back to back; the clamped ones are not used.
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int i = min(i0 + u * static_cast<int>(blockDim.x), N - 1);
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+          const int cc = min(c0 + c, a.n_chunks - 1);
+          part[u][c] = __ldg(a.src + static_cast<size_t>(cc) * a.chunk_stride + base + i);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < U; ++u)
+#pragma unroll
+        for (int c = 0; c < 8; ++c)
+          if (c0 + c < a.n_chunks) v[u] = (c0 + c == 0) ? part[u][c] : v[u] + part[u][c];
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int i = i0 + u * blockDim.x;
+      if (i >= N) break;
+      if (a.logits_out) a.logits_out[base + i] = v[u];
+      if (a.probs_out) a.probs_out[base + i] = 1.0f / (1.0f + expf(-v[u]));
+      if (i >= a.r0 && i < a.r1 && v[u] != v[u]) *s_nan = 1;
+      keys[i] = order_key(v[u]);
+    }
+  }
+}
+
 __global__ void __launch_bounds__(kTopkThreads) topk_kernel(TopkArgs a) {
   griddep_wait();
   griddep_launch_dependents();
@@ -69,6 +116,7 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(TopkArgs a) {
   __shared__ uint32_t warp_tot[32];
   __shared__ uint32_t s_prefix, s_remaining;
   __shared__ int s_nan;
+  __shared__ uint32_t s_ballot[kTopkThreads / 32][kMaxSteps];
 
   const int tid = threadIdx.x;
   const int b = blockIdx.x;
@@ -77,23 +125,11 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(TopkArgs a) {
   if (tid == 0) s_nan = 0;
   __syncthreads();
 
-  // 1. logits (reduced from partial sums in chunk order) -> keys; the
-  // partial rows are read eight at a time so their loads overlap.
-  for (int i = tid; i < N; i += blockDim.x) {
-    float v = 0.f;
-    for (int c0 = 0; c0 < a.n_chunks; c0 += 8) {
-      float part[8];
-#pragma unroll
-      for (int c = 0; c < 8; ++c)
-        part[c] = c0 + c < a.n_chunks ? __ldg(a.src + static_cast<size_t>(c0 + c) * a.chunk_stride + base + i) : 0.f;
-#pragma unroll
-      for (int c = 0; c < 8; ++c)
-        if (c0 + c < a.n_chunks) v = (c0 + c == 0) ? part[c] : v + part[c];
-    }
-    if (a.logits_out) a.logits_out[base + i] = v;
-    if (a.probs_out) a.probs_out[base + i] = 1.0f / (1.0f + expf(-v));
-    if (i >= a.r0 && i < a.r1 && v != v) s_nan = 1;
-    keys[i] = order_key(v);
+  // 1. logits (reduced from partial sums in chunk order) -> keys
+  if (N >= 2 * static_cast<int>(blockDim.x)) {
+    reduce_logits<kLoadUnroll>(a, base, keys, &s_nan);
+  } else {
+    reduce_logits<1>(a, base, keys, &s_nan);
   }
   __syncthreads();
 
@@ -162,54 +198,54 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(TopkArgs a) {
     need_eq = remaining;
   }
 
-  // 3. keep decisions in token order; ties to T ranked by index
-  const int seg = (N + blockDim.x - 1) / blockDim.x;
-  const int s0 = min(tid * seg, N);
-  const int s1 = min(s0 + seg, N);
-  uint32_t eq_cnt = 0;
-  if (!keep_all && !keep_none) {
-    for (int i = s0; i < s1; ++i)
-      if (i >= a.r0 && i < a.r1 && keys[i] == thr) ++eq_cnt;
-  }
-  const uint32_t eq_before = block_exclusive_scan(eq_cnt, warp_tot);
-
-  uint32_t keep_cnt = 0;
-  {
-    uint32_t er = eq_before;
-    for (int i = s0; i < s1; ++i) {
-      bool keep;
-      if (i < a.r0 || i >= a.r1 || keep_all) {
-        keep = true;
-      } else if (keep_none) {
-        keep = false;
-      } else {
-        const uint32_t k = keys[i];
-        if (k > thr) keep = true;
-        else if (k == thr) keep = (er++ < need_eq);
-        else keep = false;
-      }
-      keep_cnt += keep ? 1u : 0u;
+  // 3. keep decisions in token order; ties to T ranked by index.  Warp w owns
+  // tokens [w * steps * 32, (w + 1) * steps * 32), 32 per step.
+  const int lane = tid & 31, warp = tid >> 5;
+  const uint32_t lt = (1u << lane) - 1u;
+  const int steps = (N + blockDim.x - 1) / blockDim.x;
+  const int c0 = warp * steps * 32;
+  const bool select = !keep_all && !keep_none;
+  uint32_t eq_w = 0;
+  if (select) {
+    for (int st = 0; st < steps; ++st) {
+      const int i = c0 + st * 32 + lane;
+      const bool eq = i < N && i >= a.r0 && i < a.r1 && keys[i] == thr;
+      eq_w += __popc(__ballot_sync(0xffffffffu, eq));
     }
   }
-  const uint32_t pos0 = block_exclusive_scan(keep_cnt, warp_tot);
+  uint32_t er = __shfl_sync(0xffffffffu, block_exclusive_scan(lane == 0 ? eq_w : 0u, warp_tot), 0);
+
+  uint32_t keep_w = 0;
+  for (int st = 0; st < steps; ++st) {
+    const int i = c0 + st * 32 + lane;
+    const bool valid = i < N;
+    const bool routable = valid && i >= a.r0 && i < a.r1;
+    const uint32_t k = valid ? keys[i] : 0u;
+    const bool eq = select && routable && k == thr;
+    const uint32_t eqb = __ballot_sync(0xffffffffu, eq);
+    const uint32_t rank = er + __popc(eqb & lt);
+    er += __popc(eqb);
+    bool keep;
+    if (!valid) keep = false;
+    else if (!routable || keep_all) keep = true;
+    else if (keep_none) keep = false;
+    else keep = k > thr || (eq && rank < need_eq);
+    const uint32_t kb = __ballot_sync(0xffffffffu, keep);
+    if (lane == 0) s_ballot[warp][st] = kb;
+    keep_w += __popc(kb);
+  }
+  uint32_t pos = __shfl_sync(0xffffffffu, block_exclusive_scan(lane == 0 ? keep_w : 0u, warp_tot), 0);
 
   const int k_tot = K + N - Nr;
   int32_t* idx = a.idx + static_cast<size_t>(b) * k_tot;
-  uint32_t er = eq_before, pos = pos0;
-  for (int i = s0; i < s1; ++i) {
-    bool keep;
-    if (i < a.r0 || i >= a.r1 || keep_all) {
-      keep = true;
-    } else if (keep_none) {
-      keep = false;
-    } else {
-      const uint32_t k = keys[i];
-      if (k > thr) keep = true;
-      else if (k == thr) keep = (er++ < need_eq);
-      else keep = false;
-    }
-    if (keep && pos < static_cast<uint32_t>(k_tot)) idx[pos++] = i;
-    if (a.mask) a.mask[base + i] = keep ? 1 : 0;
+  for (int st = 0; st < steps; ++st) {
+    const int i = c0 + st * 32 + lane;
+    const uint32_t kb = s_ballot[warp][st];   // written by this warp's lane 0 (block scan barriers since)
+    const bool keep = (kb >> lane) & 1u;
+    const uint32_t slot = pos + __popc(kb & lt);
+    if (keep && slot < static_cast<uint32_t>(k_tot)) idx[slot] = i;
+    if (a.mask && i < N) a.mask[base + i] = keep ? 1 : 0;
+    pos += __popc(kb);
   }
   if (tid == 0 && s_nan) record_status(a.status, CER_DEV_NAN);
 }
