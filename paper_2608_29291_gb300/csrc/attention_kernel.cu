@@ -258,173 +258,177 @@ __global__ void __launch_bounds__(kAttnThreads, 1) packed_attention_kernel(const
 
   if (warp == 0) {
     // ---------------------------------------------------------------- Q and K producer
-    // K streams ahead, limited only by its own ring: S(j) needs just K_j.
-    uint32_t gk = 0, items = 0;
-    bool ok = true;
-    for (int item = blockIdx.x; item < p.n_items && ok; item += gridDim.x, ++items) {
-      const AttnItem it = attn_item(p, item);
-      const int row0 = it.b * p.L;
-      if (!warp_wait(q_empty, (items & 1) ^ 1, abort_flag, p.status)) {
-        ok = false;
-        break;
-      }
-      if (lane == 0) {
-        const int qrow = row0 + it.qt * 128;
-        mbar_arrive_expect_tx(q_full, kQBytes);
-        tma_load_2d(q_tile, &p.tm_qkv, q_full, it.h * kHeadDim, qrow);
-        tma_load_2d(q_tile + kBox, &p.tm_qkv, q_full, it.h * kHeadDim + 64, qrow);
-      }
-      __syncwarp();
-      const int kcol = (p.Hq + it.kh) * kHeadDim;
-      for (int j = 0; j < it.n_kv && ok; ++j) {
-        const uint32_t ks = gk % kKSlots;
-        if (!warp_wait(&k_empty[ks], ((gk / kKSlots) & 1) ^ 1, abort_flag, p.status)) {
+    // One thread issues everything here (TMA copies, mbarrier operations,
+    // tcgen05.mma and commits are per thread): warp-wide waits would only
+    // add a broadcast and a reconvergence to every step.
+    if (lane == 0) {
+      // K streams ahead, limited only by its own ring: S(j) needs just K_j.
+      uint32_t gk = 0, items = 0;
+      bool ok = true;
+      for (int item = blockIdx.x; item < p.n_items && ok; item += gridDim.x, ++items) {
+        const AttnItem it = attn_item(p, item);
+        const int row0 = it.b * p.L;
+        if (!mbar_wait(q_empty, (items & 1) ^ 1, abort_flag, p.status)) {
           ok = false;
           break;
         }
         if (lane == 0) {
-          uint8_t* slot = k_ring + ks * kKBytes;
-          mbar_arrive_expect_tx(&k_full[ks], kKBytes);
-          tma_load_2d(slot, &p.tm_qkv, &k_full[ks], kcol, row0 + j * 128);
-          tma_load_2d(slot + kBox, &p.tm_qkv, &k_full[ks], kcol + 64, row0 + j * 128);
+          const int qrow = row0 + it.qt * 128;
+          mbar_arrive_expect_tx(q_full, kQBytes);
+          tma_load_2d(q_tile, &p.tm_qkv, q_full, it.h * kHeadDim, qrow);
+          tma_load_2d(q_tile + kBox, &p.tm_qkv, q_full, it.h * kHeadDim + 64, qrow);
         }
-        __syncwarp();
-        ++gk;
+        const int kcol = (p.Hq + it.kh) * kHeadDim;
+        for (int j = 0; j < it.n_kv && ok; ++j) {
+          const uint32_t ks = gk % kKSlots;
+          if (!mbar_wait(&k_empty[ks], ((gk / kKSlots) & 1) ^ 1, abort_flag, p.status)) {
+            ok = false;
+            break;
+          }
+          if (lane == 0) {
+            uint8_t* slot = k_ring + ks * kKBytes;
+            mbar_arrive_expect_tx(&k_full[ks], kKBytes);
+            tma_load_2d(slot, &p.tm_qkv, &k_full[ks], kcol, row0 + j * 128);
+            tma_load_2d(slot + kBox, &p.tm_qkv, &k_full[ks], kcol + 64, row0 + j * 128);
+          }
+          ++gk;
+        }
       }
+      if (!ok && lane == 0) unwind_pause(1000000ull);
     }
-    if (!ok && lane == 0) unwind_pause(1000000ull);
+    __syncwarp();
   } else if (warp == 10) {
     // ---------------------------------------------------------------- V producer
-    uint32_t gv = 0;
-    bool ok = true;
-    for (int item = blockIdx.x; item < p.n_items && ok; item += gridDim.x) {
-      const AttnItem it = attn_item(p, item);
-      const int row0 = it.b * p.L;
-      const int vcol = (p.Hq + p.Hkv + it.kh) * kHeadDim;
-      for (int j = 0; j < it.n_kv && ok; ++j) {
-        const uint32_t vs = gv % kVSlots;
-        if (!warp_wait(&v_empty[vs], ((gv / kVSlots) & 1) ^ 1, abort_flag, p.status)) {
-          ok = false;
-          break;
+    if (lane == 0) {
+      uint32_t gv = 0;
+      bool ok = true;
+      for (int item = blockIdx.x; item < p.n_items && ok; item += gridDim.x) {
+        const AttnItem it = attn_item(p, item);
+        const int row0 = it.b * p.L;
+        const int vcol = (p.Hq + p.Hkv + it.kh) * kHeadDim;
+        for (int j = 0; j < it.n_kv && ok; ++j) {
+          const uint32_t vs = gv % kVSlots;
+          if (!mbar_wait(&v_empty[vs], ((gv / kVSlots) & 1) ^ 1, abort_flag, p.status)) {
+            ok = false;
+            break;
+          }
+          if (lane == 0) {
+            uint8_t* slot = v_ring + vs * kVBytes;
+            mbar_arrive_expect_tx(&v_full[vs], kVBytes);
+            tma_load_2d(slot, &p.tm_qkv, &v_full[vs], vcol, row0 + j * 128);
+            tma_load_2d(slot + kBox, &p.tm_qkv, &v_full[vs], vcol + 64, row0 + j * 128);
+          }
+          ++gv;
         }
-        if (lane == 0) {
-          uint8_t* slot = v_ring + vs * kVBytes;
-          mbar_arrive_expect_tx(&v_full[vs], kVBytes);
-          tma_load_2d(slot, &p.tm_qkv, &v_full[vs], vcol, row0 + j * 128);
-          tma_load_2d(slot + kBox, &p.tm_qkv, &v_full[vs], vcol + 64, row0 + j * 128);
-        }
-        __syncwarp();
-        ++gv;
       }
+      if (!ok && lane == 0) unwind_pause(1000000ull);
     }
-    if (!ok && lane == 0) unwind_pause(1000000ull);
+    __syncwarp();
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer
-    // Per item: S(0), S(1); then per key block j: S(j + 2), P(j) V_j.
-    uint32_t gk = 0, gv = 0, items = 0, g = 0, o_taken = 0;
-    bool ok = true;
-    bool issued_any = false;
-    // S(gb) = Q K^T from K slot ks, once P(gb - 3) V (the buffer's previous
-    // reader) has completed.  That wait cannot meet a barrier two phases
-    // ahead: P(gb) V needs S(gb).
-    auto issue_s = [&](uint32_t ks, uint32_t gb) -> bool {
-      const uint32_t buf = gb % kSBufs;
-      if (gb >= kSBufs &&
-          !warp_wait(&pv_done[buf], ((gb - kSBufs) / kSBufs) & 1, abort_flag, p.status))
-        return false;
-      tc_fence_after();
-      if (lane == 0) {
-        const uint32_t q_base = smem_u32(q_tile);
-        const uint32_t k_base = smem_u32(k_ring + ks * kKBytes);
+    if (lane == 0) {
+      // Per item: S(0), S(1); then per key block j: S(j + 2), P(j) V_j.
+      uint32_t gk = 0, gv = 0, items = 0, g = 0, o_taken = 0;
+      bool ok = true;
+      bool issued_any = false;
+      // S(gb) = Q K^T from K slot ks, once P(gb - 3) V (the buffer's previous
+      // reader) has completed.  That wait cannot meet a barrier two phases
+      // ahead: P(gb) V needs S(gb).
+      auto issue_s = [&](uint32_t ks, uint32_t gb) -> bool {
+        const uint32_t buf = gb % kSBufs;
+        if (gb >= kSBufs &&
+            !mbar_wait(&pv_done[buf], ((gb - kSBufs) / kSBufs) & 1, abort_flag, p.status))
+          return false;
+        tc_fence_after();
+        if (lane == 0) {
+          const uint32_t q_base = smem_u32(q_tile);
+          const uint32_t k_base = smem_u32(k_ring + ks * kKBytes);
 #pragma unroll
-        for (int k = 0; k < 8; ++k) {
-          const uint32_t off = (k >> 2) * kBox + (k & 3) * 32;
-          umma_bf16(tmem_base + buf * 128, sdesc_kmajor_sw128(q_base + off), sdesc_kmajor_sw128(k_base + off),
-                    kIdescS, k > 0 ? 1u : 0u);
+          for (int k = 0; k < 8; ++k) {
+            const uint32_t off = (k >> 2) * kBox + (k & 3) * 32;
+            umma_bf16(tmem_base + buf * 128, sdesc_kmajor_sw128(q_base + off), sdesc_kmajor_sw128(k_base + off),
+                      kIdescS, k > 0 ? 1u : 0u);
+          }
+          umma_commit(&s_full[buf]);
+          issued_any = true;
         }
-        umma_commit(&s_full[buf]);
-        issued_any = true;
-      }
-      __syncwarp();
-      return true;
-    };
-    // O (+)= P(gb) V from V slot vs; first: the item's first block (also waits
-    // until the previous item's O has been read out); last: its last block.
-    auto issue_pv = [&](uint32_t vs, uint32_t gb, bool first, bool last) -> bool {
-      const uint32_t buf = gb % kSBufs;
-      if (!warp_wait(&p_full[buf], (gb / kSBufs) & 1, abort_flag, p.status)) return false;
-      if (first) {
-        if (!warp_wait(o_free, (o_taken & 1) ^ 1, abort_flag, p.status)) return false;
-        ++o_taken;
-      }
-      tc_fence_after();
-      if (lane == 0) {
-        const uint32_t v_base = smem_u32(v_ring + vs * kVBytes);
+        return true;
+      };
+      // O (+)= P(gb) V from V slot vs; first: the item's first block (also waits
+      // until the previous item's O has been read out); last: its last block.
+      auto issue_pv = [&](uint32_t vs, uint32_t gb, bool first, bool last) -> bool {
+        const uint32_t buf = gb % kSBufs;
+        if (!mbar_wait(&p_full[buf], (gb / kSBufs) & 1, abort_flag, p.status)) return false;
+        if (first) {
+          if (!mbar_wait(o_free, (o_taken & 1) ^ 1, abort_flag, p.status)) return false;
+          ++o_taken;
+        }
+        tc_fence_after();
+        if (lane == 0) {
+          const uint32_t v_base = smem_u32(v_ring + vs * kVBytes);
 #pragma unroll
-        for (int k = 0; k < 8; ++k) {
-          const uint64_t bdesc = sdesc_mnmajor_sw128(v_base + k * 2048, kBox, 1024);
-          umma_bf16_tmem_a(tmem_base + 384, tmem_base + buf * 128 + k * 8, bdesc, kIdescPV,
-                           (!first || k > 0) ? 1u : 0u);
+          for (int k = 0; k < 8; ++k) {
+            const uint64_t bdesc = sdesc_mnmajor_sw128(v_base + k * 2048, kBox, 1024);
+            umma_bf16_tmem_a(tmem_base + 384, tmem_base + buf * 128 + k * 8, bdesc, kIdescPV,
+                             (!first || k > 0) ? 1u : 0u);
+          }
+          umma_commit(&pv_done[buf]);
+          if (last) umma_commit(o_done);
+          issued_any = true;
         }
-        umma_commit(&pv_done[buf]);
-        if (last) umma_commit(o_done);
-        issued_any = true;
-      }
-      __syncwarp();
-      return true;
-    };
-    for (int item = blockIdx.x; item < p.n_items && ok; item += gridDim.x, ++items) {
-      const AttnItem it = attn_item(p, item);
-      const int n = it.n_kv;
-      if (!warp_wait(q_full, items & 1, abort_flag, p.status)) {
-        ok = false;
-        break;
-      }
-      for (int j = 0; j < 2 && j < n; ++j) {
-        const uint32_t ks = gk % kKSlots;
-        if (!warp_wait(&k_full[ks], (gk / kKSlots) & 1, abort_flag, p.status) || !issue_s(ks, g + j)) {
+        return true;
+      };
+      for (int item = blockIdx.x; item < p.n_items && ok; item += gridDim.x, ++items) {
+        const AttnItem it = attn_item(p, item);
+        const int n = it.n_kv;
+        if (!mbar_wait(q_full, items & 1, abort_flag, p.status)) {
           ok = false;
           break;
         }
-        if (lane == 0) {
-          umma_commit(&k_empty[ks]);
-          if (j + 1 == n) umma_commit(q_empty);
-        }
-        __syncwarp();
-        ++gk;
-      }
-      for (int j = 0; j < n && ok; ++j) {
-        // S(j + 2) first: it needs only K and P(j - 1) V, so it runs while
-        // the softmax still works on block j.
-        if (j + 2 < n) {
+        for (int j = 0; j < 2 && j < n; ++j) {
           const uint32_t ks = gk % kKSlots;
-          if (!warp_wait(&k_full[ks], (gk / kKSlots) & 1, abort_flag, p.status) || !issue_s(ks, g + j + 2)) {
+          if (!mbar_wait(&k_full[ks], (gk / kKSlots) & 1, abort_flag, p.status) || !issue_s(ks, g + j)) {
             ok = false;
             break;
           }
           if (lane == 0) {
             umma_commit(&k_empty[ks]);
-            if (j + 3 == n) umma_commit(q_empty);
+            if (j + 1 == n) umma_commit(q_empty);
           }
-          __syncwarp();
           ++gk;
         }
-        const uint32_t vs = gv % kVSlots;
-        if (!warp_wait(&v_full[vs], (gv / kVSlots) & 1, abort_flag, p.status) ||
-            !issue_pv(vs, g + j, j == 0, j + 1 == n)) {
-          ok = false;
-          break;
+        for (int j = 0; j < n && ok; ++j) {
+          // S(j + 2) first: it needs only K and P(j - 1) V, so it runs while
+          // the softmax still works on block j.
+          if (j + 2 < n) {
+            const uint32_t ks = gk % kKSlots;
+            if (!mbar_wait(&k_full[ks], (gk / kKSlots) & 1, abort_flag, p.status) || !issue_s(ks, g + j + 2)) {
+              ok = false;
+              break;
+            }
+            if (lane == 0) {
+              umma_commit(&k_empty[ks]);
+              if (j + 3 == n) umma_commit(q_empty);
+            }
+            ++gk;
+          }
+          const uint32_t vs = gv % kVSlots;
+          if (!mbar_wait(&v_full[vs], (gv / kVSlots) & 1, abort_flag, p.status) ||
+              !issue_pv(vs, g + j, j == 0, j + 1 == n)) {
+            ok = false;
+            break;
+          }
+          if (lane == 0) umma_commit(&v_empty[vs]);
+          ++gv;
         }
-        if (lane == 0) umma_commit(&v_empty[vs]);
-        __syncwarp();
-        ++gv;
+        g += n;
       }
-      g += n;
+      if (!ok && lane == 0 && issued_any) {
+        umma_commit(drain);
+        drain_wait(drain, 0);
+      }
     }
-    if (!ok && lane == 0 && issued_any) {
-      umma_commit(drain);
-      drain_wait(drain, 0);
-    }
+    __syncwarp();
   } else if (warp < 10) {
     // ---------------------------------------------------------------- softmax
     const int qd = warp & 3;            // TMEM lane quadrant

@@ -326,74 +326,78 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1)
 
   if (warp == 0) {
     // ---------------------------------------------------------------- producer
-    typename P::ProdState st;
-    SegCursor cur(slot, n_slots, ntiles, nkb, dp_tiles);
-    int stage = 0;
-    uint32_t phase = 0;
-    long issued = 0;
-    bool ok = true;
-    // With a pair MMA the even CTA's ring barriers count both CTAs' copies.
-    const uint32_t leader_full = PAIR ? mapa_shared(smem_u32(full), 0) : 0u;
-    int tile, kb0, kb1;
-    while (ok && cur.next(tile, kb0, kb1)) {
-      P::prod_tile(p, tile, rank, st);
-      for (int kb = kb0; kb < kb1; ++kb) {
-        if (!warp_wait(&empty[stage], phase ^ 1, abort_flag, p.status)) {
-          ok = false;
-          break;
+    // One thread: TMA copies and mbarrier operations are per thread, and a
+    // warp-wide wait (test, broadcast, reconverge) would double the cost of
+    // issuing a stage.
+    if (lane == 0) {
+      typename P::ProdState st;
+      SegCursor cur(slot, n_slots, ntiles, nkb, dp_tiles);
+      int stage = 0;
+      uint32_t phase = 0;
+      long issued = 0;
+      bool ok = true;
+      // With a pair MMA the even CTA's ring barriers count both CTAs' copies.
+      const uint32_t leader_full = PAIR ? mapa_shared(smem_u32(full), 0) : 0u;
+      int tile, kb0, kb1;
+      while (ok && cur.next(tile, kb0, kb1)) {
+        P::prod_tile(p, tile, rank, st);
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, p.status)) {
+            ok = false;
+            break;
+          }
+          if (!PAIR || rank == 0) mbar_arrive_expect_tx(&full[stage], P::stage_bytes(p, tile, kb));
+          if constexpr (PAIR) {
+            P::prod_kb(p, st, tile, kb, 0, a_ring + stage * kATileBytes, b_ring + stage * B_BYTES,
+                       leader_full + static_cast<uint32_t>(stage) * 8u);
+          } else {
+            P::prod_kb(p, st, tile, kb, 0, a_ring + stage * kATileBytes, b_ring + stage * B_BYTES, &full[stage]);
+          }
+          ++issued;
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
         }
-        if (!PAIR || rank == 0) {
-          const uint32_t bytes = P::stage_bytes(p, tile, kb);
-          if (lane == 0) mbar_arrive_expect_tx(&full[stage], bytes);
-        }
-        __syncwarp();
-        if constexpr (PAIR) {
-          P::prod_kb(p, st, tile, kb, lane, a_ring + stage * kATileBytes, b_ring + stage * B_BYTES,
-                     leader_full + static_cast<uint32_t>(stage) * 8u);
+      }
+      if (!ok) {
+        // Let the copies already issued land before the CTA's memory goes away
+        // (the odd CTA of a pair cannot see the barrier its copies count on).
+        if (PAIR && rank != 0) {
+          unwind_pause(1000000ull);
         } else {
-          P::prod_kb(p, st, tile, kb, lane, a_ring + stage * kATileBytes, b_ring + stage * B_BYTES, &full[stage]);
-        }
-        ++issued;
-        if (++stage == STAGES) {
-          stage = 0;
-          phase ^= 1;
+          for (long n = issued - 1; n >= 0 && n >= issued - STAGES; --n)
+            drain_wait(&full[n % STAGES], static_cast<uint32_t>((n / STAGES) & 1));
         }
       }
     }
-    if (!ok && lane == 0) {
-      // Let the copies already issued land before the CTA's memory goes away
-      // (the odd CTA of a pair cannot see the barrier its copies count on).
-      if (PAIR && rank != 0) {
-        unwind_pause(1000000ull);
-      } else {
-        for (long n = issued - 1; n >= 0 && n >= issued - STAGES; --n)
-          drain_wait(&full[n % STAGES], static_cast<uint32_t>((n / STAGES) & 1));
-      }
-    }
+    __syncwarp();
   } else if (warp == 1 && (!PAIR || rank == 0)) {
     // ---------------------------------------------------------------- MMA issuer
-    SegCursor cur(slot, n_slots, ntiles, nkb, dp_tiles);
-    int stage = 0;
-    uint32_t phase = 0;
-    int acc = 0;
-    uint32_t acc_phase = 0;
-    bool ok = true;
-    bool issued_any = false;
-    int tile, kb0, kb1;
-    while (ok && cur.next(tile, kb0, kb1)) {
-      if (!warp_wait(&tempty[acc], acc_phase ^ 1, abort_flag, p.status)) {
-        ok = false;
-        break;
-      }
-      tc_fence_after();
-      const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
-      for (int kb = kb0; kb < kb1; ++kb) {
-        if (!warp_wait(&full[stage], phase, abort_flag, p.status)) {
+    // One thread, like the producer (tcgen05.mma and tcgen05.commit are
+    // issued by a single thread).
+    if (lane == 0) {
+      SegCursor cur(slot, n_slots, ntiles, nkb, dp_tiles);
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      bool ok = true;
+      bool issued_any = false;
+      int tile, kb0, kb1;
+      while (ok && cur.next(tile, kb0, kb1)) {
+        if (!mbar_wait(&tempty[acc], acc_phase ^ 1, abort_flag, p.status)) {
           ok = false;
           break;
         }
         tc_fence_after();
-        if (lane == 0) {
+        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!mbar_wait(&full[stage], phase, abort_flag, p.status)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
           const uint32_t a_base = smem_u32(a_ring + stage * kATileBytes);
           const uint32_t b_base = smem_u32(b_ring + stage * B_BYTES);
 #pragma unroll
@@ -411,33 +415,30 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1)
           else
             umma_commit(&empty[stage]);
           issued_any = true;
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
         }
-        __syncwarp();
-        if (++stage == STAGES) {
-          stage = 0;
-          phase ^= 1;
-        }
-      }
-      if (!ok) break;
-      if (lane == 0) {
+        if (!ok) break;
         if (PAIR)
           umma_commit_pair_multicast(&tfull[acc], kPairMask);   // both CTAs' epilogues
         else
           umma_commit(&tfull[acc]);
+        if (++acc == 2) {
+          acc = 0;
+          acc_phase ^= 1;
+        }
       }
-      __syncwarp();
-      if (++acc == 2) {
-        acc = 0;
-        acc_phase ^= 1;
+      if (!ok && issued_any) {
+        if (PAIR)
+          umma_commit_pair(drain);
+        else
+          umma_commit(drain);
+        drain_wait(drain, 0);
       }
     }
-    if (!ok && lane == 0 && issued_any) {
-      if (PAIR)
-        umma_commit_pair(drain);
-      else
-        umma_commit(drain);
-      drain_wait(drain, 0);
-    }
+    __syncwarp();
   } else if (warp >= 2) {
     // ---------------------------------------------------------------- epilogue
     const int q = warp & 3;            // TMEM lane quadrant this warp may access
