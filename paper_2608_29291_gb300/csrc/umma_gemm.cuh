@@ -200,14 +200,13 @@ __device__ __forceinline__ void unwind_pause(uint64_t ns) {
   while (globaltimer_ns() - t0 < ns) __nanosleep(1000);
 }
 
-// Lane 0 waits, the whole warp takes its verdict: keeps every branch after a
-// wait warp-uniform, which the .sync.aligned tcgen05 instructions require.
+// Every lane waits on the same barrier; one vote gives the warp a single
+// verdict, so every branch after a wait stays warp-uniform, which the
+// .sync.aligned tcgen05 instructions require.  (Lane 0 waiting alone and
+// broadcasting its result costs a divergence and a reconvergence per wait.)
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int* status) {
-  int ok = 1;
-  if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, abort_flag, status) ? 1 : 0;
-  ok = __shfl_sync(0xffffffffu, ok, 0);
-  __syncwarp();
-  return ok != 0;
+  const bool ok = mbar_wait(bar, parity, abort_flag, status);
+  return __all_sync(0xffffffffu, ok);
 }
 
 // What an epilogue half (4 warps, 128 threads) shares: the reserved shared
