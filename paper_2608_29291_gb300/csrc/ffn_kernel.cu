@@ -76,13 +76,15 @@ struct GateUpProblemT {
     st.rank = rank;
   }
   // Pair MMA: N columns 0..127 (gate) come from rank 0's B slot, 128..255 (up)
-  // from rank 1's; every copy counts on the even CTA's barrier.
+  // from rank 1's; every copy counts on the even CTA's barrier.  `part`
+  // selects the activation copy, the weight copy or both (kPart*).
+  __device__ static bool weights_first(const Params&) { return true; }
   __device__ static void prod_kb(const Params& p, const ProdState& st, int, int kb, int lane, uint8_t* a,
-                                 uint8_t* b, uint32_t leader_bar) {
+                                 uint8_t* b, uint32_t leader_bar, int part) {
     if (lane == 0) {
       const int x = kb * 64;
-      tma_load_2d_pair(a, &p.tm_x, leader_bar, x, st.m0);
-      tma_load_2d_pair(b, st.rank == 0 ? &p.tm_wg : &p.tm_wu, leader_bar, x, st.c0);
+      if (part & kPartAct) tma_load_2d_pair(a, &p.tm_x, leader_bar, x, st.m0);
+      if (part & kPartWeights) tma_load_2d_pair(b, st.rank == 0 ? &p.tm_wg : &p.tm_wu, leader_bar, x, st.c0);
     }
   }
   __device__ static uint64_t bdesc(uint32_t saddr) { return sdesc_kmajor_sw128(saddr); }
@@ -215,20 +217,26 @@ struct DownProblem {
     st.n0 = nt * BN + (PAIR_ ? rank * CTA_N : 0);
     st.n_atoms = PAIR_ ? ATOMS : atoms(p, nt);
   }
+  // The K extent may come from a device flag the previous kernel writes (the
+  // UCS gate); only without it may the weights go out before that kernel ends.
+  __device__ static bool weights_first(const Params& p) { return p.use_small_k == nullptr; }
   __device__ static void prod_kb(const Params& p, const ProdState& st, int, int kb, int lane, uint8_t* a,
-                                 uint8_t* b, uint64_t* bar) {
+                                 uint8_t* b, uint64_t* bar, int part) {
     if (lane == 0) {
-      tma_load_2d(a, &p.tm_act, bar, kb * 64, st.m0);
-      for (int at = 0; at < st.n_atoms; ++at) tma_load_2d(b + at * kAtomBytes, &p.tm_wdt, bar, st.n0 + at * 64, kb * 64);
+      if (part & kPartAct) tma_load_2d(a, &p.tm_act, bar, kb * 64, st.m0);
+      if (part & kPartWeights)
+        for (int at = 0; at < st.n_atoms; ++at) tma_load_2d(b + at * kAtomBytes, &p.tm_wdt, bar, st.n0 + at * 64, kb * 64);
     }
   }
   __device__ static void prod_kb(const Params& p, const ProdState& st, int, int kb, int lane, uint8_t* a,
-                                 uint8_t* b, uint32_t leader_bar) {
+                                 uint8_t* b, uint32_t leader_bar, int part) {
     if (lane == 0) {
-      tma_load_2d_pair(a, &p.tm_act, leader_bar, kb * 64, st.m0);
+      if (part & kPartAct) tma_load_2d_pair(a, &p.tm_act, leader_bar, kb * 64, st.m0);
+      if (part & kPartWeights) {
 #pragma unroll
-      for (int at = 0; at < ATOMS; ++at)
-        tma_load_2d_pair(b + at * kAtomBytes, &p.tm_wdt, leader_bar, st.n0 + at * 64, kb * 64);
+        for (int at = 0; at < ATOMS; ++at)
+          tma_load_2d_pair(b + at * kAtomBytes, &p.tm_wdt, leader_bar, st.n0 + at * 64, kb * 64);
+      }
     }
   }
   __device__ static uint64_t bdesc(uint32_t saddr) { return sdesc_mnmajor_sw128(saddr, kAtomBytes, 1024); }

@@ -157,18 +157,24 @@ struct ScoreProblem {
     if (st.chunk < p.n_core) {
       st.wrow = st.chunk * BN;
     } else {
-      const double seg = floor(static_cast<double>(p.t[st.b]) * p.S);
-      int m = seg < p.S - 1 ? static_cast<int>(seg) : p.S - 1;
-      if (m < 0) m = 0;
+      int m = 0;
+      if (p.S > 1) {
+        const double seg = floor(static_cast<double>(p.t[st.b]) * p.S);
+        m = seg < p.S - 1 ? static_cast<int>(seg) : p.S - 1;
+        if (m < 0) m = 0;
+      }
       st.wrow = m * p.He + (st.chunk - p.n_core) * BN;
     }
   }
+  // With several expansion segments the weight rows depend on t, which a
+  // previous kernel may write; with one, the weights may go out first.
+  __device__ static bool weights_first(const Params& p) { return p.S <= 1; }
   __device__ static uint32_t stage_bytes(const Params&, int, int) { return kATileBytes + BN * 128; }
   __device__ static void prod_kb(const Params& p, const ProdState& st, int, int kb, int lane, uint8_t* a,
-                                 uint8_t* b, uint64_t* bar) {
+                                 uint8_t* b, uint64_t* bar, int part) {
     if (lane == 0) {
-      tma_load_2d(a, &p.tm_h, bar, kb * 64, st.b * p.N + st.rt * 128);
-      tma_load_2d(b, st.chunk < p.n_core ? &p.tm_w1 : &p.tm_w1e, bar, kb * 64, st.wrow);
+      if (part & kPartAct) tma_load_2d(a, &p.tm_h, bar, kb * 64, st.b * p.N + st.rt * 128);
+      if (part & kPartWeights) tma_load_2d(b, st.chunk < p.n_core ? &p.tm_w1 : &p.tm_w1e, bar, kb * 64, st.wrow);
     }
   }
   __device__ static uint64_t bdesc(uint32_t saddr) { return sdesc_kmajor_sw128(saddr); }

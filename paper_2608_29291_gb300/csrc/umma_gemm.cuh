@@ -58,8 +58,12 @@
 //   BN, STAGES, B_MN_MAJOR, EPI_WARPS, CLUSTER, MMA_PAIR, kBStepBytes,
 //   Params (with `int* status`), num_tiles(p) (cluster tiles),
 //   num_kb(p), prod_tile(p, tile, rank, state),
-//   prod_kb(p, state, tile, kb, lane, a_smem, b_smem, bar) (with MMA_PAIR,
-//   `bar` is the cluster address of the even CTA's ring barrier),
+//   prod_kb(p, state, tile, kb, lane, a_smem, b_smem, bar, part) (with
+//   MMA_PAIR, `bar` is the cluster address of the even CTA's ring barrier;
+//   `part` selects the activation copy, the weight copy or both),
+//   weights_first(p): true when num_tiles, num_kb, prod_tile and the weight
+//   copies read nothing a previous kernel may write, so the producer may
+//   send the first stages' weights before that kernel has finished,
 //   stage_bytes(p, tile, kb) (with MMA_PAIR, the bytes of both CTAs),
 //   bdesc(saddr), prefetch(p) (prefetches the tensor maps' descriptors),
 //   kEpiSmemBytes (shared memory reserved for the epilogue, may be 0),
@@ -73,6 +77,13 @@
 #pragma once
 
 #include <atomic>
+
+namespace cer {
+// Parts of a stage's copies (prod_kb).
+constexpr int kPartAct = 1;       // the A operand, produced by the previous kernel
+constexpr int kPartWeights = 2;   // the B operand, static weights
+constexpr int kPartAll = kPartAct | kPartWeights;
+}
 
 #include "kernels.h"
 #include "ptx.cuh"
@@ -316,7 +327,12 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1)
   }
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  griddep_wait();                 // inputs written by the previous kernel are visible
+  // Inputs written by the previous kernel are visible after this wait.  The
+  // producer, when the weights allow it, first sends its first stages'
+  // weight copies and waits afterwards (programmatic dependent launch starts
+  // this kernel while the previous one is still finishing).
+  const bool weights_first = P::weights_first(p);
+  if (warp != 0 || !weights_first) griddep_wait();
   griddep_launch_dependents();
 
   const int ntiles = P::num_tiles(p);
@@ -337,20 +353,46 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1)
       bool ok = true;
       // With a pair MMA the even CTA's ring barriers count both CTAs' copies.
       const uint32_t leader_full = PAIR ? mapa_shared(smem_u32(full), 0) : 0u;
+      // Stages whose weights went out before the wait (first segment only;
+      // the ring is fresh, so they need no empty-slot wait).
+      long pre = 0;
+      if (weights_first) {
+        SegCursor first = cur;
+        int t0, a0, b0;
+        if (first.next(t0, a0, b0)) {
+          P::prod_tile(p, t0, rank, st);
+          pre = b0 - a0 < STAGES ? b0 - a0 : STAGES;
+          for (int i = 0; i < pre; ++i) {
+            if (!PAIR || rank == 0) mbar_arrive_expect_tx(&full[i], P::stage_bytes(p, t0, a0 + i));
+            if constexpr (PAIR) {
+              P::prod_kb(p, st, t0, a0 + i, 0, a_ring + i * kATileBytes, b_ring + i * B_BYTES,
+                         leader_full + static_cast<uint32_t>(i) * 8u, kPartWeights);
+            } else {
+              P::prod_kb(p, st, t0, a0 + i, 0, a_ring + i * kATileBytes, b_ring + i * B_BYTES, &full[i],
+                         kPartWeights);
+            }
+          }
+        }
+        griddep_wait();
+      }
       int tile, kb0, kb1;
       while (ok && cur.next(tile, kb0, kb1)) {
         P::prod_tile(p, tile, rank, st);
         for (int kb = kb0; kb < kb1; ++kb) {
-          if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, p.status)) {
-            ok = false;
-            break;
+          const bool early = issued < pre;   // its weights and byte count are already out
+          if (!early) {
+            if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, p.status)) {
+              ok = false;
+              break;
+            }
+            if (!PAIR || rank == 0) mbar_arrive_expect_tx(&full[stage], P::stage_bytes(p, tile, kb));
           }
-          if (!PAIR || rank == 0) mbar_arrive_expect_tx(&full[stage], P::stage_bytes(p, tile, kb));
+          const int part = early ? kPartAct : kPartAll;
           if constexpr (PAIR) {
             P::prod_kb(p, st, tile, kb, 0, a_ring + stage * kATileBytes, b_ring + stage * B_BYTES,
-                       leader_full + static_cast<uint32_t>(stage) * 8u);
+                       leader_full + static_cast<uint32_t>(stage) * 8u, part);
           } else {
-            P::prod_kb(p, st, tile, kb, 0, a_ring + stage * kATileBytes, b_ring + stage * B_BYTES, &full[stage]);
+            P::prod_kb(p, st, tile, kb, 0, a_ring + stage * kATileBytes, b_ring + stage * B_BYTES, &full[stage], part);
           }
           ++issued;
           if (++stage == STAGES) {
