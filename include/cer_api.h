@@ -347,8 +347,12 @@ cer_status cer_packed_attention(const void* qkv, int B, int L, int Hq, int Hkv, 
  *          KV cache of the sublayer
  * Requires d a multiple of 64 in [64, 16384] and the head conditions above.
  * The projections accumulate in fp32 on the tensor cores (tcgen05 pair
- * MMA) and round to bf16, like the FFN.
- * Workspace: cer_routed_attention_workspace_size(B, L, d, Hq, Hkv).       */
+ * MMA) and round to bf16, like the FFN; the rotary embedding is applied to
+ * the QKV projection's fp32 accumulator before that rounding (one rounding
+ * instead of cer_rope_packed's two), with the same angles.
+ * Workspace: cer_routed_attention_workspace_size(B, L, d, Hq, Hkv): the
+ * packed rows, qkv, the attention output, the rows' rotary (cos, sin) and
+ * the stream-K area.                                                       */
 cer_status cer_routed_attention(void* h, void* out, int B, int N, int d, const int32_t* idx, int L,
                                 const void* WqkvT, const void* WoT, int Hq, int Hkv, int causal, double base,
                                 void* qkv, void* workspace, size_t workspace_bytes, cudaStream_t stream);

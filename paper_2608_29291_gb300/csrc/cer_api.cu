@@ -939,7 +939,8 @@ size_t cer_routed_attention_workspace_size(int B, int L, int d, int Hq, int Hkv)
   const long long M = static_cast<long long>(B) * L;
   const size_t width = static_cast<size_t>(Hq + 2 * Hkv) * cer::kHeadDim;
   return round256(static_cast<size_t>(M) * d * 2) + round256(static_cast<size_t>(M) * width * 2) +
-         round256(static_cast<size_t>(M) * Hq * cer::kHeadDim * 2) + ffn_stream_k_bytes(M);
+         round256(static_cast<size_t>(M) * Hq * cer::kHeadDim * 2) +
+         round256(static_cast<size_t>(M) * (cer::kHeadDim / 2) * sizeof(float2)) + ffn_stream_k_bytes(M);
 }
 
 cer_status cer_routed_attention(void* h, void* out, int B, int N, int d, const int32_t* idx, int L,
@@ -993,14 +994,21 @@ cer_status cer_routed_attention(void* h, void* out, int B, int N, int d, const i
   ws += round256(static_cast<size_t>(M) * width * 2);
   __nv_bfloat16* attn = reinterpret_cast<__nv_bfloat16*>(ws);
   ws += round256(static_cast<size_t>(M) * Hq * cer::kHeadDim * 2);
+  float2* rope_cs = reinterpret_cast<float2*>(ws);
+  ws += round256(static_cast<size_t>(M) * (cer::kHeadDim / 2) * sizeof(float2));
   cer::FfnArgs proj{};
   carve_stream_k(&ws, M, &proj);
   __nv_bfloat16* qkv_rows = qkv ? static_cast<__nv_bfloat16*>(qkv) : qkv_ws;
 
-  // pack R
-  e = cer::launch_gather(static_cast<const __nv_bfloat16*>(h), B, N, d, idx, L, X, dev->status, dev->n_sm, stream);
+  // pack R, with the rotary (cos, sin) of every packed row's original position
+  cer::RopeFreqTable ft;
+  for (int j = 0; j < cer::kHeadDim / 2; ++j)
+    ft.g[j] = std::pow(base, -2.0 * j / cer::kHeadDim) / (2.0 * M_PI);
+  e = cer::launch_gather_rope(static_cast<const __nv_bfloat16*>(h), B, N, d, idx, L, X, rope_cs, ft, dev->status,
+                              dev->n_sm, stream);
   if (e != cudaSuccess) return cuda_fail(e, "gather launch");
-  // qkv = X WqkvT: the down-projection GEMM in plain-output mode (K = d, N = width)
+  // qkv = X WqkvT: the down-projection GEMM in plain-output mode (K = d,
+  // N = width), the query and key heads rotated in its epilogue
   cer::FfnArgs q = proj;
   q.act = X;
   q.M = M;
@@ -1009,15 +1017,12 @@ cer_status cer_routed_attention(void* h, void* out, int B, int N, int d, const i
   q.WdT = static_cast<const __nv_bfloat16*>(WqkvT);
   q.Y = qkv_rows;
   q.scatter = 0;
+  q.rope_cs = rope_cs;
+  q.rope_heads = Hq + Hkv;
   q.status = dev->status;
   e = cer::launch_ffn_down(q, dev->n_sm, stream);
   if (e != cudaSuccess) return cuda_fail(e, "QKV projection launch");
-  // rotary embedding at the original positions, then attention on the packed rows
-  cer::RopeFreqTable ft;
-  for (int j = 0; j < cer::kHeadDim / 2; ++j)
-    ft.g[j] = std::pow(base, -2.0 * j / cer::kHeadDim) / (2.0 * M_PI);
-  e = cer::launch_rope(qkv_rows, M, Hq, Hkv, idx, ft, dev->status, dev->n_sm, stream);
-  if (e != cudaSuccess) return cuda_fail(e, "rotary embedding launch");
+  // attention on the packed rows
   e = cer::launch_packed_attention(qkv_rows, B, L, Hq, Hkv, causal, attn, dev->status, dev->n_sm, stream);
   if (e != cudaSuccess) return cuda_fail(e, "packed attention launch");
   // out[b, idx] = bf16(h + A WoT): the down-projection GEMM with its fused unpack

@@ -182,8 +182,10 @@ struct DownProblem {
     const __nv_bfloat16* hin;    // scatter mode: residual input
     __nv_bfloat16* out;          // Y [M, d] or the residual output
     const uint8_t* use_small_k;  // optional device flag: contract only the first C_small channels
+    const float2* rope_cs;       // optional rotary (cos, sin) per row (plain mode, BN == 256)
     int* status;
     int scatter;
+    int rope_heads;
     int M, d, C, C_small, N, k_tot, n_mt, n_mtp, n_nt;   // n_mtp: row-tile pairs
   };
   struct ProdState {
@@ -264,6 +266,38 @@ struct DownProblem {
       }
     }
     constexpr int kChunksPerHalf = BN / 64;
+    if constexpr (BN == 256) {
+      // Rotary embedding: with BN = 256 an epilogue half is one whole head
+      // (128 columns), so pair (j, j + 64) is chunk q and chunk q + 2 of the
+      // half.  Rotated from the fp32 accumulator, rounded once.
+      const int col0 = nt * BN + half * 128;
+      if (p.rope_cs != nullptr && !p.scatter && col0 < p.rope_heads * kHeadDim) {
+        const float4* cs4 = reinterpret_cast<const float4*>(p.rope_cs + static_cast<size_t>(valid ? m : 0) * 64);
+#pragma unroll 1
+        for (int q = 0; q < 2; ++q) {
+          float a[32], bv[32];
+          tmem_ld_32x32(taddr + (4 * half + q) * 32, a);
+          tmem_ld_32x32(taddr + (4 * half + q + 2) * 32, bv);
+          if (valid) {
+            uint32_t lo[16], hi[16];
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+              const float4 t = __ldg(cs4 + 16 * q + e);   // cos, sin of j = 32q + 2e and j + 1
+              lo[e] = pack_bf16x2(fmaf(a[2 * e], t.x, -bv[2 * e] * t.y), fmaf(a[2 * e + 1], t.z, -bv[2 * e + 1] * t.w));
+              hi[e] = pack_bf16x2(fmaf(bv[2 * e], t.x, a[2 * e] * t.y), fmaf(bv[2 * e + 1], t.z, a[2 * e + 1] * t.w));
+            }
+            uint4* dlo = reinterpret_cast<uint4*>(p.out + dst_row * p.d + col0 + 32 * q);
+            uint4* dhi = reinterpret_cast<uint4*>(p.out + dst_row * p.d + col0 + 64 + 32 * q);
+#pragma unroll
+            for (int w = 0; w < 4; ++w) {
+              dlo[w] = make_uint4(lo[4 * w], lo[4 * w + 1], lo[4 * w + 2], lo[4 * w + 3]);
+              dhi[w] = make_uint4(hi[4 * w], hi[4 * w + 1], hi[4 * w + 2], hi[4 * w + 3]);
+            }
+          }
+        }
+        return true;
+      }
+    }
 #pragma unroll 1
     for (int c = kChunksPerHalf * half; c < kChunksPerHalf * (half + 1); ++c) {
       float v[32];
@@ -325,6 +359,8 @@ static cudaError_t launch_down(const FfnArgs& a, int n_sm, cudaStream_t stream) 
   p.hin = a.h;
   p.out = a.scatter ? a.out : a.Y;
   p.use_small_k = a.use_small_k;
+  p.rope_cs = a.rope_cs;
+  p.rope_heads = a.rope_heads;
   p.status = a.status;
   p.scatter = a.scatter;
   p.M = a.M;
@@ -362,7 +398,12 @@ int down_tile_width(int M, int d, int n_sm) {
 }
 
 cudaError_t launch_ffn_down(const FfnArgs& a, int n_sm, cudaStream_t stream) {
-  switch (down_tile_width(a.M, a.d, n_sm)) {
+  const int width = down_tile_width(a.M, a.d, n_sm);
+  if (a.rope_cs != nullptr) {
+    // the fused rotary embedding wants whole heads in each epilogue half
+    return width == 0 ? launch_down<256, 1>(a, n_sm, stream) : launch_down<256, 0>(a, n_sm, stream);
+  }
+  switch (width) {
     case 0: return launch_down<256, 1>(a, n_sm, stream);
     case 192: return launch_down<192, 0>(a, n_sm, stream);
     case 128: return launch_down<128, 0>(a, n_sm, stream);

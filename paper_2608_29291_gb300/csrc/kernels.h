@@ -149,6 +149,12 @@ struct FfnArgs {
   const uint8_t* use_small_k;
   int C_small;
   StreamKArea sk;   // optional
+  // Rotary embedding fused into a plain-output down GEMM (the attention
+  // sublayer's QKV projection): with rope_cs != NULL, output columns of heads
+  // [0, rope_heads) (128 columns each) are rotated, pair (j, j + 64) by the
+  // angle of row m whose (cos, sin) is rope_cs[m * 64 + j].
+  const float2* rope_cs;
+  int rope_heads;
   int* status;
 };
 cudaError_t launch_ffn_gateup(const FfnArgs& a, int n_sm, cudaStream_t stream);
@@ -185,6 +191,12 @@ struct RopeFreqTable {
 // original position pos[row] (the keep list, [B * L]).
 cudaError_t launch_rope(__nv_bfloat16* qkv, long long rows, int Hq, int Hkv, const int32_t* pos,
                         const RopeFreqTable& ft, int* status, int n_sm, cudaStream_t stream);
+// The row gather (S3) that also writes, for every packed row m, the rotary
+// (cos, sin) of its position idx[m] for the 64 frequencies: cs [M][64], the
+// same arithmetic as the rotary-embedding kernel.
+cudaError_t launch_gather_rope(const __nv_bfloat16* h, int B, int N, int d, const int32_t* idx, int k_tot,
+                               __nv_bfloat16* X, float2* cs, const RopeFreqTable& ft, int* status, int n_sm,
+                               cudaStream_t stream);
 
 // out [B * L, Hq * 128] = softmax(Q K^T / sqrt(128)) V per sequence and query
 // head over the packed tokens (causal: key index <= query index).

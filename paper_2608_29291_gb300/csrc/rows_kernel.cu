@@ -12,9 +12,15 @@ namespace cer {
 
 constexpr int kRowThreads = 512;
 
+// With ROPE the warp also writes row m's rotary (cos, sin) for the 64
+// frequencies, two per lane: the angle in turns x = i * g_j (fp64, reduced
+// exactly) through fp32 sincospif, as in the rotary-embedding kernel.
+template <bool ROPE>
 __global__ void __launch_bounds__(kRowThreads) gather_rows_kernel(const uint4* __restrict__ h, int N, int d16,
                                                                   const int32_t* __restrict__ idx, int k_tot,
-                                                                  int M, uint4* __restrict__ X, int* status) {
+                                                                  int M, uint4* __restrict__ X, int* status,
+                                                                  float2* __restrict__ cs,
+                                                                  const __grid_constant__ RopeFreqTable ft) {
   griddep_wait();
   griddep_launch_dependents();
   const int lane = threadIdx.x & 31;
@@ -25,6 +31,16 @@ __global__ void __launch_bounds__(kRowThreads) gather_rows_kernel(const uint4* _
     if (i < 0 || i >= N) {
       if (lane == 0) record_status(status, CER_DEV_INDEX);
       continue;
+    }
+    if constexpr (ROPE) {
+#pragma unroll
+      for (int u = 0; u < 2; ++u) {
+        const int j = lane + 32 * u;
+        const double x = static_cast<double>(i) * ft.g[j];
+        float sn, cn;
+        sincospif(2.0f * static_cast<float>(x - rint(x)), &sn, &cn);
+        cs[static_cast<size_t>(m) * (kHeadDim / 2) + j] = make_float2(cn, sn);
+      }
     }
     const uint4* src = h + (static_cast<size_t>(b) * N + i) * d16;
     uint4* dst = X + static_cast<size_t>(m) * d16;
@@ -91,8 +107,19 @@ cudaError_t launch_gather(const __nv_bfloat16* h, int B, int N, int d, const int
                           __nv_bfloat16* X, int* status, int n_sm, cudaStream_t stream) {
   const int M = B * k_tot;
   if (M == 0 || d == 0) return cudaSuccess;
-  return launch_k(gather_rows_kernel, dim3(row_grid(M, n_sm)), dim3(kRowThreads), 0, stream, 1,
-                  reinterpret_cast<const uint4*>(h), N, d / 8, idx, k_tot, M, reinterpret_cast<uint4*>(X), status);
+  return launch_k(gather_rows_kernel<false>, dim3(row_grid(M, n_sm)), dim3(kRowThreads), 0, stream, 1,
+                  reinterpret_cast<const uint4*>(h), N, d / 8, idx, k_tot, M, reinterpret_cast<uint4*>(X), status,
+                  static_cast<float2*>(nullptr), RopeFreqTable{});
+}
+
+cudaError_t launch_gather_rope(const __nv_bfloat16* h, int B, int N, int d, const int32_t* idx, int k_tot,
+                               __nv_bfloat16* X, float2* cs, const RopeFreqTable& ft, int* status, int n_sm,
+                               cudaStream_t stream) {
+  const int M = B * k_tot;
+  if (M == 0 || d == 0) return cudaSuccess;
+  return launch_k(gather_rows_kernel<true>, dim3(row_grid(M, n_sm)), dim3(kRowThreads), 0, stream, 1,
+                  reinterpret_cast<const uint4*>(h), N, d / 8, idx, k_tot, M, reinterpret_cast<uint4*>(X), status, cs,
+                  ft);
 }
 
 cudaError_t launch_scatter_add(__nv_bfloat16* h, int B, int N, int d, const int32_t* idx, int k_tot,

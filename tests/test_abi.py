@@ -129,7 +129,7 @@ def test_attention_argument_checks(lib):
     assert ra(FAKE, None, 1, 16, 128, FAKE, 8, FAKE, FAKE, 4, 2, 1, 1e6, None, FAKE, 64, None) == 9    # workspace
     W = (4 + 2 * 2) * 128
     assert lib.cer_routed_attention_workspace_size(2, 10, 128, 4, 2) == \
-        _r256(20 * 128 * 2) + _r256(20 * W * 2) + _r256(20 * 512 * 2) + (24 << 20) + 8192
+        _r256(20 * 128 * 2) + _r256(20 * W * 2) + _r256(20 * 512 * 2) + _r256(20 * 64 * 8) + (24 << 20) + 8192
     assert lib.cer_routed_attention_workspace_size(2, 0, 128, 4, 2) == 0
 
 
