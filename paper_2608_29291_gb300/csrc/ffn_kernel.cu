@@ -44,7 +44,8 @@ template <int EPI_WARPS_>
 struct GateUpProblemT {
   static constexpr int BN = 256;
   static constexpr int MMA_PAIR = 1;
-  static constexpr int STAGES = 6;
+  static constexpr int KSUB = 2;
+  static constexpr int STAGES = 3;
   static constexpr int B_MN_MAJOR = 0;
   static constexpr int EPI_WARPS = EPI_WARPS_;
   static constexpr int kGroups = EPI_WARPS / 4;
@@ -69,7 +70,9 @@ struct GateUpProblemT {
   // Cluster tile t covers row tiles 2*(t % n_mtp) + {0, 1} and channel tile t / n_mtp.
   __device__ static int num_tiles(const Params& p) { return p.n_mtp * p.n_ct; }
   __device__ static int num_kb(const Params& p) { return p.d / 64; }
-  __device__ static uint32_t stage_bytes(const Params&, int, int) { return 2 * (kATileBytes + 128 * 128); }
+  __device__ static uint32_t stage_bytes(const Params&, int, int, int part) {
+    return 2 * (((part & kPartAct) ? kATileBytes : 0u) + ((part & kPartWeights) ? kBoxBytes : 0u));
+  }
   __device__ static void prod_tile(const Params& p, int tile, int rank, ProdState& st) {
     st.c0 = (tile / p.n_mtp) * 128;
     st.m0 = (2 * (tile % p.n_mtp) + rank) * 128;   // rows past M load as zeros
@@ -82,7 +85,7 @@ struct GateUpProblemT {
   __device__ static void prod_kb(const Params& p, const ProdState& st, int, int kb, int lane, uint8_t* a,
                                  uint8_t* b, uint32_t leader_bar, int part) {
     if (lane == 0) {
-      const int x = kb * 64;
+      const int x = kb * 64;   // K blocks past d load as zeros
       if (part & kPartAct) tma_load_2d_pair(a, &p.tm_x, leader_bar, x, st.m0);
       if (part & kPartWeights) tma_load_2d_pair(b, st.rank == 0 ? &p.tm_wg : &p.tm_wu, leader_bar, x, st.c0);
     }
@@ -167,7 +170,9 @@ struct DownProblem {
   static constexpr int CLUSTER = PAIR_ ? 2 : 1;
   static constexpr int CTA_N = PAIR_ ? BN / 2 : BN;   // B columns in one CTA's ring slot
   static constexpr int ATOMS = CTA_N / 64;
-  static constexpr int STAGES = PAIR_ ? 7 : BN == 256 ? 4 : BN == 192 ? 5 : 6;
+  // Two K blocks per slot where three slots fit.
+  static constexpr int KSUB = (PAIR_ || BN == 128) ? 2 : 1;
+  static constexpr int STAGES = KSUB == 2 ? 3 : BN == 256 ? 4 : 5;
   static constexpr int B_MN_MAJOR = 1;
   static constexpr int EPI_WARPS = 8;
   static constexpr uint32_t kBStepBytes = 2048;     // 16 K-rows = two 1024 B row groups
@@ -177,7 +182,7 @@ struct DownProblem {
 
   struct Params {
     CUtensorMap tm_act;  // act [M, C], box 64 x 128
-    CUtensorMap tm_wdt;  // WdT [C, d], box 64 x 64
+    CUtensorMap tm_wdt;  // WdT [C, d] as [d/64][C][64], box 64 x 64 x ATOMS: one K block's atoms
     const int32_t* idx;          // scatter mode: keep list [B][k_tot]
     const __nv_bfloat16* hin;    // scatter mode: residual input
     __nv_bfloat16* out;          // Y [M, d] or the residual output
@@ -189,7 +194,7 @@ struct DownProblem {
     int M, d, C, C_small, N, k_tot, n_mt, n_mtp, n_nt;   // n_mtp: row-tile pairs
   };
   struct ProdState {
-    int m0, n0, n_atoms;
+    int m0, atom0;
   };
 
   // Tile t: N tile t / R and row tile t % R (pair: rows 2 (t % R) + rank),
@@ -203,21 +208,15 @@ struct DownProblem {
   __device__ static int num_kb(const Params& p) {
     return (p.use_small_k != nullptr && *p.use_small_k) ? p.C_small / 64 : p.C / 64;
   }
-  __device__ static int atoms(const Params& p, int nt) {
-    const int left = (p.d - nt * BN) / 64;
-    return left < ATOMS ? left : ATOMS;
-  }
-  // The pair always loads whole atoms (columns past d read as zeros), so both
-  // CTAs' byte counts are known to the even CTA.
-  __device__ static uint32_t stage_bytes(const Params& p, int tile, int) {
-    if (PAIR_) return 2 * (kATileBytes + ATOMS * kAtomBytes);
-    return kATileBytes + atoms(p, tile / rows_per_n(p)) * kAtomBytes;
+  // Whole boxes always: atoms past d and K blocks past C load as zeros, so
+  // every slot's byte count is fixed (and, for a pair, known to the even CTA).
+  __device__ static uint32_t stage_bytes(const Params&, int, int, int part) {
+    return (PAIR_ ? 2 : 1) * (((part & kPartAct) ? kATileBytes : 0u) + ((part & kPartWeights) ? ATOMS * kAtomBytes : 0u));
   }
   __device__ static void prod_tile(const Params& p, int tile, int rank, ProdState& st) {
     const int nt = tile / rows_per_n(p);
     st.m0 = row_tile(p, tile, rank) * 128;   // rows past M load as zeros
-    st.n0 = nt * BN + (PAIR_ ? rank * CTA_N : 0);
-    st.n_atoms = PAIR_ ? ATOMS : atoms(p, nt);
+    st.atom0 = (nt * BN + (PAIR_ ? rank * CTA_N : 0)) / 64;
   }
   // The K extent may come from a device flag the previous kernel writes (the
   // UCS gate); only without it may the weights go out before that kernel ends.
@@ -226,19 +225,14 @@ struct DownProblem {
                                  uint8_t* b, uint64_t* bar, int part) {
     if (lane == 0) {
       if (part & kPartAct) tma_load_2d(a, &p.tm_act, bar, kb * 64, st.m0);
-      if (part & kPartWeights)
-        for (int at = 0; at < st.n_atoms; ++at) tma_load_2d(b + at * kAtomBytes, &p.tm_wdt, bar, st.n0 + at * 64, kb * 64);
+      if (part & kPartWeights) tma_load_3d(b, &p.tm_wdt, bar, 0, kb * 64, st.atom0);
     }
   }
   __device__ static void prod_kb(const Params& p, const ProdState& st, int, int kb, int lane, uint8_t* a,
                                  uint8_t* b, uint32_t leader_bar, int part) {
     if (lane == 0) {
       if (part & kPartAct) tma_load_2d_pair(a, &p.tm_act, leader_bar, kb * 64, st.m0);
-      if (part & kPartWeights) {
-#pragma unroll
-        for (int at = 0; at < ATOMS; ++at)
-          tma_load_2d_pair(b + at * kAtomBytes, &p.tm_wdt, leader_bar, st.n0 + at * 64, kb * 64);
-      }
+      if (part & kPartWeights) tma_load_3d_pair(b, &p.tm_wdt, leader_bar, 0, kb * 64, st.atom0);
     }
   }
   __device__ static uint64_t bdesc(uint32_t saddr) { return sdesc_mnmajor_sw128(saddr, kAtomBytes, 1024); }
@@ -354,7 +348,7 @@ static cudaError_t launch_down(const FfnArgs& a, int n_sm, cudaStream_t stream) 
   using P = DownProblem<BN, PAIR>;
   typename P::Params p{};
   if (!encode_bf16_2d(&p.tm_act, a.act, a.M, a.C, 64, 128)) return cudaErrorInvalidValue;
-  if (!encode_bf16_2d(&p.tm_wdt, a.WdT, a.C, a.d, 64, 64)) return cudaErrorInvalidValue;
+  if (!encode_bf16_col_blocks(&p.tm_wdt, a.WdT, a.C, a.d, 64, P::ATOMS)) return cudaErrorInvalidValue;
   p.idx = a.idx;
   p.hin = a.h;
   p.out = a.scatter ? a.out : a.Y;

@@ -17,6 +17,14 @@ namespace cer {
 bool encode_bf16_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_cols,
                     uint32_t box_rows);
 
+// Encode a row-major bf16 matrix (rows x cols, cols a multiple of 64) as the
+// 3-D tensor [cols / 64][rows][64] with a box of 64 x box_rows x box_blocks:
+// one copy brings box_blocks consecutive 64-column blocks of box_rows rows,
+// each block a 128-byte-swizzled [box_rows][64] tile, the blocks one after
+// another in shared memory.  The innermost coordinate is always 0.
+bool encode_bf16_col_blocks(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows,
+                            uint32_t box_blocks);
+
 // Launch `kernel` with programmatic dependent launch allowed (and a cluster
 // dimension when cluster_x > 1): it may start while the previous kernel on
 // the stream finishes; its griddep_wait() orders it after that kernel.

@@ -120,7 +120,8 @@ struct ScoreProblem {
   static constexpr int BN = BN_;
   static constexpr int MMA_PAIR = 0;
   static constexpr int CLUSTER = 1;
-  static constexpr int STAGES = BN == 256 ? 4 : BN == 128 ? 6 : 8;
+  static constexpr int KSUB = BN == 256 ? 1 : 2;   // K blocks per ring slot
+  static constexpr int STAGES = BN == 128 ? 3 : 4;
   static constexpr int B_MN_MAJOR = 0;
   static constexpr int EPI_WARPS = 8;
   static constexpr uint32_t kBStepBytes = 32;
@@ -169,12 +170,15 @@ struct ScoreProblem {
   // With several expansion segments the weight rows depend on t, which a
   // previous kernel may write; with one, the weights may go out first.
   __device__ static bool weights_first(const Params& p) { return p.S <= 1; }
-  __device__ static uint32_t stage_bytes(const Params&, int, int) { return kATileBytes + BN * 128; }
+  __device__ static uint32_t stage_bytes(const Params&, int, int, int part) {
+    return ((part & kPartAct) ? kATileBytes : 0u) + ((part & kPartWeights) ? BN * 128u : 0u);
+  }
   __device__ static void prod_kb(const Params& p, const ProdState& st, int, int kb, int lane, uint8_t* a,
                                  uint8_t* b, uint64_t* bar, int part) {
     if (lane == 0) {
-      if (part & kPartAct) tma_load_2d(a, &p.tm_h, bar, kb * 64, st.b * p.N + st.rt * 128);
-      if (part & kPartWeights) tma_load_2d(b, st.chunk < p.n_core ? &p.tm_w1 : &p.tm_w1e, bar, kb * 64, st.wrow);
+      const int x = kb * 64;   // K blocks past d load as zeros
+      if (part & kPartAct) tma_load_2d(a, &p.tm_h, bar, x, st.b * p.N + st.rt * 128);
+      if (part & kPartWeights) tma_load_2d(b, st.chunk < p.n_core ? &p.tm_w1 : &p.tm_w1e, bar, x, st.wrow);
     }
   }
   __device__ static uint64_t bdesc(uint32_t saddr) { return sdesc_kmajor_sw128(saddr); }

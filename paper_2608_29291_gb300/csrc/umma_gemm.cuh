@@ -1,17 +1,20 @@
 // umma_gemm.cuh -- persistent, warp-specialised tcgen05 GEMM skeleton for
 // sm_103a, shared by the scorer and the two FFN contractions.
 //
-// One CTA per SM (64 + 32*EPI_WARPS threads, up to ~225 KB shared memory,
+// One CTA per SM (96 + 32*EPI_WARPS threads, up to ~225 KB shared memory,
 // 2*BN TMEM columns):
-//   warp 0     producer: TMA box loads of the A tile (128 rows x 64 bf16)
-//              and the B tile (BN rows x 64 bf16, or 64 K-rows x BN for an
-//              MN-major B) into a STAGES-deep ring;
+//   warp 0     activation producer: TMA loads of the A tile (128 rows x 64
+//              bf16 per K block) into a STAGES-deep ring;
+//   warp 2     weight producer: TMA loads of the B tile (BN rows x 64 bf16,
+//              or 64 K-rows x BN for an MN-major B) into the same ring; a
+//              ring slot holds KSUB consecutive 64-wide K blocks, each with
+//              its own "full" barrier and one "empty" barrier for the slot;
 //   warp 1     allocates TMEM, one elected lane issues tcgen05.mma
 //              (M=128, N=BN, K=16) four times per 64-wide K block and
-//              commits the ring slot back to the producer;
-//   warps 2..  epilogue, EPI_WARPS = 4 or 8: read the fp32 accumulator out of
-//              TMEM (lane = tile row; with 8 warps, warps 2-5 take the first
-//              half of the columns and warps 6-9 the second) and apply the
+//              commits the ring slot back to both producers;
+//   warps 3..  epilogue, EPI_WARPS = 4 or 8: read the fp32 accumulator out of
+//              TMEM (lane = tile row; with 8 warps, warps 3-6 take the first
+//              half of the columns and warps 7-10 the second) and apply the
 //              problem's fused epilogue.
 // The accumulator is double-buffered in TMEM so the epilogue of one tile
 // overlaps the MMAs of the next.
@@ -51,20 +54,41 @@
 // K-block rate per slot drops as slots are added), so splitting only pays
 // where a last wave would leave most slots idle; see stream_k_dp_tiles.
 //
+// Slots, barriers and threads, as measured on GB300 (globaltimer traces of
+// the FFN GEMMs):
+//   - every slot costs the MMA thread a wait, a fence and a commit; with one
+//     64-wide K block per slot that overhead made the 256 x 256 pair tile
+//     ~10% slower than with two (KSUB = 2);
+//   - a ring of three 64 KB slots gives a freed slot ~1 us to refill before
+//     the MMAs need it, about one copy latency; with a single barrier per
+//     slot the MMA thread waited for data a fifth of its time.  A "full"
+//     barrier per K block lets the MMAs start on the first half of a slot
+//     while the second half still streams in;
+//   - each slot costs a producer thread an empty-slot wait, an expect_tx and
+//     one TMA instruction per box, a few hundred cycles whatever the box
+//     size; one thread per operand keeps that below the MMA time.
+// When the weights come from no earlier kernel the weight producer never
+// waits for it (programmatic dependent launch): its copies start at once.
+//
 // Every wait is bounded (ptx.cuh); on a timeout the CTA unwinds, waits
 // briefly for its own copies and MMAs, frees TMEM and exits.
 //
 // A problem class P supplies:
 //   BN, STAGES, B_MN_MAJOR, EPI_WARPS, CLUSTER, MMA_PAIR, kBStepBytes,
+//   KSUB (64-wide K blocks per ring slot, 1 or 2),
 //   Params (with `int* status`), num_tiles(p) (cluster tiles),
-//   num_kb(p), prod_tile(p, tile, rank, state),
-//   prod_kb(p, state, tile, kb, lane, a_smem, b_smem, bar, part) (with
-//   MMA_PAIR, `bar` is the cluster address of the even CTA's ring barrier;
-//   `part` selects the activation copy, the weight copy or both),
+//   num_kb(p) (64-wide K blocks; K blocks of the last slot past the end are
+//   still copied -- zeros or unused data -- but their MMAs are skipped),
+//   prod_tile(p, tile, rank, state),
+//   prod_kb(p, state, tile, kb, lane, a_smem, b_smem, bar, part): the copies
+//   of 64-wide K block kb (with MMA_PAIR, `bar` is the cluster address of
+//   the even CTA's barrier; `part` selects the activation copy, the weight
+//   copy or both),
 //   weights_first(p): true when num_tiles, num_kb, prod_tile and the weight
-//   copies read nothing a previous kernel may write, so the producer may
-//   send the first stages' weights before that kernel has finished,
-//   stage_bytes(p, tile, kb) (with MMA_PAIR, the bytes of both CTAs),
+//   copies read nothing a previous kernel may write, so the weight producer
+//   need not wait for that kernel to finish,
+//   stage_bytes(p, tile, kb, part) (the bytes of the selected copies of one
+//   K block; with MMA_PAIR, of both CTAs),
 //   bdesc(saddr), prefetch(p) (prefetches the tensor maps' descriptors),
 //   kEpiSmemBytes (shared memory reserved for the epilogue, may be 0),
 //   epilogue(p, tile, row, half, taddr, ctx) -> false to abort (ctx.rank is
@@ -92,8 +116,9 @@ namespace cer {
 
 template <class P>
 constexpr int gemm_threads() {
-  return 64 + 32 * P::EPI_WARPS;
+  return 96 + 32 * P::EPI_WARPS;
 }
+constexpr int kFirstEpiWarp = 3;
 constexpr uint32_t kATileBytes = 128 * 128;  // 128 rows x 64 bf16
 
 template <int BN>
@@ -102,15 +127,26 @@ struct TmemCols {
   static constexpr uint32_t value = need <= 32 ? 32 : need <= 64 ? 64 : need <= 128 ? 128 : need <= 256 ? 256 : 512;
 };
 
-// Bytes of one ring slot's B tile in one CTA (half of it with a pair MMA).
+// Bytes of one 64-wide K block of the B tile in one CTA (half of it with a
+// pair MMA).
 template <class P>
 __host__ __device__ constexpr uint32_t b_stage_bytes() {
   return static_cast<uint32_t>(P::MMA_PAIR ? P::BN / 2 : P::BN) * 128u;
 }
 
+// One ring slot (KSUB K blocks) of each operand in one CTA.
+template <class P>
+__host__ __device__ constexpr uint32_t a_slot_bytes() {
+  return static_cast<uint32_t>(P::KSUB) * kATileBytes;
+}
+template <class P>
+__host__ __device__ constexpr uint32_t b_slot_bytes() {
+  return static_cast<uint32_t>(P::KSUB) * b_stage_bytes<P>();
+}
+
 template <class P>
 constexpr size_t gemm_smem_bytes() {
-  return 1024 + static_cast<size_t>(P::STAGES) * (kATileBytes + b_stage_bytes<P>()) + P::kEpiSmemBytes + 256;
+  return 1024 + static_cast<size_t>(P::STAGES) * (a_slot_bytes<P>() + b_slot_bytes<P>()) + P::kEpiSmemBytes + 256;
 }
 
 // Stream-K split of a launch (see above).  partial == nullptr: every tile
@@ -266,17 +302,20 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1)
   constexpr int STAGES = P::STAGES;
   constexpr int HALVES = P::EPI_WARPS / 4;
   constexpr int HALF_COLS = BN / HALVES;
-  constexpr uint32_t B_BYTES = b_stage_bytes<P>();
+  constexpr int KSUB = P::KSUB;
+  static_assert(KSUB == 1 || KSUB == 2, "one or two K blocks per ring slot");
+  constexpr uint32_t A_BYTES = a_slot_bytes<P>();
+  constexpr uint32_t B_BYTES = b_slot_bytes<P>();
   constexpr uint32_t TMEM_COLS = TmemCols<BN>::value;
   constexpr uint32_t IDESC = idesc_bf16(PAIR ? 256 : 128, BN, P::B_MN_MAJOR);
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* a_ring = smem;
-  uint8_t* b_ring = smem + STAGES * kATileBytes;
+  uint8_t* b_ring = smem + STAGES * A_BYTES;
   uint8_t* epi_smem = b_ring + STAGES * B_BYTES;  // 1024-byte aligned
-  uint64_t* full = reinterpret_cast<uint64_t*>(epi_smem + P::kEpiSmemBytes);
-  uint64_t* empty = full + STAGES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(epi_smem + P::kEpiSmemBytes);   // [STAGES][KSUB]
+  uint64_t* empty = full + STAGES * KSUB;
   uint64_t* tfull = empty + STAGES;
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tempty + 2;
@@ -293,10 +332,10 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1)
 
   if (threadIdx.x == 32) P::prefetch(p);   // tensor-map descriptors, ahead of the first copy
   if (threadIdx.x == 0) {
-    for (int s = 0; s < STAGES; ++s) {
-      mbar_init(&full[s], 1);
+    for (int s = 0; s < STAGES * KSUB; ++s)
+      mbar_init(&full[s], 2);    // the two producers' expect_tx (the even CTA's, with a pair MMA)
+    for (int s = 0; s < STAGES; ++s)
       mbar_init(&empty[s], 1);   // one MMA commit (the even CTA's, with a pair MMA)
-    }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull[a], 1);
       // Every epilogue thread (with a pair MMA: every epilogue warp of both CTAs).
@@ -327,24 +366,34 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1)
   }
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  // Inputs written by the previous kernel are visible after this wait.  The
-  // producer, when the weights allow it, first sends its first stages'
-  // weight copies and waits afterwards (programmatic dependent launch starts
-  // this kernel while the previous one is still finishing).
+  // Inputs written by the previous kernel are visible after this wait
+  // (programmatic dependent launch starts this kernel while the previous one
+  // is still finishing).  The weight producer skips it when the weights and
+  // the tile walk depend on nothing that kernel writes.  It then does not
+  // signal the dependents either: the first signal of any thread releases
+  // the CTA, and every CTA signalling only after its own wait keeps the rule
+  // that when a kernel starts, the kernels two or more launches back have
+  // completed -- which is what makes weights written there safe to read
+  // without the wait.
   const bool weights_first = P::weights_first(p);
-  if (warp != 0 || !weights_first) griddep_wait();
-  griddep_launch_dependents();
+  if (warp != 2 || !weights_first) {
+    griddep_wait();
+    griddep_launch_dependents();
+  }
 
   const int ntiles = P::num_tiles(p);
-  const int nkb = P::num_kb(p);
+  const int nk64 = P::num_kb(p);                 // 64-wide K blocks
+  const int nkb = (nk64 + KSUB - 1) / KSUB;      // ring slots per tile
   const int dp_tiles = sk.partial != nullptr && sk.dp_tiles < ntiles ? sk.dp_tiles : ntiles;
 
-  if (warp == 0) {
-    // ---------------------------------------------------------------- producer
-    // One thread: TMA copies and mbarrier operations are per thread, and a
-    // warp-wide wait (test, broadcast, reconverge) would double the cost of
-    // issuing a stage.
+  if (warp == 0 || warp == 2) {
+    // ---------------------------------------------------------------- producers
+    // One thread each: TMA copies and mbarrier operations are per thread, and
+    // a warp-wide wait (test, broadcast, reconverge) would double the cost of
+    // issuing a slot.  Warp 0 copies the activations, warp 2 the weights;
+    // both walk the same slots and each adds its own bytes to a slot's count.
     if (lane == 0) {
+      const int part = warp == 0 ? kPartAct : kPartWeights;
       typename P::ProdState st;
       SegCursor cur(slot, n_slots, ntiles, nkb, dp_tiles);
       int stage = 0;
@@ -353,46 +402,26 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1)
       bool ok = true;
       // With a pair MMA the even CTA's ring barriers count both CTAs' copies.
       const uint32_t leader_full = PAIR ? mapa_shared(smem_u32(full), 0) : 0u;
-      // Stages whose weights went out before the wait (first segment only;
-      // the ring is fresh, so they need no empty-slot wait).
-      long pre = 0;
-      if (weights_first) {
-        SegCursor first = cur;
-        int t0, a0, b0;
-        if (first.next(t0, a0, b0)) {
-          P::prod_tile(p, t0, rank, st);
-          pre = b0 - a0 < STAGES ? b0 - a0 : STAGES;
-          for (int i = 0; i < pre; ++i) {
-            if (!PAIR || rank == 0) mbar_arrive_expect_tx(&full[i], P::stage_bytes(p, t0, a0 + i));
-            if constexpr (PAIR) {
-              P::prod_kb(p, st, t0, a0 + i, 0, a_ring + i * kATileBytes, b_ring + i * B_BYTES,
-                         leader_full + static_cast<uint32_t>(i) * 8u, kPartWeights);
-            } else {
-              P::prod_kb(p, st, t0, a0 + i, 0, a_ring + i * kATileBytes, b_ring + i * B_BYTES, &full[i],
-                         kPartWeights);
-            }
-          }
-        }
-        griddep_wait();
-      }
       int tile, kb0, kb1;
       while (ok && cur.next(tile, kb0, kb1)) {
         P::prod_tile(p, tile, rank, st);
         for (int kb = kb0; kb < kb1; ++kb) {
-          const bool early = issued < pre;   // its weights and byte count are already out
-          if (!early) {
-            if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, p.status)) {
-              ok = false;
-              break;
-            }
-            if (!PAIR || rank == 0) mbar_arrive_expect_tx(&full[stage], P::stage_bytes(p, tile, kb));
+          if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, p.status)) {   // a fresh slot passes at once
+            ok = false;
+            break;
           }
-          const int part = early ? kPartAct : kPartAll;
-          if constexpr (PAIR) {
-            P::prod_kb(p, st, tile, kb, 0, a_ring + stage * kATileBytes, b_ring + stage * B_BYTES,
-                       leader_full + static_cast<uint32_t>(stage) * 8u, part);
-          } else {
-            P::prod_kb(p, st, tile, kb, 0, a_ring + stage * kATileBytes, b_ring + stage * B_BYTES, &full[stage], part);
+#pragma unroll
+          for (int j = 0; j < KSUB; ++j) {
+            const int k64 = kb * KSUB + j;
+            const int fb = stage * KSUB + j;
+            uint8_t* a_dst = a_ring + stage * A_BYTES + j * kATileBytes;
+            uint8_t* b_dst = b_ring + stage * B_BYTES + j * b_stage_bytes<P>();
+            if (!PAIR || rank == 0) mbar_arrive_expect_tx(&full[fb], P::stage_bytes(p, tile, k64, part));
+            if constexpr (PAIR) {
+              P::prod_kb(p, st, tile, k64, 0, a_dst, b_dst, leader_full + static_cast<uint32_t>(fb) * 8u, part);
+            } else {
+              P::prod_kb(p, st, tile, k64, 0, a_dst, b_dst, &full[fb], part);
+            }
           }
           ++issued;
           if (++stage == STAGES) {
@@ -408,7 +437,8 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1)
           unwind_pause(1000000ull);
         } else {
           for (long n = issued - 1; n >= 0 && n >= issued - STAGES; --n)
-            drain_wait(&full[n % STAGES], static_cast<uint32_t>((n / STAGES) & 1));
+            for (int j = 0; j < KSUB; ++j)
+              drain_wait(&full[(n % STAGES) * KSUB + j], static_cast<uint32_t>((n / STAGES) & 1));
         }
       }
     }
@@ -434,28 +464,37 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1)
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
         for (int kb = kb0; kb < kb1; ++kb) {
-          if (!mbar_wait(&full[stage], phase, abort_flag, p.status)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          const uint32_t a_base = smem_u32(a_ring + stage * kATileBytes);
+          const uint32_t a_base = smem_u32(a_ring + stage * A_BYTES);
           const uint32_t b_base = smem_u32(b_ring + stage * B_BYTES);
+          const int nsub = nk64 - kb * KSUB < KSUB ? nk64 - kb * KSUB : KSUB;   // K blocks in this slot
 #pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            const uint64_t adesc = sdesc_kmajor_sw128(a_base + k * 32);
-            const uint64_t bdesc = P::bdesc(b_base + k * P::kBStepBytes);
-            const uint32_t accumulate = ((kb - kb0) | k) != 0 ? 1u : 0u;
-            if (PAIR)
-              umma_bf16_pair(d_tmem, adesc, bdesc, IDESC, accumulate);
-            else
-              umma_bf16(d_tmem, adesc, bdesc, IDESC, accumulate);
+          for (int j = 0; j < KSUB; ++j) {
+            // Every K block of the slot was copied (the barrier phases stay in
+            // step); only those inside the contraction are multiplied.
+            if (!mbar_wait(&full[stage * KSUB + j], phase, abort_flag, p.status)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            if (j < nsub) {
+              issued_any = true;
+#pragma unroll
+              for (int k = 0; k < 4; ++k) {
+                const uint64_t adesc = sdesc_kmajor_sw128(a_base + j * kATileBytes + k * 32);
+                const uint64_t bdesc = P::bdesc(b_base + j * b_stage_bytes<P>() + k * P::kBStepBytes);
+                const uint32_t accumulate = ((kb - kb0) | j | k) != 0 ? 1u : 0u;
+                if (PAIR)
+                  umma_bf16_pair(d_tmem, adesc, bdesc, IDESC, accumulate);
+                else
+                  umma_bf16(d_tmem, adesc, bdesc, IDESC, accumulate);
+              }
+            }
           }
+          if (!ok) break;
           if (PAIR)
             umma_commit_pair_multicast(&empty[stage], kPairMask);   // frees the slot in both CTAs
           else
             umma_commit(&empty[stage]);
-          issued_any = true;
           if (++stage == STAGES) {
             stage = 0;
             phase ^= 1;
@@ -480,11 +519,11 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1)
       }
     }
     __syncwarp();
-  } else if (warp >= 2) {
+  } else if (warp >= kFirstEpiWarp) {
     // ---------------------------------------------------------------- epilogue
-    const int q = warp & 3;            // TMEM lane quadrant this warp may access
-    const int row = q * 32 + lane;     // accumulator row = TMEM lane
-    const int half = (warp - 2) >> 2;  // which half of the accumulator columns
+    const int q = warp & 3;                        // TMEM lane quadrant this warp may access
+    const int row = q * 32 + lane;                 // accumulator row = TMEM lane
+    const int half = (warp - kFirstEpiWarp) >> 2;  // which half of the accumulator columns
     EpiCtx ctx{epi_smem, rank, &half_bar[half], 0u, abort_flag, p.status};
     const uint32_t leader_tempty = PAIR ? mapa_shared(smem_u32(tempty), 0) : 0u;
     const long long sk_units = static_cast<long long>(ntiles - dp_tiles) * nkb;
@@ -522,7 +561,7 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1)
           // partial is copied into the (idle) ring, then added into TMEM.
           const long long tile_end = static_cast<long long>(tile - dp_tiles + 1) * nkb;
           constexpr uint32_t kHalfBytes = 128u * HALF_COLS * 4u;
-          static_assert(HALVES * kHalfBytes <= STAGES * (kATileBytes + B_BYTES), "partials fit in the ring");
+          static_assert(HALVES * kHalfBytes <= STAGES * (A_BYTES + B_BYTES), "partials fit in the ring");
           static_assert(kHalfBytes % 16384 == 0, "copied in 16 KB pieces");
           const float4* stage = reinterpret_cast<const float4*>(a_ring + half * kHalfBytes) + row * (HALF_COLS / 4);
           for (int s2 = slot + 1; ok && s2 < n_slots && sk_first_unit(sk_units, s2, n_slots) < tile_end; ++s2) {
@@ -606,9 +645,9 @@ inline unsigned long long next_stream_k_token() {
   return z | 1ull;
 }
 
-// Launches umma_gemm_kernel<P> over `tiles` cluster tiles of `nkb` K blocks
-// (the fewest the kernel may take, for a contraction length decided on the
-// device).  The persistent grid holds at most as many slots (clusters) as can
+// Launches umma_gemm_kernel<P> over `tiles` cluster tiles of `nkb` 64-wide
+// K blocks (the fewest the kernel may take, for a contraction length decided
+// on the device).  The persistent grid holds at most as many slots (clusters) as can
 // be resident at once; with a stream-K region the tiles may be split.
 template <class P>
 cudaError_t launch_gemm(const typename P::Params& p, int tiles, int nkb, const StreamKArea* area, int n_sm,
