@@ -49,6 +49,11 @@ struct GateUpProblemT {
   static constexpr int B_MN_MAJOR = 0;
   static constexpr int EPI_WARPS = EPI_WARPS_;
   static constexpr int kGroups = EPI_WARPS / 4;
+  // A group's SwiGLU reads the gate columns of its channels and the up
+  // columns 128 further on; with two groups each would read columns of the
+  // other group's half, which a stream-K owner fixes up only for its own
+  // half (and eight warps measured 3% slower anyway).
+  static_assert(EPI_WARPS == 4, "one epilogue group reads both accumulator halves");
   static constexpr int CLUSTER = 2;
   static constexpr uint32_t kBStepBytes = 32;
   static constexpr uint32_t kBoxBytes = 128 * 128;          // 128 rows x 64 bf16

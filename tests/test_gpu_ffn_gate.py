@@ -53,6 +53,7 @@ def _check_gate(X, Wg, Wu, WdT, chan, delta, got_sal_perm, got_leak, got_flag, p
 
 
 @pytest.mark.parametrize("M,d,I,C,delta,zero", [(300, 256, 1024, 768, 0.15, False), (300, 256, 1024, 768, 0.99, False),
+                                                (300, 320, 1024, 576, 0.99, False),
                                                 (129, 512, 2048, 1024, 0.15, True), (1, 256, 512, 256, 0.5, False),
                                                 (2348, 1536, 8960, 6720, 0.15, False)])
 def test_gated_ffn_matches_oracle(M, d, I, C, delta, zero):

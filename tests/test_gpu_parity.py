@@ -145,6 +145,12 @@ def _score_case(name):
         inp = dict(h=bf((B, N, d), 1), W1=bf((Hc, d), d ** -.5), w2=rng.normal(0, Hc ** -.5, Hc).astype(np.float32),
                    b1=rng.normal(0, .1, Hc).astype(np.float32), t=np.zeros(B, np.float32))
         return inp, 0
+    if name == "und_odd_d":
+        # d / 64 odd: the last ring slot of two K blocks is half past the contraction
+        B, N, d, Hc = 2, 200, 320, 128
+        inp = dict(h=bf((B, N, d), 1), W1=bf((Hc, d), d ** -.5), w2=rng.normal(0, Hc ** -.5, Hc).astype(np.float32),
+                   b1=rng.normal(0, .1, Hc).astype(np.float32), t=np.zeros(B, np.float32))
+        return inp, 0
     if name in ("gen_segments", "gen_segments_noU"):
         B, N, d, Hc, He, E, S = 4, 130, 384, 192, 128, 32, 4
         inp = dict(h=bf((B, N, d), 1), W1=bf((Hc, d), d ** -.5), w2=rng.normal(0, Hc ** -.5, Hc).astype(np.float32),
@@ -161,7 +167,7 @@ def _oracle_logits(inp, task):
                      inp.get("w2e"), inp.get("Ue"), inp.get("b1e"))
 
 
-@pytest.mark.parametrize("name", ["tiny", "und_ragged_bias", "gen_segments", "gen_segments_noU"])
+@pytest.mark.parametrize("name", ["tiny", "und_ragged_bias", "und_odd_d", "gen_segments", "gen_segments_noU"])
 def test_score_matches_oracle(name):
     inp, task = _score_case(name)
     B, N, d = inp["h"].shape
@@ -184,6 +190,7 @@ def test_score_matches_oracle(name):
 # (129, 1536, ...) and (200, 4096, ...), the gate/up GEMM of (1000, 1792, ...),
 # and both GEMMs of (100, 3584, ...) (one-CTA down tiles, ragged rows).
 @pytest.mark.parametrize("M,d,I,C,pruned", [(1, 256, 1024, 512, True), (127, 256, 1024, 512, True),
+                                            (65, 320, 640, 576, True),
                                             (300, 512, 640, 640, False), (129, 1536, 8960, 6720, True),
                                             (1000, 1792, 1536, 960, True), (2000, 2560, 4096, 4096, False),
                                             (200, 4096, 10240, 10240, False), (100, 3584, 18944, 4736, True)])
