@@ -3,9 +3,12 @@
 // monotonic, App. B.2).
 //
 // One 1024-thread CTA per sequence keeps the N order-preserving 32-bit keys in
-// shared memory.  A four-pass MSB-first radix select (8-bit digits, shared
-// histograms) finds the K-th largest routable key T and how many tokens equal
-// to T must be taken.  Each warp then owns a contiguous run of tokens, read 32
+// shared memory.  An MSB-first radix select (8-bit digits, shared histograms)
+// finds the K-th largest routable key T and how many tokens equal to T must
+// be taken; as soon as at most 32 routable keys share the digits found so
+// far, one warp ranks those candidates exactly and the remaining passes are
+// skipped (real-valued logits get there after one or two passes, heavy ties
+// take all four).  Each warp then owns a contiguous run of tokens, read 32
 // at a time (a token per lane, no bank conflicts): ballots rank every tie
 // (lowest index first) and every kept token, and two scans over the warps'
 // counts place them, so the kept list comes out in ascending token order with
@@ -114,7 +117,8 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(TopkArgs a) {
   __shared__ uint32_t hist[256];
   __shared__ uint32_t sub[kSubHist][256];
   __shared__ uint32_t warp_tot[32];
-  __shared__ uint32_t s_prefix, s_remaining;
+  __shared__ uint32_t s_prefix, s_remaining, s_count, s_ncand;
+  __shared__ uint32_t s_cand[32];
   __shared__ int s_nan;
   __shared__ uint32_t s_ballot[kTopkThreads / 32][kMaxSteps];
 
@@ -122,7 +126,10 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(TopkArgs a) {
   const int b = blockIdx.x;
   const int N = a.N;
   const size_t base = static_cast<size_t>(b) * N;
-  if (tid == 0) s_nan = 0;
+  if (tid == 0) {
+    s_nan = 0;
+    s_ncand = 0;
+  }
   __syncthreads();
 
   // 1. logits (reduced from partial sums in chunk order) -> keys
@@ -185,6 +192,7 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(TopkArgs a) {
           if (cum < remaining && cum + local[j] >= remaining) {
             s_prefix = prefix | (static_cast<uint32_t>(8 * lane + j) << shift);
             s_remaining = remaining - cum;
+            s_count = local[j];
           }
           cum += local[j];
         }
@@ -193,6 +201,37 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(TopkArgs a) {
       prefix = s_prefix;
       remaining = s_remaining;
       pmask |= 255u << shift;
+      if (shift > 0 && s_count <= 32u) {
+        // Few routable keys share the digits found so far (the usual case
+        // for real-valued logits after one or two passes): gather them and
+        // let one warp rank them exactly instead of running the remaining
+        // passes.  The threshold is the candidate with fewer than
+        // `remaining` larger candidates and at least `remaining` larger or
+        // equal ones; need_eq is what is left of `remaining` above it.
+        for (int i = a.r0 + tid; i < a.r1; i += blockDim.x) {
+          const uint32_t k = keys[i];
+          if ((k & pmask) == prefix) s_cand[atomicAdd(&s_ncand, 1u)] = k;
+        }
+        __syncthreads();
+        if (tid < 32) {
+          const uint32_t n = s_ncand;
+          const uint32_t k = tid < static_cast<int>(n) ? s_cand[tid] : 0u;
+          uint32_t gt = 0, ge = 0;
+          for (uint32_t j = 0; j < n; ++j) {
+            const uint32_t o = s_cand[j];
+            gt += o > k ? 1u : 0u;
+            ge += o >= k ? 1u : 0u;
+          }
+          if (tid < static_cast<int>(n) && gt < remaining && ge >= remaining) {
+            s_prefix = k;                 // lanes holding equal keys write equal values
+            s_remaining = remaining - gt;
+          }
+        }
+        __syncthreads();
+        prefix = s_prefix;
+        remaining = s_remaining;
+        break;
+      }
     }
     thr = prefix;
     need_eq = remaining;
