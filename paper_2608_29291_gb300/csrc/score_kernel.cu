@@ -246,8 +246,10 @@ int score_max_partials(int Hc, int He, int gen) {
   return 2 * (Hc + (gen ? He : 0)) / 64;
 }
 
-// Chunk width for a launch: the widest that still gives every SM a tile,
-// else the narrowest available (more, smaller tiles).
+// Chunk width for a launch: the widest whose tiles fill at least ~90% of a
+// wave, else the narrowest available (more, smaller tiles).  Generation at
+// B = 8, N = 1088 (144 tiles of 256 hidden units on 152 SMs) measured 2 us
+// faster as one 256-wide wave than as two waves of 128-wide tiles.
 static int pick_chunk_width(const ScoreArgs& a, int n_sm) {
   const int Ht = a.Hc + (a.gen ? a.He : 0);
   const long rows = static_cast<long>(a.B) * ((a.N + 127) / 128);
@@ -255,7 +257,7 @@ static int pick_chunk_width(const ScoreArgs& a, int n_sm) {
   for (int bn : {256, 128, 64}) {
     if (a.Hc % bn != 0 || (a.gen && a.He % bn != 0)) continue;
     best = bn;
-    if (rows * (Ht / bn) >= n_sm) return bn;
+    if (10 * rows * (Ht / bn) >= 9 * static_cast<long>(n_sm)) return bn;   // at least ~90% of a wave
   }
   return best;
 }
