@@ -52,7 +52,7 @@
 //
 // When every slot is busy these contractions are bound by L2 bandwidth (the
 // K-block rate per slot drops as slots are added), so splitting only pays
-// where a last wave would leave most slots idle; see stream_k_dp_tiles.
+// where a last wave would leave most slots idle; see stream_k_plan.
 //
 // Slots, barriers and threads, as measured on GB300 (globaltimer traces of
 // the FFN GEMMs):
@@ -103,10 +103,10 @@
 #include <atomic>
 
 namespace cer {
-// Parts of a stage's copies (prod_kb).
+// Parts of a K block's copies (prod_kb, stage_bytes): each producer thread
+// issues one of them.
 constexpr int kPartAct = 1;       // the A operand, produced by the previous kernel
 constexpr int kPartWeights = 2;   // the B operand, static weights
-constexpr int kPartAll = kPartAct | kPartWeights;
 }
 
 #include "kernels.h"
