@@ -2,11 +2,15 @@
 """Benchmark of the routed block (score -> top-K -> gather -> pruned SwiGLU FFN
 -> scatter-add) on GB300, one JSON line on stdout (rank 0).
 
-  python bench.py [--gpus N] [--steps K] [--warmup W] [--config und_1p5b]
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--config long_7b] [--quick]
   python bench.py --impl reference ...      # the CPU oracle on the same workload
+  python bench.py --sweep                   # the 7B sweep grid, one line per point
 
 A step is one cer_routed_block call (in place on the residual stream h) over
-the whole synthetic batch of the workload, inputs resident in HBM.  Between
+the whole synthetic batch of the workload, inputs resident in HBM.  The
+headline workload is the largest config, long_7b (B = 2, N = 4096, d = 3584);
+the line also carries the other full-size configs (und_1p5b, gen_1p5b) and a
+summary of the whole 7B sweep grid, each stage against its roofline.  Between
 timed steps, outside the timed interval, h is restored from a pristine copy
 and L2 is flushed (a 256 MiB write); each step is timed with CUDA events on
 the launching stream.  For N > 1 each
@@ -332,6 +336,207 @@ def run_reference(args, info):
 
 # ------------------------------------------------------------------ GPU arm
 
+def _bf(torch, dev, bits):
+    import numpy as _np
+    return torch.from_numpy(_np.ascontiguousarray(bits).view(_np.int16)).view(torch.bfloat16).to(dev)
+
+
+def _f32(torch, dev, a):
+    return None if a is None else torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(dev)
+
+
+class BlockSetup:
+    """One workload's tensors on the device: scorers, h (and a pristine copy,
+    restored before every step since the block updates h in place), t, the FFN
+    weights as kept-channel slices packed once (the static mask of App. A.4, as
+    at model load) and the block's workspace."""
+
+    def __init__(self, torch, cer, w, inp, dev, full_ffn=None):
+        self.w = w
+        bf = lambda bits: _bf(torch, dev, bits)  # noqa: E731
+        f32 = lambda a: _f32(torch, dev, a)       # noqa: E731
+        self.core = cer.Scorer(W1=bf(inp["W1"]), w2=f32(inp["w2"]), b1=f32(inp.get("b1")))
+        self.exp = None
+        if w.task == 1:
+            self.exp = cer.Scorer(W1=bf(inp["W1e"]), w2=f32(inp["w2e"]),
+                                  U=bf(inp["Ue"]) if inp.get("Ue") is not None else None)
+        self.h = bf(inp["h"])
+        self.h0 = self.h.clone()
+        self.t = f32(inp["t"])
+        Wg, Wu, WdT = full_ffn if full_ffn is not None else (bf(inp["Wg"]), bf(inp["Wu"]), bf(inp["WdT"]))
+        self.pack_ms = None
+        if w.C < w.I:
+            chan = torch.from_numpy(inp["chan"]).to(dev)
+            cer.pack_ffn_weights(Wg, Wu, WdT, chan)            # warm
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            Wg, Wu, WdT = cer.pack_ffn_weights(Wg, Wu, WdT, chan)
+            e1.record()
+            torch.cuda.synchronize(dev)
+            self.pack_ms = e0.elapsed_time(e1)
+        self.Wg, self.Wu, self.WdT = Wg, Wu, WdT
+        self.ws = cer.workspace(cer.cer_routed_block_workspace_size(w.B, w.N, w.d, w.Hc, w.He if w.task else 0,
+                                                                    w.task, w.r0, w.r1, w.K, w.C, False), dev)
+
+    def step(self, cer, stream, stage_events=None):
+        w = self.w
+        cer.cer_routed_block(self.h, self.core, self.exp, self.t, w.task, w.r0, w.r1, w.K, self.Wg, self.Wu,
+                             self.WdT, None, ws=self.ws, stage_events=stage_events, stream=stream)
+
+
+def prepare_step(torch, setup, flush, i):
+    """Outside the timed interval: restore h (the block updates it in place),
+    evict L2 with a 256 MiB write so the step reads its inputs from HBM, and
+    keep the GPU busy (a short spin) while the host enqueues the step, so host
+    launch latency is not counted as device time."""
+    setup.h.copy_(setup.h0)
+    flush.fill_(float(i))
+    torch.cuda._sleep(200000)
+
+
+def time_block(torch, cer, setup, flush, stream, steps, warmup, n_stage, clocks=None, dist=None, dev=None):
+    """W warm-up steps, then K steps each bracketed by CUDA events on the
+    launching stream (no event between the kernels, so programmatic dependent
+    launch overlaps them as in production); then a separate pass of n_stage
+    steps with the library's stage events between kernels (serialised) for
+    the per-stage times.  Returns (per-step ms, per-stage mean ms [5])."""
+    for i in range(warmup):
+        prepare_step(torch, setup, flush, i)
+        setup.step(cer, stream)
+    cer.cer_sync_status(stream)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    if clocks is not None:
+        clocks.start()
+        time.sleep(0.3)
+    runtime.barrier(dist)
+    torch.cuda.synchronize(dev)
+    for i in range(steps):
+        prepare_step(torch, setup, flush, i)
+        ev[i][0].record(stream)
+        setup.step(cer, stream)
+        ev[i][1].record(stream)
+    torch.cuda.synchronize(dev)
+    runtime.barrier(dist)
+    if clocks is not None:
+        clocks.stop()
+    cer.cer_sync_status(stream)
+    step_ms = np.array([a.elapsed_time(b) for a, b in ev])
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(n_stage)]
+    for i in range(n_stage):
+        prepare_step(torch, setup, flush, i)
+        setup.step(cer, stream, evs[i])
+    torch.cuda.synchronize(dev)
+    cer.cer_sync_status(stream)
+    stage = np.array([[e[j].elapsed_time(e[j + 1]) for j in range(5)] for e in evs]).mean(axis=0)
+    return step_ms, stage
+
+
+STAGES = ("score", "topk", "gather", "ffn_gateup", "ffn_down_scatter")
+
+
+def stage_report(w: gen.Workload, stage_ms, peaks) -> dict:
+    """Each serialised stage against its own roofline: the algorithmic bytes
+    and flops of the stage (not what the kernels happen to move), the time
+    they need at the measured HBM bandwidth and at the bf16 burst peak, the
+    larger of the two as the bound, and bound / measured as the fraction."""
+    bw = float(peaks["hbm_gbs"]) * 1e9
+    pk = float(peaks["bf16_tflops"]) * 1e12
+    Ht = w.Hc + (w.He if w.task == 1 else 0)
+    M, d, C, BN = w.M, w.d, w.C, w.B * w.N
+    work = {
+        # reads h once (+ the scorer weights); 2 B N d Ht flop
+        "score": (2.0 * BN * d + 2.0 * Ht * d, 2.0 * BN * d * Ht),
+        # reads the logits, writes the keep list
+        "topk": (4.0 * BN + 4.0 * M, 0.0),
+        # kept rows in and out, plus the keep list
+        "gather": (4.0 * M * d + 4.0 * M, 0.0),
+        # packed rows, gate and up slices in; act out
+        "ffn_gateup": (2.0 * M * d + 4.0 * C * d + 2.0 * M * C, 4.0 * M * d * C),
+        # act and down slice in; kept rows of h read and written
+        "ffn_down_scatter": (2.0 * M * C + 2.0 * C * d + 4.0 * M * d, 2.0 * M * d * C),
+    }
+    out = {}
+    for name, t_ms in zip(STAGES, stage_ms):
+        nbytes, flops = work[name]
+        t = float(t_ms) * 1e-3
+        t_hbm, t_tc = nbytes / bw, flops / pk
+        bound = "tensor" if t_tc > t_hbm else "hbm"
+        r = {"us": round(t * 1e6, 2), "bound": bound, "frac": round(max(t_hbm, t_tc) / t, 4) if t > 0 else None,
+             "gbs": round(nbytes / t / 1e9, 1) if t > 0 else None}
+        if flops:
+            r["tflops"] = round(flops / t / 1e12, 1) if t > 0 else None
+        out[name] = r
+    t_ffn = (float(stage_ms[3]) + float(stage_ms[4])) * 1e-3
+    ffn_b = work["ffn_gateup"][0] + work["ffn_down_scatter"][0] - 2.0 * M * C * 2   # act stays on chip in the bound
+    ffn_f = work["ffn_gateup"][1] + work["ffn_down_scatter"][1]
+    out["ffn"] = {"us": round(t_ffn * 1e6, 2), "bound": "tensor" if ffn_f / pk > ffn_b / bw else "hbm",
+                  "frac": round(max(ffn_f / pk, ffn_b / bw) / t_ffn, 4), "tflops": round(ffn_f / t_ffn / 1e12, 1)}
+    return out
+
+
+SWEEP_N = (1024, 2048, 4096, 8192, 16384)
+SWEEP_R = (0.1, 0.3, 0.5, 0.7, 0.9)
+SWEEP_F = (0.25, 0.5, 1.0)
+
+
+def sweep_points(torch, cer, dev, flush, stream, peaks, steps=5, warmup=3, ffn_bits=None):
+    """The 7B sweep (B = 1, d = 3584, I = 18944, all routable, generation) on
+    the whole grid N x token keep ratio x FFN keep ratio.  The inputs of every
+    point are those of gen.sweep(N, r, f) (h, scorer weights and t depend on
+    N only; the channel keep set on the FFN ratio only), so each N's tensors
+    and each ratio's packed weight slices are made once.  Yields one dict per
+    point: the whole step (L2 flushed between steps) and every stage against
+    its roofline."""
+    if ffn_bits is None:    # the FFN weights of (seed 0, I = 18944, d = 3584), drawn once
+        base = gen.make_inputs(gen.sweep(SWEEP_N[0], 0.5, 1.0))
+        ffn_bits = (base["Wg"], base["Wu"], base["WdT"])
+    full = tuple(_bf(torch, dev, x) for x in ffn_bits)
+    packed = {}
+    for f in SWEEP_F:
+        w = gen.sweep(SWEEP_N[0], 0.5, f)
+        if w.C < w.I:
+            chan = torch.from_numpy(gen.channel_keep_set(w.seed, "chan", w.I, w.C)).to(dev)
+            packed[f] = cer.pack_ffn_weights(*full, chan)
+        else:
+            packed[f] = full
+    for n in SWEEP_N:
+        inp = gen.make_inputs(gen.sweep(n, 0.5, 1.0), ffn_weights=ffn_bits)
+        setup = BlockSetup(torch, cer, gen.sweep(n, 0.5, 1.0), inp, dev, full_ffn=full)
+        for r in SWEEP_R:
+            for f in SWEEP_F:
+                w = gen.sweep(n, r, f)
+                setup.w = w
+                setup.Wg, setup.Wu, setup.WdT = packed[f]
+                setup.ws = cer.workspace(cer.cer_routed_block_workspace_size(w.B, w.N, w.d, w.Hc, w.He, w.task,
+                                                                             w.r0, w.r1, w.K, w.C, False), dev)
+                step_ms, stage = time_block(torch, cer, setup, flush, stream, steps, warmup, steps, dev=dev)
+                ms = float(step_ms.mean())
+                yield {"N": n, "token_ratio": r, "ffn_ratio": f, "K": w.K, "M": w.M, "C": w.C,
+                       "ms_per_step": round(ms, 4), "tokens_per_s": w.B * w.N / (ms * 1e-3),
+                       "stages": stage_report(w, stage, peaks)}
+        del setup
+    del full, packed
+
+
+def sweep_summary(points) -> dict:
+    """min / median / max over the sweep's points of every stage's roofline
+    fraction (and of the whole step's tokens/s)."""
+    out = {"points": len(points),
+           "grid": {"N": list(SWEEP_N), "token_ratio": list(SWEEP_R), "ffn_ratio": list(SWEEP_F)}}
+    for name in STAGES + ("ffn",):
+        fr = np.array([p["stages"][name]["frac"] for p in points], dtype=np.float64)
+        out[f"{name}_frac"] = {"min": round(float(fr.min()), 4), "median": round(float(np.median(fr)), 4),
+                               "max": round(float(fr.max()), 4)}
+    tps = np.array([p["tokens_per_s"] for p in points])
+    out["tokens_per_s"] = {"min": float(tps.min()), "median": float(np.median(tps)), "max": float(tps.max())}
+    out["per_point"] = [[p["N"], p["token_ratio"], p["ffn_ratio"], p["ms_per_step"],
+                         [p["stages"][k]["us"] for k in STAGES], [p["stages"][k]["frac"] for k in STAGES],
+                         p["stages"]["ffn"]["frac"]] for p in points]
+    out["per_point_fields"] = ["N", "token_ratio", "ffn_ratio", "ms_per_step", "stage_us (" + ", ".join(STAGES) + ")",
+                               "stage_frac", "ffn_frac"]
+    return out
+
+
 def run_gpu(args, info):
     import torch
     from paper_2608_29291_gb300 import cer
@@ -340,94 +545,27 @@ def run_gpu(args, info):
     dev = torch.device("cuda", info.local_rank)
     dist = runtime.init_group(info, "nccl")
     cer.load()
+    peaks, peak_kind = load_peaks()
+    flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
 
     base = gen.WORKLOADS[args.config]()
     w = gen.Workload(**{**base.__dict__, "seed": runtime.replica_seed(base.seed, info.rank)})
     inp = gen.make_inputs(w)
-
-    def bf(bits):
-        return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).to(dev)
-
-    def f32(a):
-        return None if a is None else torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(dev)
-
-    core = cer.Scorer(W1=bf(inp["W1"]), w2=f32(inp["w2"]), b1=f32(inp.get("b1")))
-    exp = None
-    if w.task == 1:
-        exp = cer.Scorer(W1=bf(inp["W1e"]), w2=f32(inp["w2e"]), U=bf(inp["Ue"]) if inp.get("Ue") is not None else None)
-    h = bf(inp["h"])
-    h0 = h.clone()          # pristine residual stream, restored before every step
-    t = f32(inp["t"])
-    Wg, Wu, WdT = bf(inp["Wg"]), bf(inp["Wu"]), bf(inp["WdT"])
-    pack_ms = None
-    if w.C < w.I:
-        # the static channel mask (one per layer) applied once, as at model load
-        chan_full = torch.from_numpy(inp["chan"]).to(dev)
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        cer.pack_ffn_weights(Wg, Wu, WdT, chan_full)            # warm
-        e0.record()
-        Wg, Wu, WdT = cer.pack_ffn_weights(Wg, Wu, WdT, chan_full)
-        e1.record()
-        torch.cuda.synchronize(dev)
-        pack_ms = e0.elapsed_time(e1)
+    S = BlockSetup(torch, cer, w, inp, dev)
+    core, exp, h, h0, t = S.core, S.exp, S.h, S.h0, S.t
+    Wg, Wu, WdT, ws = S.Wg, S.Wu, S.WdT, S.ws
     chan = None
-    ws = cer.workspace(cer.cer_routed_block_workspace_size(w.B, w.N, w.d, w.Hc, w.He if w.task else 0, w.task,
-                                                           w.r0, w.r1, w.K, w.C, False), dev)
-    flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
-    stream = torch.cuda.current_stream(dev)
 
-    def step(stage_events=None):
-        cer.cer_routed_block(h, core, exp, t, w.task, w.r0, w.r1, w.K, Wg, Wu, WdT, chan, ws=ws,
-                             stage_events=stage_events, stream=stream)
-
-    def prepare(i):
-        """Outside the timed interval: restore h (the block updates it in place),
-        evict L2 with a 256 MiB write so the step reads its inputs from HBM, and
-        keep the GPU busy (a short spin) while the host enqueues the step, so
-        host launch latency is not counted as device time."""
-        h.copy_(h0)
-        flush.fill_(float(i))
-        torch.cuda._sleep(200000)
-
-    for i in range(args.warmup):
-        prepare(i)
-        step()
-    cer.cer_sync_status(stream)
-
-    # ---- device-timed region: K steps, L2 flushed between steps; events only
-    # around each whole step so consecutive kernels overlap as in production
-    # (programmatic dependent launch)
-    step_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    # ---- device-timed region: K steps, L2 flushed between steps
     clocks = ClockSampler(smi_index(info.local_rank))
-    clocks.start()
-    time.sleep(0.3)
-    runtime.barrier(dist)
-    torch.cuda.synchronize(dev)
-    for i in range(args.steps):
-        prepare(i)
-        step_ev[i][0].record(stream)
-        step()
-        step_ev[i][1].record(stream)
-    torch.cuda.synchronize(dev)
-    runtime.barrier(dist)
-    clocks.stop()
-    cer.cer_sync_status(stream)
-    step_ms = np.array([a.elapsed_time(b) for a, b in step_ev])
+    n_stage = max(3, min(args.steps, 50))
+    step_ms, stage = time_block(torch, cer, S, flush, stream, args.steps, args.warmup, n_stage, clocks=clocks,
+                                dist=dist, dev=dev)
     mean_ms = float(step_ms.mean())
     slow_ms = runtime.max_over_ranks(dist, mean_ms, device=dev)
     tokens = w.B * w.N * info.world
     value = tokens / (slow_ms * 1e-3)
-
-    # ---- per-stage breakdown (a separate pass: events between the kernels
-    # serialise them, so each stage is timed alone)
-    n_stage = max(3, min(args.steps, 50))
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(n_stage)]
-    for i in range(n_stage):
-        prepare(i)
-        step(evs[i])
-    torch.cuda.synchronize(dev)
-    cer.cer_sync_status(stream)
-    stage = np.array([[e[j].elapsed_time(e[j + 1]) for j in range(5)] for e in evs])   # ms
 
     # ---- end to end through the public API: pinned host h in, h out.  Every
     # step uploads its own h (and t) from pinned host memory, runs the block,
@@ -435,12 +573,12 @@ def run_gpu(args, info):
     # the uploads and downloads of neighbouring steps with the compute, as a
     # serving loop would (with two buffers a buffer's upload, compute and
     # download run back to back every two steps, which the host link -- about
-    # 190 GB/s each way, 315 GB/s both ways together on GB300 -- cannot hide).  Instead of an L2 flush inside the timed loop, consecutive
-    # steps take different copies of the scorer and FFN weights (as the layers
-    # of a model would), so many that the copies a step does not use exceed
-    # the flush size: every step reads its weights from HBM.  The serialised
-    # time of one step (upload, compute, download back to back) is reported
-    # beside it.
+    # 190 GB/s each way, 315 GB/s both ways together on GB300 -- cannot hide).
+    # Instead of an L2 flush inside the timed loop, consecutive steps take
+    # different copies of the scorer and FFN weights (as the layers of a model
+    # would), so many that the copies a step does not use exceed the flush
+    # size: every step reads its weights from HBM.  The serialised time of one
+    # step (upload, compute, download back to back) is reported beside it.
     set_bytes = sum(x.numel() * x.element_size() for x in (Wg, Wu, WdT))
     n_sets = 1 + -(-FLUSH_BYTES // set_bytes)
 
@@ -510,19 +648,42 @@ def run_gpu(args, info):
         raise RuntimeError("end-to-end steps on the same input disagree")
     h2d = h_host.numel() * 2 + t_host.numel() * 4
     d2h = out_host[0].numel() * 2
+    del layers, h_buf, out_host
 
     # ---- UCS statistics on this step's tensors (Sec. 3.4): drop-set J/RDA of
     # two keep masks, redundancy gap of the block's input and output
     ucs = measure_ucs(cer, torch, w, h0, h, flush, stream, dev, core, exp, t, Wg, Wu, WdT, ws, inp)
-    peaks, peak_kind = load_peaks()
     # ---- attention on the packed sequence (Sec. 3.4): rotary embedding and
     # softmax attention over the retained tokens, with the backbone's heads
     attn = measure_attention(cer, torch, w, flush, stream, dev, float(peaks["bf16_tflops"]))
+    pack_ms = S.pack_ms
+    del S
+
+    # ---- the other full-size configs (each its own step, stages and
+    # roofline fractions) and the whole 7B sweep grid, on rank 0 only
+    others, sweep = {}, None
+    if info.is_root and not args.quick:
+        for name in ("und_1p5b", "gen_1p5b", "long_7b"):
+            if name == args.config:
+                continue
+            wo = gen.WORKLOADS[name]()
+            so = BlockSetup(torch, cer, wo, gen.make_inputs(wo), dev)
+            sm, st = time_block(torch, cer, so, flush, stream, max(5, min(args.steps, 20)), 3,
+                                max(5, min(args.steps, 20)), dev=dev)
+            others[name] = {"workload": wo.name, "B": wo.B, "N": wo.N, "d": wo.d, "kept_rows": wo.M,
+                            "kept_channels": wo.C, "ms_per_step": float(sm.mean()),
+                            "tokens_per_s": wo.B * wo.N / (float(sm.mean()) * 1e-3),
+                            "stages": stage_report(wo, st, peaks)}
+            del so
+        s7 = gen.sweep(SWEEP_N[0], 0.5, 1.0)
+        same = (w.seed, w.I, w.d) == (s7.seed, s7.I, s7.d)
+        sweep = sweep_summary(list(sweep_points(torch, cer, dev, flush, stream, peaks,
+                                                ffn_bits=(inp["Wg"], inp["Wu"], inp["WdT"]) if same else None)))
 
     if not info.is_root:
         return 0
 
-    score_ms, topk_ms, gather_ms, gateup_ms, down_ms = (float(x) for x in stage.mean(axis=0))
+    score_ms, topk_ms, gather_ms, gateup_ms, down_ms = (float(x) for x in stage)
     gateup_flops = 4.0 * w.M * w.d * w.C
     achieved = gateup_flops / (gateup_ms * 1e-3) / 1e12
     peak = float(peaks["bf16_tflops"])
@@ -548,6 +709,7 @@ def run_gpu(args, info):
                      "traffic": profiled_traffic(w.name)},
         "stages_ms": {"score": score_ms, "topk": topk_ms, "gather": gather_ms, "ffn_gateup": gateup_ms,
                       "ffn_down_scatter": down_ms},
+        "stages": stage_report(w, stage, peaks),
         "gather_gbs": gather_bytes / (gather_ms * 1e-3) / 1e9,
         "ffn_weights": "kept-channel slices packed once from the full weights by cer_pack_ffn_weights "
                        f"(static mask; {pack_ms:.3f} ms, not part of a step)" if pack_ms is not None else
@@ -567,6 +729,9 @@ def run_gpu(args, info):
         "ucs": {**ucs, "redundancy_gap_hbm_frac": ucs["redundancy_gap_gbs"] / float(peaks["hbm_gbs"]),
                 "peak_source": f"hbm_gbs of {peak_kind}"},
         "attention": {**attn, "rope_hbm_frac": attn["rope_gbs"] / float(peaks["hbm_gbs"])},
+        "other_configs": others or None,
+        "sweep_7b": sweep,
+        "stage_peaks": f"hbm_gbs and bf16_tflops (burst) of {peak_kind}",
         "gpu_launches": kernels_per_step(w.task) * args.steps,
         "stage_pass": f"per-stage times from a separate pass of {n_stage} steps with events between kernels",
         "clocks": clocks.summary(),
@@ -575,15 +740,8 @@ def run_gpu(args, info):
     return 0
 
 
-SWEEP_POINTS = [(n, r, f) for n in (1024, 4096, 16384) for r in (0.1, 0.5, 0.9) for f in (0.25, 1.0)]
-
-
 def run_sweep(args):
-    """The 7B sweep (B = 1, N in 1K..16K, all routable, generation): one JSON
-    line per (N, token keep ratio, channel keep ratio) point with the whole
-    step time and the FFN stages against their own bound -- the weight stream
-    from HBM for small M, the tensor pipe for large M (the FFN's arithmetic
-    intensity is about M flop per byte)."""
+    """The 7B sweep on the whole grid, one JSON line per point."""
     import torch
     from paper_2608_29291_gb300 import cer
 
@@ -591,95 +749,28 @@ def run_sweep(args):
     torch.cuda.set_device(dev)
     cer.load()
     peaks, peak_kind = load_peaks()
-    peak_tf = float(peaks["bf16_tflops"])
-    peak_gbs = float(peaks["hbm_gbs"])
-
-    def bf(bits):
-        return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).to(dev)
-
-    def f32(a):
-        return None if a is None else torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(dev)
-
-    base = gen.make_inputs(gen.sweep(max(n for n, _, _ in SWEEP_POINTS), 0.5, 1.0))
-    ffn = (base["Wg"], base["Wu"], base["WdT"])
-    Wg_full, Wu_full, WdT_full = bf(ffn[0]), bf(ffn[1]), bf(ffn[2])
     flush = torch.empty(FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream(dev)
-    for n, r, f in SWEEP_POINTS:
-        w = gen.sweep(n, r, f)
-        inp = gen.make_inputs(w, ffn_weights=ffn)
-        core = cer.Scorer(W1=bf(inp["W1"]), w2=f32(inp["w2"]), b1=f32(inp.get("b1")))
-        exp = cer.Scorer(W1=bf(inp["W1e"]), w2=f32(inp["w2e"]), U=bf(inp["Ue"]) if inp.get("Ue") is not None else None)
-        h = bf(inp["h"])
-        h0 = h.clone()
-        t = f32(inp["t"])
-        if w.C < w.I:
-            Wg, Wu, WdT = cer.pack_ffn_weights(Wg_full, Wu_full, WdT_full, torch.from_numpy(inp["chan"]).to(dev))
-        else:
-            Wg, Wu, WdT = Wg_full, Wu_full, WdT_full
-        ws = cer.workspace(cer.cer_routed_block_workspace_size(w.B, w.N, w.d, w.Hc, w.He, w.task, w.r0, w.r1, w.K,
-                                                               w.C, False), dev)
-
-        def step(stage_events=None):
-            cer.cer_routed_block(h, core, exp, t, w.task, w.r0, w.r1, w.K, Wg, Wu, WdT, None, ws=ws,
-                                 stage_events=stage_events, stream=stream)
-
-        def prepare(i):
-            h.copy_(h0)
-            flush.fill_(float(i))
-            torch.cuda._sleep(200000)
-
-        for i in range(args.warmup):
-            prepare(i)
-            step()
-        cer.cer_sync_status(stream)
-        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
-        for i in range(args.steps):
-            prepare(i)
-            ev[i][0].record(stream)
-            step()
-            ev[i][1].record(stream)
-        torch.cuda.synchronize(dev)
-        step_ms = float(np.mean([a.elapsed_time(b) for a, b in ev]))
-        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(args.steps)]
-        for i in range(args.steps):
-            prepare(i)
-            step(evs[i])
-        torch.cuda.synchronize(dev)
-        cer.cer_sync_status(stream)
-        stage = np.array([[e[j].elapsed_time(e[j + 1]) for j in range(5)] for e in evs]).mean(axis=0)   # ms
-        M = w.B * (w.K + w.N - (w.r1 - w.r0))
-        ffn_s = (stage[3] + stage[4]) * 1e-3
-        flops = 6.0 * M * w.d * w.C
-        wbytes = 6.0 * w.d * w.C
-        t_tensor = flops / (peak_tf * 1e12)
-        t_hbm = (wbytes + 4.0 * M * w.d) / (peak_gbs * 1e9)
-        bound = "tensor" if t_tensor >= t_hbm else "hbm"
-        line = {"sweep_point": w.name, "N": w.N, "K": w.K, "M": M, "C": w.C, "ms_per_step": step_ms,
-                "tokens_per_s": w.B * w.N / (step_ms * 1e-3),
-                "stages_us": {k: round(v * 1e3, 2) for k, v in zip(("score", "topk", "gather", "ffn_gateup",
-                                                                     "ffn_down_scatter"), stage)},
-                "ffn_bound": bound, "ffn_tflops": flops / ffn_s / 1e12,
-                "ffn_weight_gbs": (wbytes + 4.0 * M * w.d) / ffn_s / 1e9,
-                "ffn_frac": (t_tensor if bound == "tensor" else t_hbm) / ffn_s,
-                "peak_source": f"bf16_tflops (burst) / hbm_gbs of {peak_kind}",
-                "steps": args.steps, "warmup": args.warmup, "l2": "flushed between timed steps"}
-        print(json.dumps(line), flush=True)
-        del h, h0, ws, Wg, Wu, WdT
+    for p in sweep_points(torch, cer, dev, flush, stream, peaks, steps=args.steps, warmup=args.warmup):
+        p["peak_source"] = f"hbm_gbs / bf16_tflops (burst) of {peak_kind}"
+        p["l2"] = "flushed between timed steps"
+        print(json.dumps(p), flush=True)
     return 0
 
 
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=("cer", "reference"), default="cer")
-    ap.add_argument("--config", choices=sorted(gen.WORKLOADS), default="und_1p5b")
+    ap.add_argument("--config", choices=sorted(gen.WORKLOADS), default="long_7b")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--quick", action="store_true",
+                    help="leave out the other configs and the sweep (the headline workload's line only)")
     ap.add_argument("--sweep", action="store_true",
-                    help="time the 7B sweep points (one JSON line each) instead of the bench line")
+                    help="time the 7B sweep grid (one JSON line per point) instead of the bench line")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

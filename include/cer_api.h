@@ -109,8 +109,9 @@ size_t cer_score_workspace_size(int B, int N, int core_hidden, int exp_hidden, i
  * process exits.  Sizes whose cer_score_workspace_size() exceeds 4 MiB are
  * rejected with CER_ERR_WORKSPACE before any work is enqueued.  The call
  * allocates nothing.  Its first call on a device looks up the array's device
- * address (with that device current); make that first call before any
- * stream capture.  All calls share the array: calls whose GPU work can
+ * address (with that device current), and so does the first call in a new
+ * context of that device (after cudaDeviceReset, say); make that first call
+ * before any stream capture.  All calls share the array: calls whose GPU work can
  * overlap (other streams, other host threads) race on it; calls on one
  * stream are safe.                                                          */
 cer_status cer_score_static(const void* h, int B, int N, int d,
@@ -182,6 +183,17 @@ cer_status cer_pack_ffn_weights(const void* Wg, const void* Wu, const void* WdT,
  *   duplicates within a sequence, Y bf16 [B*k_tot, d].                        */
 cer_status cer_scatter_add(void* h, int B, int N, int d, const int32_t* idx, int k_tot,
                            const void* Y, cudaStream_t stream);
+
+/* cer_scatter_add_checked: the same unpack for index lists that may break
+ * cer_scatter_add's precondition (no paper counterpart: a validation mode).
+ * Each sequence's list is first checked on the device: an entry outside
+ * [0, N) or an entry repeated within the sequence (two updates of one row
+ * would race) sets CER_ERR_INDEX in the device status word, and then none of
+ * that sequence's rows is written; valid sequences are updated exactly as by
+ * cer_scatter_add.  One CTA per sequence, so slower than cer_scatter_add for
+ * few sequences.  N <= 393216.                                              */
+cer_status cer_scatter_add_checked(void* h, int B, int N, int d, const int32_t* idx, int k_tot,
+                                   const void* Y, cudaStream_t stream);
 
 /* ------------------------------------------------------------------ fused block
  * The whole routed block S1..S5 on one stream:
@@ -293,9 +305,10 @@ cer_status cer_redundancy_gap(const void* h_in, const void* h_out, const uint8_t
 size_t cer_redundancy_gap_workspace_size(int B, int N);
 
 /* ------------------------------------------------------------------ attention on the packed sequence
- * Sec. 3.4: the retained tokens are packed into a shorter sequence for
- * attention and FFN; for understanding, the packed keys and values form the
- * compressed key-value cache that decoding reuses.  Backbone (App. A.5):
+ * Sec. 3.4 (task-adaptive token compaction): attention, like the FFN, runs
+ * only over the kept tokens of R, gathered into a compact sequence; in
+ * understanding mode the keys and values of that compact sequence are the
+ * reduced key-value cache later decoding steps read.  Backbone (App. A.5):
  * Qwen2.5, head size 128, grouped key/value heads, rotary embedding.
  *
  * Packed rows: qkv bf16 [B * L, (Hq + 2 Hkv) * 128] (device, 16-byte
@@ -357,6 +370,24 @@ cer_status cer_routed_attention(void* h, void* out, int B, int N, int d, const i
                                 const void* WqkvT, const void* WoT, int Hq, int Hkv, int causal, double base,
                                 void* qkv, void* workspace, size_t workspace_bytes, cudaStream_t stream);
 size_t cer_routed_attention_workspace_size(int B, int L, int d, int Hq, int Hkv);
+
+/* ------------------------------------------------------------------ bounded-wait self-test
+ * cer_selftest_bounded_wait: a check of this library's failure detection (no
+ * paper counterpart).  Every wait inside its kernels (on an mbarrier phase or
+ * on a flag another CTA publishes) gives up after a limit, records
+ * CER_ERR_TIMEOUT in the device status word and unwinds.  This entry point
+ * launches one single-thread kernel that waits the same way, with a limit of
+ * limit_us microseconds (1 .. 100000), for
+ *   kind 0: the device word *flag (8-byte aligned device memory) to equal
+ *           token, polled with acquire loads;
+ *   kind 1: an mbarrier phase in the kernel's shared memory, completed only
+ *           if arrive != 0 (the thread then arrives on it before waiting);
+ *           flag is not read.
+ * When the wait runs out, the kernel records CER_ERR_TIMEOUT and returns with
+ * nothing in flight, so the context stays usable: cer_sync_status then
+ * returns CER_ERR_TIMEOUT and clears it.                                    */
+cer_status cer_selftest_bounded_wait(int kind, const unsigned long long* flag, unsigned long long token,
+                                     int arrive, int limit_us, cudaStream_t stream);
 
 /* ------------------------------------------------------------------ status
  * cer_sync_status: synchronise `stream`, then return and clear the current

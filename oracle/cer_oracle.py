@@ -18,8 +18,8 @@ Computation Scheduling"):
     scalar output; M segments of the denoising timesteps.
   * Sec. 3.4, Eq. 6 (router_inference_outputs): p = sigmoid(l), R = TopK(p, K);
     App. B.2: the sigmoid is monotonic, so ranking logits gives the same set.
-  * Sec. 3.4, task-adaptive token compaction: R is packed into a shorter
-    sequence for the FFN, D bypasses unchanged.
+  * Sec. 3.4, task-adaptive token compaction: the kept set R is gathered into
+    a compact sequence for the FFN, the dropped set D passes through unchanged.
   * Sec. 3.4 (2) FFN pruning and App. A.4: FFN restricted to the channels kept
     by the static mask; the backbone is Qwen2.5 (App. A.5), a SwiGLU FFN.
 
@@ -52,9 +52,9 @@ UCS statistics (Sec. 3.4, Unified Computation Scheduling):
   retained set R is every kept token; a zero-norm pair has cosine 1 when the
   vectors are equal, else 0; empty R gives g = 0.
 
-Attention on the packed sequence (Sec. 3.4: the retained tokens are packed
-into a shorter sequence for attention and FFN; for understanding the packed
-keys and values form a compressed KV cache):
+Attention on the packed sequence (Sec. 3.4, token compaction: attention runs,
+like the FFN, only over the kept tokens gathered into a compact sequence; in
+understanding mode their keys and values are the reduced KV cache):
   * rope: rotary position embedding of the Qwen2.5 backbone (App. A.5),
     rotate-half pairing (j, j + dh/2), theta_j = base^(-2j/dh);
   * packed_attention: softmax(Q K^T / sqrt(dh)) V per head over one packed

@@ -27,12 +27,12 @@ STATUS_NAMES = {0: "CER_OK", 1: "CER_ERR_NULL", 2: "CER_ERR_SHAPE", 3: "CER_ERR_
 
 # Every symbol include/cer_api.h declares.
 EXPORTS = ("cer_score", "cer_score_workspace_size", "cer_score_static", "cer_select_topk", "cer_gather", "cer_routed_ffn",
-           "cer_routed_ffn_workspace_size", "cer_pack_ffn_weights", "cer_scatter_add", "cer_routed_block",
+           "cer_routed_ffn_workspace_size", "cer_pack_ffn_weights", "cer_scatter_add", "cer_scatter_add_checked", "cer_routed_block",
            "cer_routed_block_workspace_size", "cer_ffn_channel_norms", "cer_routed_ffn_gated",
            "cer_routed_ffn_gated_workspace_size", "cer_routed_block_gated", "cer_routed_block_gated_workspace_size",
            "cer_drop_set_stats", "cer_redundancy_gap",
            "cer_redundancy_gap_workspace_size", "cer_rope_packed", "cer_packed_attention",
-           "cer_routed_attention", "cer_routed_attention_workspace_size", "cer_sync_status",
+           "cer_routed_attention", "cer_routed_attention_workspace_size", "cer_selftest_bounded_wait", "cer_sync_status",
            "cer_get_error", "cer_status_string", "cer_version")
 
 
@@ -62,6 +62,7 @@ _SIGS = {
     "cer_routed_ffn_workspace_size": ([_i, _i, _i, _i], _sz),
     "cer_pack_ffn_weights": ([_vp, _vp, _vp, _i, _i, _vp, _i, _vp, _vp, _vp, _vp], _i),
     "cer_scatter_add": ([_vp, _i, _i, _i, _vp, _i, _vp, _vp], _i),
+    "cer_scatter_add_checked": ([_vp, _i, _i, _i, _vp, _i, _vp, _vp], _i),
     "cer_routed_block": ([_vp, _vp, _i, _i, _i, _SCP, _SCP, _vp, _i, _i, _i, _i, _vp, _vp, _vp, _i, _vp, _i,
                           _vp, _vp, _vp, _vp, _sz, _vp, _i, _vp], _i),
     "cer_routed_block_workspace_size": ([_i, _i, _i, _i, _i, _i, _i, _i, _i, _i, _i], _sz),
@@ -79,6 +80,7 @@ _SIGS = {
     "cer_routed_attention": ([_vp, _vp, _i, _i, _i, _vp, _i, _vp, _vp, _i, _i, _i, ctypes.c_double, _vp, _vp,
                               _sz, _vp], _i),
     "cer_routed_attention_workspace_size": ([_i, _i, _i, _i, _i], _sz),
+    "cer_selftest_bounded_wait": ([_i, _vp, ctypes.c_ulonglong, _i, _i, _vp], _i),
     "cer_sync_status": ([_vp], _i),
     "cer_get_error": ([], ctypes.c_char_p),
     "cer_status_string": ([_i], ctypes.c_char_p),
@@ -206,6 +208,14 @@ def cer_scatter_add(h, idx, Y, stream=None):
     _check(load().cer_scatter_add(_p(h), B, N, d, _p(idx), idx.shape[1], _p(Y), _stream(stream)))
 
 
+def cer_scatter_add_checked(h, idx, Y, stream=None):
+    """cer_scatter_add that first checks each sequence's index list on the
+    device (range, no repeats); a bad sequence is left unwritten and
+    cer_sync_status raises CER_ERR_INDEX."""
+    B, N, d = h.shape
+    _check(load().cer_scatter_add_checked(_p(h), B, N, d, _p(idx), idx.shape[1], _p(Y), _stream(stream)))
+
+
 def cer_routed_block_workspace_size(B, N, d, core_hidden, exp_hidden, task, r0, r1, K, C, with_chan) -> int:
     return load().cer_routed_block_workspace_size(B, N, d, core_hidden, exp_hidden, task, r0, r1, K, C,
                                                   int(bool(with_chan)))
@@ -326,6 +336,14 @@ def cer_routed_attention(h, idx, WqkvT, WoT, Hq, Hkv, causal, base=1e6, out=None
     _check(load().cer_routed_attention(_p(h), _p(out), B, N, d, _p(idx), L, _p(WqkvT), _p(WoT), Hq, Hkv,
                                        int(causal), float(base), _p(qkv), _p(ws), ws.numel(), _stream(stream)))
     return h if out is None else out
+
+
+def cer_selftest_bounded_wait(kind, flag=None, token=0, arrive=False, limit_us=1000, stream=None):
+    """One bounded wait on the device (kind 0: *flag == token; kind 1: an
+    mbarrier phase, completed only when ``arrive``); a wait that runs out
+    shows as CER_ERR_TIMEOUT at the next cer_sync_status."""
+    _check(load().cer_selftest_bounded_wait(int(kind), _p(flag), int(token), int(bool(arrive)), int(limit_us),
+                                            _stream(stream)))
 
 
 def cer_sync_status(stream=None) -> None:

@@ -1,7 +1,8 @@
-// attention_kernel.cu -- attention on the packed sequence (Sec. 3.4: the
-// retained tokens are packed into a shorter sequence for attention and FFN;
-// for understanding the packed keys and values are the compressed KV cache),
-// with the rotary position embedding of the Qwen2.5 backbone (App. A.5).
+// attention_kernel.cu -- attention on the packed sequence (Sec. 3.4, token
+// compaction: only the kept tokens of R take part in attention, as in the
+// FFN, and in understanding mode their keys and values are the reduced KV
+// cache), with the rotary position embedding of the Qwen2.5 backbone
+// (App. A.5).
 //
 // Packed rows are laid out as one bf16 matrix qkv [B * L, (Hq + 2 Hkv) * 128]:
 // per row Hq query heads, Hkv key heads, Hkv value heads of 128 values.  A

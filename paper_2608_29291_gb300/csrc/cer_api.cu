@@ -48,7 +48,8 @@ struct DeviceInfo {
   bool ready = false;
   bool supported = false;
   int n_sm = 0;
-  int* status = nullptr;  // device address of g_status_word
+  int* status = nullptr;             // device address of g_status_word
+  unsigned long long ctx = 0;        // the context that address belongs to
 };
 
 std::mutex g_dev_mu;
@@ -59,17 +60,22 @@ cer_status device_info(DeviceInfo** out) {
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
   if (dev < 0 || dev >= kMaxDevices) return fail(CER_ERR_DEVICE, "device index %d out of range", dev);
+  const unsigned long long ctx = cer::current_context_id();
   std::lock_guard<std::mutex> lk(g_dev_mu);
   DeviceInfo& d = g_dev[dev];
-  if (!d.ready) {
+  // The status word's address is looked up again whenever the context is not
+  // the one it was taken in (or cannot be identified).
+  if (!d.ready || (d.supported && (ctx == 0 || ctx != d.ctx))) {
     int major = 0, minor = 0;
     cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
     cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
     d.supported = (major == 10 && minor == 3);
     cudaDeviceGetAttribute(&d.n_sm, cudaDevAttrMultiProcessorCount, dev);
+    d.ready = false;
     if (d.supported) {
       e = cudaGetSymbolAddress(reinterpret_cast<void**>(&d.status), g_status_word);
       if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(status)");
+      d.ctx = cer::current_context_id();
     }
     d.ready = true;
   }
@@ -231,6 +237,37 @@ static PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
   return encode;
 }
 
+using PfnCtxGetCurrent = CUresult (*)(CUcontext*);
+using PfnCtxGetId = CUresult (*)(CUcontext, unsigned long long*);
+
+unsigned long long current_context_id() {
+  static PfnCtxGetCurrent get_current = nullptr;
+  static PfnCtxGetId get_id = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    cudaDriverEntryPointQueryResult q;
+    void* fn = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &fn, 4000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_current = reinterpret_cast<PfnCtxGetCurrent>(fn);
+    fn = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &fn, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_id = reinterpret_cast<PfnCtxGetId>(fn);
+  });
+  if (get_current == nullptr || get_id == nullptr) return 0;
+  CUcontext c = nullptr;
+  if (get_current(&c) != CUDA_SUCCESS || c == nullptr) return 0;
+  unsigned long long id = 0;
+  if (get_id(c, &id) != CUDA_SUCCESS) return 0;
+  return id;
+}
+
+cer_status require_supported_device() {
+  DeviceInfo* d = nullptr;
+  return device_info(&d);
+}
+
 bool encode_bf16_2d(CUtensorMap* map, const void* base, uint64_t rows, uint64_t cols, uint32_t box_cols,
                     uint32_t box_rows) {
   const PFN_cuTensorMapEncodeTiled_v12000 encode = tensor_map_encoder();
@@ -259,15 +296,19 @@ bool encode_bf16_col_blocks(CUtensorMap* map, const void* base, uint64_t rows, u
 }
 
 cudaError_t ensure_max_smem(const void* func, size_t bytes) {
+  // A function attribute belongs to the context it was set in: remembered per
+  // (context, function), and set on every call when the context cannot be
+  // identified.
   static std::mutex mu;
-  static std::set<std::pair<int, const void*>> done;
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return e;
+  static std::set<std::pair<unsigned long long, const void*>> done;
+  const unsigned long long ctx = current_context_id();
   std::lock_guard<std::mutex> lk(mu);
-  if (done.count({dev, func})) return cudaSuccess;
-  e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes));
-  if (e == cudaSuccess) done.insert({dev, func});
+  if (ctx != 0 && done.count({ctx, func})) return cudaSuccess;
+  cudaError_t e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes));
+  if (e == cudaSuccess) {
+    const unsigned long long now = current_context_id();
+    if (now != 0) done.insert({now, func});
+  }
   return e;
 }
 
@@ -419,6 +460,44 @@ cer_status cer_scatter_add(void* h, int B, int N, int d, const int32_t* idx, int
   cudaError_t e = cer::launch_scatter_add(static_cast<__nv_bfloat16*>(h), B, N, d, idx, k_tot,
                                           static_cast<const __nv_bfloat16*>(Y), dev->status, dev->n_sm, stream);
   if (e != cudaSuccess) return cuda_fail(e, "scatter-add launch");
+  return CER_OK;
+}
+
+cer_status cer_scatter_add_checked(void* h, int B, int N, int d, const int32_t* idx, int k_tot, const void* Y,
+                                   cudaStream_t stream) {
+  CER_PTR_IF(h, static_cast<long long>(B) * N > 0);
+  CER_PTR_IF(idx, static_cast<long long>(B) * k_tot > 0);
+  CER_PTR_IF(Y, static_cast<long long>(B) * k_tot > 0);
+  CER_ALIGN(h);
+  CER_ALIGN(idx);
+  CER_ALIGN(Y);
+  CER_REQUIRE(B >= 0 && N >= 0 && k_tot >= 0 && k_tot <= N, CER_ERR_SHAPE, "B=%d N=%d k_tot=%d", B, N, k_tot);
+  CER_REQUIRE(N <= cer::kScatterCheckedMaxN, CER_ERR_SHAPE, "N=%d exceeds %d for the checked scatter-add", N,
+              cer::kScatterCheckedMaxN);
+  CER_REQUIRE(d > 0 && d % 8 == 0, CER_ERR_SHAPE, "d=%d must be a positive multiple of 8", d);
+  DeviceInfo* dev = nullptr;
+  cer_status s = device_info(&dev);
+  if (s != CER_OK) return s;
+  cudaError_t e = cer::launch_scatter_add_checked(static_cast<__nv_bfloat16*>(h), B, N, d, idx, k_tot,
+                                                  static_cast<const __nv_bfloat16*>(Y), dev->status, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "checked scatter-add launch");
+  return CER_OK;
+}
+
+cer_status cer_selftest_bounded_wait(int kind, const unsigned long long* flag, unsigned long long token, int arrive,
+                                     int limit_us, cudaStream_t stream) {
+  CER_REQUIRE(kind == 0 || kind == 1, CER_ERR_RANGE, "kind=%d must be 0 (flag) or 1 (mbarrier)", kind);
+  CER_REQUIRE(kind == 1 || flag != nullptr, CER_ERR_NULL, "flag is NULL");
+  CER_REQUIRE(flag == nullptr || (reinterpret_cast<uintptr_t>(flag) & 7u) == 0, CER_ERR_ALIGN,
+              "flag is not 8-byte aligned");
+  CER_REQUIRE(limit_us >= 1 && limit_us <= 100000, CER_ERR_RANGE, "limit_us=%d must be in [1, 100000]", limit_us);
+  DeviceInfo* dev = nullptr;
+  cer_status s = device_info(&dev);
+  if (s != CER_OK) return s;
+  cudaError_t e = cer::launch_bounded_wait_selftest(kind, flag, token, arrive ? 1 : 0,
+                                                    static_cast<unsigned long long>(limit_us) * 1000ull, dev->status,
+                                                    stream);
+  if (e != cudaSuccess) return cuda_fail(e, "bounded-wait self-test launch");
   return CER_OK;
 }
 

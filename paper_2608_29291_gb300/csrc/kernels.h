@@ -56,6 +56,21 @@ inline cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, siz
 // Record a printf-style message for cer_get_error() and return `status`.
 cer_status internal_fail(cer_status status, const char* fmt, ...);
 
+// CER_OK if the current device is an sm_103 GPU this library can run on;
+// otherwise the status and message every entry point gives for it.
+cer_status require_supported_device();
+
+// Identity of the current CUDA context (cuCtxGetId), 0 if none is current.
+// Device addresses of module symbols and per-function attributes belong to a
+// context: a cache of them is valid only while this value is unchanged (a
+// cudaDeviceReset, for one, makes a new primary context).
+unsigned long long current_context_id();
+
+// The bounded-wait self-test kernel: kind 0 waits for *flag == token, kind 1
+// for an mbarrier phase (completed only when arrive != 0), at most limit_ns.
+cudaError_t launch_bounded_wait_selftest(int kind, const unsigned long long* flag, unsigned long long token,
+                                         int arrive, unsigned long long limit_ns, int* status, cudaStream_t stream);
+
 // Raise a kernel's dynamic shared-memory limit to `bytes` (its largest
 // launch) once per device.
 cudaError_t ensure_max_smem(const void* func, size_t bytes);
@@ -134,6 +149,12 @@ cudaError_t launch_gather(const __nv_bfloat16* h, int B, int N, int d, const int
                           __nv_bfloat16* X, int* status, int n_sm, cudaStream_t stream);
 cudaError_t launch_scatter_add(__nv_bfloat16* h, int B, int N, int d, const int32_t* idx, int k_tot,
                                const __nv_bfloat16* Y, int* status, int n_sm, cudaStream_t stream);
+// The validating scatter-add: a sequence whose index list holds an entry out
+// of [0, N) or a repeated entry records CER_ERR_INDEX and is left unwritten.
+// N <= kScatterCheckedMaxN (its bitmap lives in shared memory).
+constexpr int kScatterCheckedMaxN = 393216;
+cudaError_t launch_scatter_add_checked(__nv_bfloat16* h, int B, int N, int d, const int32_t* idx, int k_tot,
+                                       const __nv_bfloat16* Y, int* status, cudaStream_t stream);
 
 // ------------------------------------------------------------------ S4 FFN
 struct FfnArgs {

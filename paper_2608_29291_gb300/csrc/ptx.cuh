@@ -104,18 +104,37 @@ constexpr uint64_t kWaitLimitNs = 2000000000ull;
 
 // Wait for the phase of `bar` with the given parity to complete.  Returns
 // false if the CTA is aborting (another role gave up) or the limit ran out.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag,
-                                          int* status) {
+// `limit_ns` is kWaitLimitNs everywhere but in the bounded-wait self-test.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, int* status,
+                                          uint64_t limit_ns = kWaitLimitNs) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   while (true) {
     if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
     if (*abort_flag) return false;
-    if (globaltimer_ns() - t0 > kWaitLimitNs) {
+    if (globaltimer_ns() - t0 > limit_ns) {
       *abort_flag = 1;
       record_status(status, CER_DEV_TIMEOUT);
       return false;
     }
+  }
+}
+
+// Wait until a global flag written by another CTA of the grid holds `token`
+// (acquire loads), bounded like every wait.
+__device__ __forceinline__ bool flag_wait(const unsigned long long* flag, unsigned long long token,
+                                          volatile int* abort_flag, int* status, uint64_t limit_ns = kWaitLimitNs) {
+  if (ld_acquire_u64(flag) == token) return true;
+  const uint64_t t0 = globaltimer_ns();
+  while (true) {
+    if (ld_acquire_u64(flag) == token) return true;
+    if (*abort_flag) return false;
+    if (globaltimer_ns() - t0 > limit_ns) {
+      *abort_flag = 1;
+      record_status(status, CER_DEV_TIMEOUT);
+      return false;
+    }
+    __nanosleep(64);
   }
 }
 

@@ -96,6 +96,50 @@ __global__ void __launch_bounds__(kRowThreads) scatter_add_kernel(uint4* __restr
   }
 }
 
+// The validating form of the scatter-add: one CTA per sequence first marks
+// every index of the sequence in a bitmap of its N tokens in shared memory;
+// an index out of range or marked twice makes the sequence invalid, and then
+// none of its rows is written (two warps adding into one row would race) and
+// CER_DEV_INDEX is recorded.  A valid sequence's rows are then added as in
+// scatter_add_kernel, one warp per row.
+__global__ void __launch_bounds__(kRowThreads) scatter_add_checked_kernel(uint4* __restrict__ h, int N, int d16,
+                                                                          const int32_t* __restrict__ idx,
+                                                                          int k_tot, const uint4* __restrict__ Y,
+                                                                          int* status) {
+  griddep_wait();
+  griddep_launch_dependents();
+  extern __shared__ uint32_t seen[];
+  __shared__ int bad;
+  const int b = blockIdx.x;
+  const int words = (N + 31) / 32;
+  for (int i = threadIdx.x; i < words; i += blockDim.x) seen[i] = 0u;
+  if (threadIdx.x == 0) bad = 0;
+  __syncthreads();
+  const int32_t* list = idx + static_cast<size_t>(b) * k_tot;
+  for (int j = threadIdx.x; j < k_tot; j += blockDim.x) {
+    const int i = __ldg(list + j);
+    if (i < 0 || i >= N) {
+      bad = 1;
+      continue;
+    }
+    const uint32_t bit = 1u << (i & 31);
+    if (atomicOr(&seen[i >> 5], bit) & bit) bad = 1;
+  }
+  __syncthreads();
+  if (bad) {
+    if (threadIdx.x == 0) record_status(status, CER_DEV_INDEX);
+    return;
+  }
+  const int lane = threadIdx.x & 31;
+  const int wpb = blockDim.x >> 5;
+  for (int j = threadIdx.x >> 5; j < k_tot; j += wpb) {
+    const int i = __ldg(list + j);
+    uint4* row = h + (static_cast<size_t>(b) * N + i) * d16;
+    const uint4* y = Y + (static_cast<size_t>(b) * k_tot + j) * d16;
+    for (int c = lane; c < d16; c += 32) row[c] = add_row_vec(row[c], __ldg(y + c));
+  }
+}
+
 static int row_grid(int M, int n_sm) {
   const int wpb = kRowThreads / 32;
   int blocks = (M + wpb - 1) / wpb;
@@ -128,6 +172,14 @@ cudaError_t launch_scatter_add(__nv_bfloat16* h, int B, int N, int d, const int3
   if (M == 0 || d == 0) return cudaSuccess;
   return launch_k(scatter_add_kernel, dim3(row_grid(M, n_sm)), dim3(kRowThreads), 0, stream, 1,
                   reinterpret_cast<uint4*>(h), N, d / 8, idx, k_tot, M, reinterpret_cast<const uint4*>(Y), status);
+}
+
+cudaError_t launch_scatter_add_checked(__nv_bfloat16* h, int B, int N, int d, const int32_t* idx, int k_tot,
+                                       const __nv_bfloat16* Y, int* status, cudaStream_t stream) {
+  if (B == 0 || k_tot == 0 || d == 0) return cudaSuccess;
+  const size_t smem = static_cast<size_t>((N + 31) / 32) * sizeof(uint32_t);
+  return launch_k(scatter_add_checked_kernel, dim3(B), dim3(kRowThreads), smem, stream, 1, reinterpret_cast<uint4*>(h),
+                  N, d / 8, idx, k_tot, reinterpret_cast<const uint4*>(Y), status);
 }
 
 }  // namespace cer

@@ -274,23 +274,6 @@ struct EpiCtx {
   }
 };
 
-// Wait until a stream-K flag holds `token` (bounded like every wait).
-__device__ __forceinline__ bool flag_wait(const unsigned long long* flag, unsigned long long token,
-                                          volatile int* abort_flag, int* status) {
-  if (ld_acquire_u64(flag) == token) return true;
-  const uint64_t t0 = globaltimer_ns();
-  while (true) {
-    if (ld_acquire_u64(flag) == token) return true;
-    if (*abort_flag) return false;
-    if (globaltimer_ns() - t0 > kWaitLimitNs) {
-      *abort_flag = 1;
-      record_status(status, CER_DEV_TIMEOUT);
-      return false;
-    }
-    __nanosleep(64);
-  }
-}
-
 template <class P>
 __global__ void __launch_bounds__(gemm_threads<P>(), 1)
     umma_gemm_kernel(const __grid_constant__ typename P::Params p, const __grid_constant__ StreamK sk) {

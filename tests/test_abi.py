@@ -133,6 +133,28 @@ def test_attention_argument_checks(lib):
     assert lib.cer_routed_attention_workspace_size(2, 0, 128, 4, 2) == 0
 
 
+def test_checked_scatter_argument_checks(lib):
+    f = lib.cer_scatter_add_checked
+    assert f(FAKE, 1, 500000, 64, FAKE, 10, FAKE, None) == 2     # N beyond the bitmap
+    assert f(FAKE, 1, 100, 60, FAKE, 10, FAKE, None) == 2        # d % 8
+    assert f(FAKE, 1, 100, 64, FAKE, 101, FAKE, None) == 2       # k_tot > N
+    assert f(FAKE, 1, 100, 64, None, 10, FAKE, None) == 1        # NULL idx
+
+
+@pytest.mark.skipif(torch.cuda.is_available(), reason="checks the behaviour without a GPU")
+def test_static_scorer_refuses_an_unusable_device_like_cer_score(lib):
+    """cer_score_static asks whether the device is one this library runs on
+    before it looks up its static array: without a usable GPU it fails with the
+    same status and message as cer_score on the same well-formed call."""
+    core = cer.CerScorerC(FAKE.value, None, FAKE.value, None, 256, 0, 1)
+    st = lib.cer_score_static(FAKE, 1, 16, 1536, ctypes.pointer(core), None, None, 0, FAKE, None, None)
+    msg_static = _err(lib)
+    st_ws = lib.cer_score(FAKE, 1, 16, 1536, ctypes.pointer(core), None, None, 0, FAKE, None, FAKE, 1 << 30, None)
+    assert st == st_ws == 6, (st, st_ws)
+    assert msg_static == _err(lib)
+    assert "static scratch" not in msg_static
+
+
 @pytest.mark.skipif(torch.cuda.is_available(), reason="checks the behaviour without a GPU")
 def test_well_formed_call_without_gpu_fails_loudly(lib):
     st = lib.cer_select_topk(FAKE, 1, 8, 0, 8, 4, FAKE, None, None)

@@ -155,6 +155,23 @@ def test_sigmoid_ranking_equals_logit_ranking():
         assert idx[0].tolist() == want.tolist()
 
 
+def test_sigmoid_values():
+    """p = sigmoid(l) of Eq. 6 by value: sigma(0) = 1/2; sigma(ln 3) = 3/4 and
+    sigma(-ln 3) = 1/4 (1 / (1 + 1/3) and 1 / (1 + 3)); sigma(ln 9) = 9/10;
+    the symmetry sigma(x) + sigma(-x) = 1; the limits; and torch's sigmoid in
+    fp64 as an independent library routine."""
+    assert ora.sigmoid(np.array([0.0]))[0] == 0.5
+    assert abs(ora.sigmoid(np.array([math.log(3.0)]))[0] - 0.75) < 1e-15
+    assert abs(ora.sigmoid(np.array([-math.log(3.0)]))[0] - 0.25) < 1e-15
+    assert abs(ora.sigmoid(np.array([math.log(9.0)]))[0] - 0.9) < 1e-15
+    x = np.random.default_rng(4).normal(0, 4, 1000)
+    assert np.max(np.abs(ora.sigmoid(x) + ora.sigmoid(-x) - 1.0)) < 1e-15
+    with np.errstate(over="ignore"):
+        assert ora.sigmoid(np.array([-800.0]))[0] == 0.0 and ora.sigmoid(np.array([800.0]))[0] == 1.0
+    want = torch.sigmoid(torch.from_numpy(x)).numpy()
+    assert np.max(np.abs(ora.sigmoid(x) - want)) < 1e-15
+
+
 # ------------------------------------------------------------------ scalar pieces
 
 def test_bf16_widening_exact():
@@ -379,6 +396,7 @@ def _all_pin_failures():
         test_ffn_dense_matches_torch_swiglu()
         test_block_full_keep_equals_dense_block()
         test_block_invariants()
+        test_sigmoid_values()
     except AssertionError as e:
         f.append(str(e))
     return f
@@ -399,6 +417,8 @@ MUTATIONS = {
     "silu_without_gate": ("routed_ffn", lambda orig: (
         lambda X, Wg, Wu, WdT, chan: _ffn_no_silu(X, Wg, Wu, WdT, chan))),
     "bias_sign": ("mlp_score", lambda orig: (lambda x, W1, w2, bias: orig(x, W1, w2, -bias))),
+    "sigmoid_tanh_scale": ("sigmoid", lambda orig: (lambda x: 0.5 * (1 + np.tanh(np.asarray(x, np.float64))))),
+    "sigmoid_offset": ("sigmoid", lambda orig: (lambda x: orig(np.asarray(x, np.float64) + 0.01))),
 }
 
 
