@@ -205,12 +205,17 @@ def gather(h: np.ndarray, idx: np.ndarray) -> np.ndarray:
 
 
 def routed_ffn(X: np.ndarray, Wg: np.ndarray, Wu: np.ndarray, WdT: np.ndarray,
-               chan: np.ndarray) -> np.ndarray:
+               chan: np.ndarray, act_bf16: bool = False) -> np.ndarray:
     """SwiGLU FFN on the packed rows restricted to the kept channels Cs; fp64 [M, d].
 
     y = sum_{c in Cs} WdT[c, :] * SiLU(Wg[c] . x) * (Wu[c] . x), with WdT the
     down projection stored channel-major (row c is W_down[:, c], the vector whose
     norm enters the saliency of Eq. 8).
+
+    act_bf16: the activation a = SiLU(g) * u enters the down projection as a
+    bf16 operand (the precision the comparison contract fixes: bf16 operands,
+    fp32 accumulation), i.e. rounded to fp32 and then to bf16, both to nearest
+    even, before its fp64 contraction with WdT.  Everything else stays fp64.
     """
     cs = np.asarray(chan, dtype=np.int64)
     x = bf16_to_f64(X)
@@ -218,6 +223,8 @@ def routed_ffn(X: np.ndarray, Wg: np.ndarray, Wu: np.ndarray, WdT: np.ndarray,
     u = x @ bf16_to_f64(Wu[cs]).T
     with np.errstate(over="ignore"):
         a = g / (1.0 + np.exp(-g)) * u          # SiLU(g) * u, SiLU(g) = g * sigmoid(g)
+    if act_bf16:
+        a = bf16_to_f64(round_to_bf16(a))
     return a @ bf16_to_f64(WdT[cs])
 
 

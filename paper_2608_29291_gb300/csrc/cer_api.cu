@@ -387,7 +387,7 @@ cer_status cer_score(const void* h, int B, int N, int d, const cer_scorer* core,
   cer::ScoreWorkspace ws = carve_score_ws(workspace, B, N, sh);
   cer::ScoreArgs a = make_score_args(h, B, N, d, core, exp, t, sh, dev->status);
   int n_partials = 0;
-  cudaError_t e = cer::launch_score(a, ws, dev->n_sm, stream, &n_partials);
+  cudaError_t e = cer::launch_score(a, ws, nullptr, dev->n_sm, stream, &n_partials);
   if (e != cudaSuccess) return cuda_fail(e, "scorer launch");
   e = cer::launch_score_reduce(ws.partial, n_partials, static_cast<size_t>(B) * N, logits, probs, dev->n_sm,
                                stream);
@@ -752,7 +752,7 @@ cer_status routed_block_impl(void* h, void* out, int B, int N, int d, const cer_
   // S1: scorer GEMM -> partial sums
   cer::ScoreArgs sa = make_score_args(h, B, N, d, core, exp, t, sh, dev->status);
   int n_partials = 0;
-  e = cer::launch_score(sa, sws, dev->n_sm, stream, &n_partials);
+  e = cer::launch_score(sa, sws, M64 > 0 ? &fa.sk : nullptr, dev->n_sm, stream, &n_partials);
   if (e != cudaSuccess) return cuda_fail(e, "scorer launch");
   if ((e = mark(1)) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
 

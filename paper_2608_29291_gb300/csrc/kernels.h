@@ -124,8 +124,10 @@ int score_chunk_width(int Hc, int He, int gen);
 int score_max_partials(int Hc, int He, int gen);
 // Launches the bias-table and scorer kernels; *n_partials receives the number
 // of partial-score rows written (to be summed in order by the consumer).
-cudaError_t launch_score(const ScoreArgs& a, const ScoreWorkspace& ws, int n_sm, cudaStream_t stream,
-                         int* n_partials);
+// With a stream-K area (sk non-NULL, as inside the fused block) the pair-MMA
+// scorer may split tiles by K block like the FFN GEMMs.
+cudaError_t launch_score(const ScoreArgs& a, const ScoreWorkspace& ws, const StreamKArea* sk, int n_sm,
+                         cudaStream_t stream, int* n_partials);
 cudaError_t launch_score_reduce(const float* partial, int n_chunks, size_t total, float* logits, float* probs,
                                 int n_sm, cudaStream_t stream);
 
@@ -140,6 +142,7 @@ struct TopkArgs {
   int32_t* idx;          // [B][k_tot]
   uint8_t* mask;         // nullable
   int* status;
+  int chunk;             // tokens per CTA of a sequence's cluster (set by launch_topk)
 };
 constexpr int kTopkMaxN = 49152;
 cudaError_t launch_topk(const TopkArgs& a, cudaStream_t stream);

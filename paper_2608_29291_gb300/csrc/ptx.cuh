@@ -355,6 +355,26 @@ __device__ __forceinline__ void cluster_sync() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
+// The two halves of cluster_sync, so that work can go between them: arrive
+// (this thread's earlier shared-memory accesses are released to the cluster)
+// and wait (every thread of the cluster has arrived).
+__device__ __forceinline__ void cluster_arrive() { asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory"); }
+__device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory"); }
+
+__device__ __forceinline__ uint32_t cluster_nctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
+  return r;
+}
+
+// A 32-bit load from shared memory at a cluster address (mapa_shared), which
+// may lie in another CTA of the cluster (distributed shared memory).
+__device__ __forceinline__ uint32_t ld_dsmem_u32(uint32_t cluster_addr) {
+  uint32_t v;
+  asm volatile("ld.shared::cluster.u32 %0, [%1];" : "=r"(v) : "r"(cluster_addr) : "memory");
+  return v;
+}
+
 // 32 lanes x 32 consecutive fp32 columns: thread i of the warp receives lane
 // (base lane + i), columns [col, col + 32).  The load and its wait sit in one
 // asm statement so no use of the registers can be scheduled before the wait.

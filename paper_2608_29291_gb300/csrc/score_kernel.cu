@@ -217,6 +217,106 @@ struct ScoreProblem {
   }
 };
 
+// The same scorer as pair MMAs (tcgen05 cta_group::2) for wide hidden layers,
+// where the scorer is bound by the tensor pipe (Hc + He >= 512): a work tile
+// is 256 consecutive rows of h viewed as [B*N, d] (tiles may straddle
+// sequences) times one 256-wide hidden chunk.  Each CTA of the pair loads its
+// 128 rows and 128 of the chunk's weight rows, so an SM takes in 32 KB per
+// 64-wide K block for a 128 x 256 x 64 product instead of the 48 KB of a
+// one-CTA 128 x 256 tile.  Each CTA's tensor memory receives all 256
+// columns of its 128 rows; its epilogue is ScoreProblem's, with the bias and
+// w2 tables looked up per row (b = row / N).  One expansion segment only
+// (the weight chunk must be the same for both CTAs of a pair).
+struct ScorePairProblem {
+  static constexpr int BN = 256;
+  static constexpr int MMA_PAIR = 1;
+  static constexpr int CLUSTER = 2;
+  static constexpr int KSUB = 2;
+  static constexpr int STAGES = 3;
+  static constexpr int B_MN_MAJOR = 0;
+  static constexpr int EPI_WARPS = 8;
+  static constexpr uint32_t kBStepBytes = 32;
+  static constexpr uint32_t kEpiSmemBytes = 0;
+  static constexpr uint32_t kBoxBytes = 128 * 128;   // 128 weight rows x 64 bf16
+
+  struct Params {
+    CUtensorMap tm_h;    // h as [B*N, d], box 64 x 128
+    CUtensorMap tm_w1;   // core W1 [Hc, d], box 64 x 128
+    CUtensorMap tm_w1e;  // expansion W1e [He, d], box 64 x 128
+    const float* bias_tab;   // [B][Ht], or NULL: columns take b1 (or 0) and w2 directly
+    const float* w2_tab;
+    const float* b1;
+    const float* w2;
+    float* partial;
+    int* status;
+    int rows, N, d, Ht;      // rows = B * N
+    int n_rp, n_core, n_chunks;
+  };
+  struct ProdState {
+    int m0, wrow, core;
+  };
+
+  // Cluster tile t: row pair t % n_rp (rows 256 (t % n_rp) + 128 rank ..), chunk t / n_rp.
+  __device__ static int num_tiles(const Params& p) { return p.n_rp * p.n_chunks; }
+  __device__ static int num_kb(const Params& p) { return p.d / 64; }
+  __device__ static bool weights_first(const Params&) { return true; }
+  __device__ static uint32_t stage_bytes(const Params&, int, int, int part) {
+    return 2 * (((part & kPartAct) ? kATileBytes : 0u) + ((part & kPartWeights) ? kBoxBytes : 0u));
+  }
+  __device__ static void prod_tile(const Params& p, int tile, int rank, ProdState& st) {
+    const int chunk = tile / p.n_rp;
+    st.m0 = (2 * (tile % p.n_rp) + rank) * 128;   // rows past B*N load as zeros
+    st.core = chunk < p.n_core;
+    st.wrow = (st.core ? chunk : chunk - p.n_core) * BN + rank * 128;
+  }
+  __device__ static void prod_kb(const Params& p, const ProdState& st, int, int kb, int lane, uint8_t* a,
+                                 uint8_t* b, uint32_t leader_bar, int part) {
+    if (lane == 0) {
+      const int x = kb * 64;
+      if (part & kPartAct) tma_load_2d_pair(a, &p.tm_h, leader_bar, x, st.m0);
+      if (part & kPartWeights) tma_load_2d_pair(b, st.core ? &p.tm_w1 : &p.tm_w1e, leader_bar, x, st.wrow);
+    }
+  }
+  __device__ static uint64_t bdesc(uint32_t saddr) { return sdesc_kmajor_sw128(saddr); }
+  __device__ static void prefetch(const Params& p) {
+    tma_prefetch_desc(&p.tm_h);
+    tma_prefetch_desc(&p.tm_w1);
+    tma_prefetch_desc(&p.tm_w1e);
+  }
+
+  __device__ static void epilogue_done(const Params&, int, int) {}
+  __device__ static bool epilogue(const Params& p, int tile, int row, int half, uint32_t taddr, EpiCtx& ctx) {
+    const int chunk = tile / p.n_rp;
+    const int grow = (2 * (tile % p.n_rp) + ctx.rank) * 128 + row;
+    // Rows past B*N (the ragged last tile) still take part in every tensor
+    // memory load -- tcgen05.ld is warp-collective (.sync.aligned) -- and
+    // only skip the store; their bias and w2 come from the last sequence.
+    const bool valid = grow < p.rows;
+    const int b = (valid ? grow : p.rows - 1) / p.N;
+    const float* bias = p.bias_tab ? p.bias_tab + static_cast<size_t>(b) * p.Ht + chunk * BN
+                                   : (p.b1 ? p.b1 + chunk * BN : nullptr);
+    const float* w2 = p.w2_tab ? p.w2_tab + static_cast<size_t>(b) * p.Ht + chunk * BN : p.w2 + chunk * BN;
+    float s = 0.f;
+#pragma unroll 1
+    for (int c = half * 4; c < half * 4 + 4; ++c) {
+      float v[32];
+      tmem_ld_32x32(taddr + c * 32, v);
+      const float4* b4 = bias ? reinterpret_cast<const float4*>(bias + c * 32) : nullptr;
+      const float4* w4 = reinterpret_cast<const float4*>(w2 + c * 32);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const float4 bb = b4 ? __ldg(b4 + q) : make_float4(0.f, 0.f, 0.f, 0.f), ww = __ldg(w4 + q);
+        s = fmaf(ww.x, gelu_as(v[4 * q + 0] + bb.x), s);
+        s = fmaf(ww.y, gelu_as(v[4 * q + 1] + bb.y), s);
+        s = fmaf(ww.z, gelu_as(v[4 * q + 2] + bb.z), s);
+        s = fmaf(ww.w, gelu_as(v[4 * q + 3] + bb.w), s);
+      }
+    }
+    if (valid) p.partial[static_cast<size_t>(2 * chunk + half) * p.rows + grow] = s;
+    return true;
+  }
+};
+
 // ---------------------------------------------------------------- reduce
 
 __global__ void score_reduce_kernel(const float* __restrict__ partial, int n_chunks, size_t total,
@@ -295,10 +395,51 @@ static cudaError_t launch_score_gemm(const ScoreArgs& a, const float* bias_tab, 
   return launch_gemm<P>(p, a.B * p.n_rt * p.n_chunks, a.d / 64, nullptr, n_sm, stream);
 }
 
+// Whether the pair-MMA scorer takes this launch: wide hidden layers (the
+// tensor-bound case), whole 256-wide chunks, one expansion segment.
+static bool use_pair_scorer(const ScoreArgs& a) {
+  const int Ht = a.Hc + (a.gen ? a.He : 0);
+  return Ht >= 512 && a.Hc % 256 == 0 && (!a.gen || (a.He % 256 == 0 && a.S == 1));
+}
+
+static cudaError_t launch_score_pair(const ScoreArgs& a, const float* bias_tab, const float* w2_tab, float* partial,
+                                     const StreamKArea* sk, int n_sm, cudaStream_t stream) {
+  using P = ScorePairProblem;
+  P::Params p{};
+  const int Ht = a.Hc + (a.gen ? a.He : 0);
+  const uint64_t rows = static_cast<uint64_t>(a.B) * a.N;
+  if (!encode_bf16_2d(&p.tm_h, a.h, rows, a.d, 64, 128)) return cudaErrorInvalidValue;
+  if (!encode_bf16_2d(&p.tm_w1, a.W1, a.Hc, a.d, 64, 128)) return cudaErrorInvalidValue;
+  if (a.gen) {
+    if (!encode_bf16_2d(&p.tm_w1e, a.W1e, a.He, a.d, 64, 128)) return cudaErrorInvalidValue;
+  } else {
+    p.tm_w1e = p.tm_w1;
+  }
+  p.bias_tab = bias_tab;
+  p.w2_tab = w2_tab;
+  p.b1 = a.b1;
+  p.w2 = a.w2;
+  p.partial = partial;
+  p.status = a.status;
+  p.rows = static_cast<int>(rows);
+  p.N = a.N;
+  p.d = a.d;
+  p.Ht = Ht;
+  p.n_rp = static_cast<int>((rows + 255) / 256);
+  p.n_core = a.Hc / 256;
+  p.n_chunks = Ht / 256;
+  return launch_gemm<P>(p, p.n_rp * p.n_chunks, a.d / 64, sk, n_sm, stream);
+}
+
 // Understanding reads b1 and w2 directly (bias/w2 tables NULL); generation
 // first builds the per-sequence tables.
 static cudaError_t launch_score_chunks(const ScoreArgs& a, const float* bias_tab, const float* w2_tab,
-                                       float* partial, int n_sm, cudaStream_t stream, int* n_partials) {
+                                       float* partial, const StreamKArea* sk, int n_sm, cudaStream_t stream,
+                                       int* n_partials) {
+  if (use_pair_scorer(a)) {
+    *n_partials = 2 * (a.Hc + (a.gen ? a.He : 0)) / 256;
+    return launch_score_pair(a, bias_tab, w2_tab, partial, sk, n_sm, stream);
+  }
   const int bn = pick_chunk_width(a, n_sm);
   *n_partials = bn ? 2 * (a.Hc + (a.gen ? a.He : 0)) / bn : 0;
   switch (bn) {
@@ -309,9 +450,9 @@ static cudaError_t launch_score_chunks(const ScoreArgs& a, const float* bias_tab
   }
 }
 
-cudaError_t launch_score(const ScoreArgs& a, const ScoreWorkspace& ws, int n_sm, cudaStream_t stream,
-                         int* n_partials) {
-  if (!a.gen) return launch_score_chunks(a, nullptr, nullptr, ws.partial, n_sm, stream, n_partials);
+cudaError_t launch_score(const ScoreArgs& a, const ScoreWorkspace& ws, const StreamKArea* sk, int n_sm,
+                         cudaStream_t stream, int* n_partials) {
+  if (!a.gen) return launch_score_chunks(a, nullptr, nullptr, ws.partial, sk, n_sm, stream, n_partials);
   const int emb_bytes = a.U ? a.E * static_cast<int>(sizeof(float)) : 0;
   const int Ht = a.Hc + a.He;
   EmbFreqTable ft;
@@ -322,7 +463,7 @@ cudaError_t launch_score(const ScoreArgs& a, const ScoreWorkspace& ws, int n_sm,
   cudaError_t e = launch_k(time_bias_kernel, bias_grid, dim3(32 * kBiasColsPerBlock), emb_bytes, stream, 1, a, ft,
                            ws.bias_tab, ws.w2_tab);
   if (e != cudaSuccess) return e;
-  return launch_score_chunks(a, ws.bias_tab, ws.w2_tab, ws.partial, n_sm, stream, n_partials);
+  return launch_score_chunks(a, ws.bias_tab, ws.w2_tab, ws.partial, sk, n_sm, stream, n_partials);
 }
 
 cudaError_t launch_score_reduce(const float* partial, int n_chunks, size_t total, float* logits, float* probs,

@@ -1,19 +1,28 @@
 // topk_kernel.cu -- S2: the per-sequence keep set R = TopK(sigmoid(l), K) of
-// Eq. 6 (router_inference_outputs, Sec. 3.4), computed exactly on the fp32 logits (the sigmoid is
+// Eq. 6 (Sec. 3.4), computed exactly on the fp32 logits (the sigmoid is
 // monotonic, App. B.2).
 //
-// One 1024-thread CTA per sequence keeps the N order-preserving 32-bit keys in
-// shared memory.  An MSB-first radix select (8-bit digits, shared histograms)
-// finds the K-th largest routable key T and how many tokens equal to T must
-// be taken; as soon as at most 32 routable keys share the digits found so
-// far, one warp ranks those candidates exactly and the remaining passes are
-// skipped (real-valued logits get there after one or two passes, heavy ties
-// take all four).  Each warp then owns a contiguous run of tokens, read 32
-// at a time (a token per lane, no bank conflicts): ballots rank every tie
-// (lowest index first) and every kept token, and two scans over the warps'
-// counts place them, so the kept list comes out in ascending token order with
-// no sort.  When fed the scorer's partial sums it also reduces them (in chunk
-// order) into the logits.
+// A sequence is handled by a cluster of G <= 8 CTAs (G chosen so each CTA
+// holds at most ~1024 tokens; G = 1 for short sequences), CTA `rank` owning
+// the tokens [rank * chunk, (rank + 1) * chunk).  Each CTA keeps the
+// order-preserving 32-bit keys of its tokens in shared memory (reducing the
+// scorer's partial sums, in chunk order, into the logits on the way).  An
+// MSB-first radix select with 8-bit digits finds the K-th largest routable
+// key T and how many tokens equal to T must be taken: every pass counts the
+// CTA's keys into per-warp sub-histograms, publishes their sum, and after one
+// cluster barrier every CTA adds up the G histograms through distributed
+// shared memory and takes the same digit.  As soon as at most 32 routable
+// keys share the digits found so far, each CTA publishes its candidates and
+// one warp per CTA ranks all of them exactly (real-valued logits get there
+// after one or two passes, heavy ties take all four).
+//
+// Compaction: each warp owns a contiguous run of its CTA's tokens.  The warps'
+// counts of ties (key == T) and of tokens kept outright (key > T, or outside
+// the routable range) are summed per CTA and published; after one more
+// cluster barrier every CTA knows how many ties and kept tokens precede it,
+// hence how many of its ties are taken (the lowest indices first) and where
+// its kept tokens go, and writes its part of the ascending keep list with
+// warp ballots -- no sort.
 #include <cuda_runtime.h>
 
 #include "kernels.h"
@@ -22,7 +31,11 @@
 
 namespace cer {
 
-constexpr int kTopkThreads = 1024;
+constexpr int kTopkThreads = 512;
+constexpr int kTopkWarps = kTopkThreads / 32;
+constexpr int kTopkMaxCluster = 8;
+// Tokens per CTA the cluster size aims at.
+constexpr int kTopkChunkTarget = 1024;
 
 // Monotone map from fp32 to uint32: a > b (as floats) iff key(a) > key(b);
 // -0.0 is mapped like +0.0.
@@ -32,50 +45,21 @@ __device__ __forceinline__ uint32_t order_key(float v) {
   return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 
-// Exclusive prefix sum over the block (all threads must call).
-__device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t* warp_tot) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  uint32_t incl = v;
-#pragma unroll
-  for (int off = 1; off < 32; off <<= 1) {
-    const uint32_t o = __shfl_up_sync(0xffffffffu, incl, off);
-    if (lane >= off) incl += o;
-  }
-  if (lane == 31) warp_tot[warp] = incl;
-  __syncthreads();
-  if (warp == 0) {
-    const int nw = blockDim.x >> 5;
-    uint32_t t = lane < nw ? warp_tot[lane] : 0u;
-    uint32_t ti = t;
-#pragma unroll
-    for (int off = 1; off < 32; off <<= 1) {
-      const uint32_t o = __shfl_up_sync(0xffffffffu, ti, off);
-      if (lane >= off) ti += o;
-    }
-    if (lane < nw) warp_tot[lane] = ti - t;  // exclusive over warps
-  }
-  __syncthreads();
-  const uint32_t r = warp_tot[warp] + incl - v;
-  __syncthreads();
-  return r;
-}
-
 // Histogram counts go to kSubHist copies (by warp) to spread the atomic
 // contention of logits that share a few digit values; merged after each pass.
 constexpr int kSubHist = 8;
 
 // Tokens a thread reduces at once in the logits pass (their partial-sum loads
-// are in flight together), and the keep-ballot store of the compaction.
+// are in flight together).
 constexpr int kLoadUnroll = 4;
-constexpr int kMaxSteps = (kTopkMaxN + kTopkThreads - 1) / kTopkThreads;
 
-// Logits from the scorer's partial sums, summed in chunk order, into the
-// order keys: a thread takes U tokens at a time and reads their partial rows
-// eight at a time, so up to 8U loads are in flight.
+// Logits of tokens [lo, hi) from the scorer's partial sums, summed in chunk
+// order, into the order keys: a thread takes U tokens at a time and reads
+// their partial rows eight at a time, so up to 8U loads are in flight.
 template <int U>
-__device__ __forceinline__ void reduce_logits(const TopkArgs& a, size_t base, uint32_t* keys, int* s_nan) {
-  const int N = a.N;
-  for (int i0 = threadIdx.x; i0 < N; i0 += U * blockDim.x) {
+__device__ __forceinline__ void reduce_logits(const TopkArgs& a, size_t base, int lo, int hi, uint32_t* keys,
+                                              int* s_nan) {
+  for (int i0 = lo + threadIdx.x; i0 < hi; i0 += U * blockDim.x) {
     float v[U];
 #pragma unroll
     for (int u = 0; u < U; ++u) v[u] = 0.f;
@@ -85,7 +69,7 @@ __device__ __forceinline__ void reduce_logits(const TopkArgs& a, size_t base, ui
       // back to back; the clamped ones are not used.
 #pragma unroll
       for (int u = 0; u < U; ++u) {
-        const int i = min(i0 + u * static_cast<int>(blockDim.x), N - 1);
+        const int i = min(i0 + u * static_cast<int>(blockDim.x), hi - 1);
 #pragma unroll
         for (int c = 0; c < 8; ++c) {
           const int cc = min(c0 + c, a.n_chunks - 1);
@@ -101,30 +85,46 @@ __device__ __forceinline__ void reduce_logits(const TopkArgs& a, size_t base, ui
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       const int i = i0 + u * blockDim.x;
-      if (i >= N) break;
+      if (i >= hi) break;
       if (a.logits_out) a.logits_out[base + i] = v[u];
       if (a.probs_out) a.probs_out[base + i] = 1.0f / (1.0f + expf(-v[u]));
       if (i >= a.r0 && i < a.r1 && v[u] != v[u]) *s_nan = 1;
-      keys[i] = order_key(v[u]);
+      keys[i - lo] = order_key(v[u]);
     }
   }
+}
+
+// Inclusive prefix sum over the lanes of a warp.
+__device__ __forceinline__ uint32_t warp_inclusive_scan(uint32_t v, int lane) {
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const uint32_t o = __shfl_up_sync(0xffffffffu, v, off);
+    if (lane >= off) v += o;
+  }
+  return v;
 }
 
 __global__ void __launch_bounds__(kTopkThreads) topk_kernel(TopkArgs a) {
   griddep_wait();
   griddep_launch_dependents();
-  extern __shared__ uint32_t keys[];
-  __shared__ uint32_t hist[256];
+  extern __shared__ uint32_t keys[];           // keys of this CTA's tokens [lo, hi), at i - lo
   __shared__ uint32_t sub[kSubHist][256];
-  __shared__ uint32_t warp_tot[32];
-  __shared__ uint32_t s_prefix, s_remaining, s_count, s_ncand;
-  __shared__ uint32_t s_cand[32];
+  __shared__ uint32_t hist[2][256];            // this CTA's histogram of a pass (by parity); read by the cluster
+  __shared__ uint32_t s_cand[32];              // this CTA's candidate keys; read by the cluster
+  __shared__ uint32_t s_ncand;
+  __shared__ uint32_t s_cnt[2];                // this CTA's ties and outright keeps; read by the cluster
+  __shared__ uint32_t s_prefix, s_remaining, s_count;
+  __shared__ uint32_t w_eq[kTopkWarps], w_gt[kTopkWarps], w_eq_off[kTopkWarps], w_pos[kTopkWarps];
   __shared__ int s_nan;
-  __shared__ uint32_t s_ballot[kTopkThreads / 32][kMaxSteps];
 
   const int tid = threadIdx.x;
-  const int b = blockIdx.x;
+  const int lane = tid & 31, warp = tid >> 5;
+  const int G = static_cast<int>(cluster_nctarank());
+  const int rank = static_cast<int>(cluster_ctarank());
+  const int b = blockIdx.x / G;
   const int N = a.N;
+  const int lo = rank * a.chunk;
+  const int hi = min(N, lo + a.chunk);         // hi <= lo: this CTA holds no token
   const size_t base = static_cast<size_t>(b) * N;
   if (tid == 0) {
     s_nan = 0;
@@ -133,31 +133,31 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(TopkArgs a) {
   __syncthreads();
 
   // 1. logits (reduced from partial sums in chunk order) -> keys
-  if (N >= 2 * static_cast<int>(blockDim.x)) {
-    reduce_logits<kLoadUnroll>(a, base, keys, &s_nan);
+  if (hi - lo >= 2 * static_cast<int>(blockDim.x)) {
+    reduce_logits<kLoadUnroll>(a, base, lo, hi, keys, &s_nan);
   } else {
-    reduce_logits<1>(a, base, keys, &s_nan);
+    reduce_logits<1>(a, base, lo, hi, keys, &s_nan);
   }
-  __syncthreads();
 
   const int Nr = a.r1 - a.r0;
   const int K = a.K;
   const bool keep_all = (K == Nr);
   const bool keep_none = (K == 0);
+  const bool select = !keep_all && !keep_none;
+  const int rlo = max(lo, a.r0), rhi = min(hi, a.r1);   // this CTA's routable tokens
   uint32_t thr = 0, need_eq = 0;
 
-  // 2. radix select of the K-th largest routable key
-  if (!keep_all && !keep_none) {
+  // 2. radix select of the K-th largest routable key (every CTA of the
+  // cluster takes the same branches: they all see the same histograms)
+  if (select) {
     uint32_t prefix = 0, pmask = 0, remaining = static_cast<uint32_t>(K);
     for (int i = tid; i < kSubHist * 256; i += blockDim.x) (&sub[0][0])[i] = 0;
     __syncthreads();
-    // Three barriers per pass: the merge also clears the sub-histograms for
-    // the next pass, and s_prefix is rewritten only two barriers after every
-    // thread has read it.
-    for (int shift = 24; shift >= 0; shift -= 8) {
-      uint32_t* my = sub[(tid >> 5) % kSubHist];
-      for (int i = a.r0 + tid; i < a.r1; i += blockDim.x) {
-        const uint32_t k = keys[i];
+    int par = 0;
+    for (int shift = 24; shift >= 0; shift -= 8, par ^= 1) {
+      uint32_t* my = sub[warp % kSubHist];
+      for (int i = rlo + tid; i < rhi; i += blockDim.x) {
+        const uint32_t k = keys[i - lo];
         if ((k & pmask) == prefix) atomicAdd(&my[(k >> shift) & 255u], 1u);
       }
       __syncthreads();
@@ -168,17 +168,22 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(TopkArgs a) {
           c += sub[q][i];
           sub[q][i] = 0;
         }
-        hist[i] = c;
+        hist[par][i] = c;
       }
-      __syncthreads();
-      if (tid < 32) {
-        const int lane = tid;
+      // Every CTA's histogram of this pass is complete.  The other buffer
+      // (par ^ 1) is rewritten only in the next pass, after the next cluster
+      // barrier, which no CTA passes before its reads of this pass are done.
+      cluster_sync();
+      if (warp == 0) {
         uint32_t local[8];
         uint32_t tot = 0;
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
-          local[j] = hist[8 * lane + j];
-          tot += local[j];
+          const uint32_t addr = smem_u32(&hist[par][8 * lane + j]);
+          uint32_t v = 0;
+          for (int r = 0; r < G; ++r) v += ld_dsmem_u32(mapa_shared(addr, static_cast<uint32_t>(r)));
+          local[j] = v;
+          tot += v;
         }
         uint32_t incl = tot;  // sum over lanes >= lane
 #pragma unroll
@@ -202,27 +207,34 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(TopkArgs a) {
       remaining = s_remaining;
       pmask |= 255u << shift;
       if (shift > 0 && s_count <= 32u) {
-        // Few routable keys share the digits found so far (the usual case
-        // for real-valued logits after one or two passes): gather them and
-        // let one warp rank them exactly instead of running the remaining
-        // passes.  The threshold is the candidate with fewer than
+        // At most 32 routable keys of the sequence share the digits found so
+        // far: each CTA publishes its share of them, and one warp per CTA
+        // ranks them all.  The threshold is the candidate with fewer than
         // `remaining` larger candidates and at least `remaining` larger or
         // equal ones; need_eq is what is left of `remaining` above it.
-        for (int i = a.r0 + tid; i < a.r1; i += blockDim.x) {
-          const uint32_t k = keys[i];
+        for (int i = rlo + tid; i < rhi; i += blockDim.x) {
+          const uint32_t k = keys[i - lo];
           if ((k & pmask) == prefix) s_cand[atomicAdd(&s_ncand, 1u)] = k;
         }
-        __syncthreads();
-        if (tid < 32) {
-          const uint32_t n = s_ncand;
-          const uint32_t k = tid < static_cast<int>(n) ? s_cand[tid] : 0u;
+        cluster_sync();
+        if (warp == 0) {
+          uint32_t k = 0, off = 0;
+          bool have = false;
+          for (int r = 0; r < G; ++r) {
+            const uint32_t n = ld_dsmem_u32(mapa_shared(smem_u32(&s_ncand), static_cast<uint32_t>(r)));
+            if (static_cast<uint32_t>(lane) >= off && static_cast<uint32_t>(lane) < off + n) {
+              k = ld_dsmem_u32(mapa_shared(smem_u32(&s_cand[lane - off]), static_cast<uint32_t>(r)));
+              have = true;
+            }
+            off += n;
+          }
           uint32_t gt = 0, ge = 0;
-          for (uint32_t j = 0; j < n; ++j) {
-            const uint32_t o = s_cand[j];
+          for (uint32_t j = 0; j < off; ++j) {
+            const uint32_t o = __shfl_sync(0xffffffffu, k, static_cast<int>(j));
             gt += o > k ? 1u : 0u;
             ge += o >= k ? 1u : 0u;
           }
-          if (tid < static_cast<int>(n) && gt < remaining && ge >= remaining) {
+          if (have && gt < remaining && ge >= remaining) {
             s_prefix = k;                 // lanes holding equal keys write equal values
             s_remaining = remaining - gt;
           }
@@ -237,65 +249,108 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(TopkArgs a) {
     need_eq = remaining;
   }
 
-  // 3. keep decisions in token order; ties to T ranked by index.  Warp w owns
-  // tokens [w * steps * 32, (w + 1) * steps * 32), 32 per step.
-  const int lane = tid & 31, warp = tid >> 5;
+  // 3. keep decisions in token order.  Warp w owns tokens
+  // [lo + w * steps * 32, lo + (w + 1) * steps * 32) of the CTA's range.
   const uint32_t lt = (1u << lane) - 1u;
-  const int steps = (N + blockDim.x - 1) / blockDim.x;
-  const int c0 = warp * steps * 32;
-  const bool select = !keep_all && !keep_none;
-  uint32_t eq_w = 0;
-  if (select) {
-    for (int st = 0; st < steps; ++st) {
-      const int i = c0 + st * 32 + lane;
-      const bool eq = i < N && i >= a.r0 && i < a.r1 && keys[i] == thr;
-      eq_w += __popc(__ballot_sync(0xffffffffu, eq));
-    }
-  }
-  uint32_t er = __shfl_sync(0xffffffffu, block_exclusive_scan(lane == 0 ? eq_w : 0u, warp_tot), 0);
-
-  uint32_t keep_w = 0;
+  const int steps = (a.chunk + blockDim.x - 1) / blockDim.x;
+  const int c0 = lo + warp * steps * 32;
+  uint32_t eq_w = 0, gt_w = 0;
   for (int st = 0; st < steps; ++st) {
     const int i = c0 + st * 32 + lane;
-    const bool valid = i < N;
+    const bool valid = i < hi;
     const bool routable = valid && i >= a.r0 && i < a.r1;
-    const uint32_t k = valid ? keys[i] : 0u;
+    const uint32_t k = valid ? keys[i - lo] : 0u;
     const bool eq = select && routable && k == thr;
-    const uint32_t eqb = __ballot_sync(0xffffffffu, eq);
-    const uint32_t rank = er + __popc(eqb & lt);
-    er += __popc(eqb);
-    bool keep;
-    if (!valid) keep = false;
-    else if (!routable || keep_all) keep = true;
-    else if (keep_none) keep = false;
-    else keep = k > thr || (eq && rank < need_eq);
-    const uint32_t kb = __ballot_sync(0xffffffffu, keep);
-    if (lane == 0) s_ballot[warp][st] = kb;
-    keep_w += __popc(kb);
+    const bool gt = valid && (!routable || keep_all || (select && k > thr));
+    eq_w += __popc(__ballot_sync(0xffffffffu, eq));
+    gt_w += __popc(__ballot_sync(0xffffffffu, gt));
   }
-  uint32_t pos = __shfl_sync(0xffffffffu, block_exclusive_scan(lane == 0 ? keep_w : 0u, warp_tot), 0);
+  if (lane == 0) {
+    w_eq[warp] = eq_w;
+    w_gt[warp] = gt_w;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    const uint32_t e = lane < kTopkWarps ? w_eq[lane] : 0u, g = lane < kTopkWarps ? w_gt[lane] : 0u;
+    const uint32_t ei = warp_inclusive_scan(e, lane), gi = warp_inclusive_scan(g, lane);
+    if (lane == kTopkWarps - 1) {
+      s_cnt[0] = ei;
+      s_cnt[1] = gi;
+    }
+  }
+  cluster_sync();   // every CTA's counts are published
+  if (warp == 0) {
+    // Ties and kept tokens before this CTA: CTA r takes
+    // clamp(need_eq - (ties before r), 0, ties of r) of its ties.
+    uint32_t er = 0, gr = 0;
+    if (lane < G) {
+      er = ld_dsmem_u32(mapa_shared(smem_u32(&s_cnt[0]), static_cast<uint32_t>(lane)));
+      gr = ld_dsmem_u32(mapa_shared(smem_u32(&s_cnt[1]), static_cast<uint32_t>(lane)));
+    }
+    const uint32_t eb = warp_inclusive_scan(er, lane) - er;
+    const uint32_t take = need_eq > eb ? min(need_eq - eb, er) : 0u;
+    const uint32_t kr = gr + take;
+    const uint32_t kb = warp_inclusive_scan(kr, lane) - kr;
+    const uint32_t eq_before = __shfl_sync(0xffffffffu, eb, rank);
+    const uint32_t keep_before = __shfl_sync(0xffffffffu, kb, rank);
+    // the same within this CTA, over its warps
+    const uint32_t e = lane < kTopkWarps ? w_eq[lane] : 0u, g = lane < kTopkWarps ? w_gt[lane] : 0u;
+    const uint32_t ewb = eq_before + warp_inclusive_scan(e, lane) - e;
+    const uint32_t wt = need_eq > ewb ? min(need_eq - ewb, e) : 0u;
+    const uint32_t wk = g + wt;
+    const uint32_t wkb = keep_before + warp_inclusive_scan(wk, lane) - wk;
+    if (lane < kTopkWarps) {
+      w_eq_off[lane] = ewb;
+      w_pos[lane] = wkb;
+    }
+  }
+  cluster_arrive();   // this CTA's reads of the others' shared memory are done
+  __syncthreads();
 
   const int k_tot = K + N - Nr;
   int32_t* idx = a.idx + static_cast<size_t>(b) * k_tot;
+  uint32_t er = w_eq_off[warp];
+  uint32_t pos = w_pos[warp];
   for (int st = 0; st < steps; ++st) {
     const int i = c0 + st * 32 + lane;
-    const uint32_t kb = s_ballot[warp][st];   // written by this warp's lane 0 (block scan barriers since)
-    const bool keep = (kb >> lane) & 1u;
+    const bool valid = i < hi;
+    const bool routable = valid && i >= a.r0 && i < a.r1;
+    const uint32_t k = valid ? keys[i - lo] : 0u;
+    const bool eq = select && routable && k == thr;
+    const uint32_t eqb = __ballot_sync(0xffffffffu, eq);
+    const uint32_t tie_rank = er + __popc(eqb & lt);
+    er += __popc(eqb);
+    const bool keep = valid && (!routable || keep_all || (select && (k > thr || (eq && tie_rank < need_eq))));
+    const uint32_t kb = __ballot_sync(0xffffffffu, keep);
     const uint32_t slot = pos + __popc(kb & lt);
     if (keep && slot < static_cast<uint32_t>(k_tot)) idx[slot] = i;
-    if (a.mask && i < N) a.mask[base + i] = keep ? 1 : 0;
+    if (a.mask && valid) a.mask[base + i] = keep ? 1 : 0;
     pos += __popc(kb);
   }
   if (tid == 0 && s_nan) record_status(a.status, CER_DEV_NAN);
+  cluster_wait();     // no CTA leaves while another may still read its shared memory
 }
 
-cudaError_t launch_topk(const TopkArgs& a, cudaStream_t stream) {
-  if (a.B == 0 || a.N == 0) return cudaSuccess;
-  const size_t smem = static_cast<size_t>(a.N) * sizeof(uint32_t);
-  // The limit is raised once per device to the largest N ever accepted.
+// Cluster size and tokens per CTA for sequences of N tokens.
+static void topk_split(int N, int* G, int* chunk) {
+  int g = (N + kTopkChunkTarget - 1) / kTopkChunkTarget;
+  g = g < 1 ? 1 : g > kTopkMaxCluster ? kTopkMaxCluster : g;
+  int c = (N + g - 1) / g;
+  c = (c + 31) / 32 * 32;
+  *G = g;
+  *chunk = c;
+}
+
+cudaError_t launch_topk(const TopkArgs& args, cudaStream_t stream) {
+  if (args.B == 0 || args.N == 0) return cudaSuccess;
+  TopkArgs a = args;
+  int G = 1;
+  topk_split(a.N, &G, &a.chunk);
+  const size_t smem = static_cast<size_t>(a.chunk) * sizeof(uint32_t);
+  // The limit is raised once per context to the largest chunk ever accepted.
   cudaError_t e = ensure_max_smem(reinterpret_cast<const void*>(topk_kernel), kTopkMaxN * sizeof(uint32_t));
   if (e != cudaSuccess) return e;
-  return launch_k(topk_kernel, dim3(a.B), dim3(kTopkThreads), smem, stream, 1, a);
+  return launch_k(topk_kernel, dim3(a.B * G), dim3(kTopkThreads), smem, stream, G, a);
 }
 
 }  // namespace cer

@@ -76,6 +76,22 @@ def out_err_ok(got_bf16: np.ndarray, exact: np.ndarray, tol_frac: float):
     return bool(np.all(excess <= 0)), float(excess.max()) if excess.size else 0.0
 
 
+# FFN and block outputs are compared with the oracle whose SwiGLU activation
+# enters the down projection as a bf16 operand (oracle routed_ffn(...,
+# act_bf16=True)), at the benchmark spec's bar: 2e-2 x RMS plus half a bf16 ulp.
+# What is left between the two sides is fp32 accumulation and the occasional
+# activation that each side rounds to a different neighbouring bf16 value
+# (the GPU rounds its fp32 value, the oracle its fp64 one): one such step of
+# a large activation times a large weight moves an output by ~2e-3, so a bar
+# much tighter than 2e-2 x RMS would test those flips, not the kernels.
+OUT_TOL = 2e-2
+
+
+def ffn_out_ok(got_bf16: np.ndarray, exact: np.ndarray):
+    """The output bar; returns (ok, worst excess over it)."""
+    return out_err_ok(got_bf16, exact, OUT_TOL)
+
+
 def rms(x) -> float:
     x = np.asarray(x, dtype=np.float64)
     return float(np.sqrt(np.mean(x ** 2))) if x.size else 0.0

@@ -10,7 +10,7 @@ import torch
 from oracle import cer_oracle as ora
 from paper_2608_29291_gb300 import cer
 from paper_2608_29291_gb300 import inputs as gen
-from tests.gpu_helpers import bf16_dev, bits_host, f32_dev, out_err_ok, scorers
+from tests.gpu_helpers import bf16_dev, bits_host, f32_dev, ffn_out_ok, out_err_ok, scorers
 
 pytestmark = pytest.mark.gpu
 OUT_TOL = 2e-2
@@ -46,8 +46,8 @@ def _check_gate(X, Wg, Wu, WdT, chan, delta, got_sal_perm, got_leak, got_flag, p
     if abs(lam - delta) > LEAK_TOL:
         assert got_flag == (1 if lam <= delta else 0)
     use = chan if got_flag == 1 else np.arange(Wg.shape[0])
-    want = ora.routed_ffn(X, Wg, Wu, WdT, use)
-    ok, excess = out_err_ok(ora.bf16_to_f64(Y_bits), want, OUT_TOL)
+    want = ora.routed_ffn(X, Wg, Wu, WdT, use, act_bf16=True)
+    ok, excess = ffn_out_ok(ora.bf16_to_f64(Y_bits), want)
     assert ok, excess
     return lam
 
@@ -118,6 +118,6 @@ def test_gated_block_matches_oracle(delta):
     exact = ora.bf16_to_f64(inp["h"]).copy()
     for b in range(w.B):
         exact[b, gi[b]] += ora.routed_ffn(ora.gather(inp["h"][b:b + 1], gi[b:b + 1]), inp["Wg"], inp["Wu"],
-                                          inp["WdT"], use)
-    ok, excess = out_err_ok(ora.bf16_to_f64(out), exact, OUT_TOL)
+                                          inp["WdT"], use, act_bf16=True)
+    ok, excess = ffn_out_ok(ora.bf16_to_f64(out), exact)
     assert ok, excess

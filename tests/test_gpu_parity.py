@@ -12,7 +12,8 @@ import torch
 from oracle import cer_oracle as ora
 from paper_2608_29291_gb300 import cer
 from paper_2608_29291_gb300 import inputs as gen
-from tests.gpu_helpers import SCORE_FLOOR, bf16_dev, bits_host, f32_dev, i32_dev, out_err_ok, rel_err, rms, scorers
+from tests.gpu_helpers import (SCORE_FLOOR, bf16_dev, bits_host, f32_dev, ffn_out_ok, i32_dev, out_err_ok, rel_err, rms,
+                               scorers)
 
 pytestmark = pytest.mark.gpu
 
@@ -159,6 +160,18 @@ def _score_case(name):
                    b1e=rng.normal(0, .1, (S, He)).astype(np.float32),
                    t=np.array([0.05, 0.3, 0.6, 0.999], np.float32))
         return inp, 1
+    if name in ("gen_wide_ragged", "und_wide_ragged"):
+        # 256-wide core and expansion scorers (Hc + He >= 512: the pair-MMA
+        # scorer, 256 flattened rows per tile): 2100 rows end in a ragged tile
+        # whose last warp straddles the end of h
+        gen_ = name.startswith("gen")
+        B, N, d, Hc, He, E = 3, 700, 1024, 512 if not gen_ else 256, 256, 64
+        inp = dict(h=bf((B, N, d), 1), W1=bf((Hc, d), d ** -.5), w2=rng.normal(0, Hc ** -.5, Hc).astype(np.float32),
+                   b1=rng.normal(0, .1, Hc).astype(np.float32), t=np.array([0.1, 0.5, 0.9], np.float32))
+        if gen_:
+            inp.update(W1e=bf((1, He, d), d ** -.5), w2e=rng.normal(0, He ** -.5, (1, He)).astype(np.float32),
+                       Ue=bf((1, He, E), E ** -.5), b1e=None)
+        return inp, 1 if gen_ else 0
     raise KeyError(name)
 
 
@@ -167,7 +180,8 @@ def _oracle_logits(inp, task):
                      inp.get("w2e"), inp.get("Ue"), inp.get("b1e"))
 
 
-@pytest.mark.parametrize("name", ["tiny", "und_ragged_bias", "und_odd_d", "gen_segments", "gen_segments_noU"])
+@pytest.mark.parametrize("name", ["tiny", "und_ragged_bias", "und_odd_d", "gen_segments", "gen_segments_noU",
+                                  "gen_wide_ragged", "und_wide_ragged"])
 def test_score_matches_oracle(name):
     inp, task = _score_case(name)
     B, N, d = inp["h"].shape
@@ -203,8 +217,8 @@ def test_routed_ffn_matches_oracle(M, d, I, C, pruned):
     Y = torch.empty((M, d), dtype=torch.bfloat16, device="cuda")
     cer.cer_routed_ffn(bf16_dev(X), bf16_dev(Wg), bf16_dev(Wu), bf16_dev(WdT), i32_dev(chan), Y)
     cer.cer_sync_status()
-    want = ora.routed_ffn(X, Wg, Wu, WdT, chan if pruned else np.arange(I))
-    ok, excess = out_err_ok(ora.bf16_to_f64(bits_host(Y)), want, OUT_TOL)
+    want = ora.routed_ffn(X, Wg, Wu, WdT, chan if pruned else np.arange(I), act_bf16=True)
+    ok, excess = ffn_out_ok(ora.bf16_to_f64(bits_host(Y)), want)
     assert ok, excess
 
 
@@ -288,9 +302,9 @@ def _check_block(w, inp, res, rows=None):
     b_of = rows // w.k_tot
     tok = res["idx"].reshape(-1)[rows]
     X = h[b_of, tok]
-    y = ora.routed_ffn(X, inp["Wg"], inp["Wu"], inp["WdT"], inp["chan"])
+    y = ora.routed_ffn(X, inp["Wg"], inp["Wu"], inp["WdT"], inp["chan"], act_bf16=True)
     exact = ora.bf16_to_f64(X) + y
-    ok, excess = out_err_ok(ora.bf16_to_f64(res["out"][b_of, tok]), exact, OUT_TOL)
+    ok, excess = ffn_out_ok(ora.bf16_to_f64(res["out"][b_of, tok]), exact)
     assert ok, excess
 
 

@@ -304,6 +304,27 @@ def test_ffn_dense_matches_torch_swiglu():
     assert np.allclose(Y, want.numpy(), rtol=1e-12, atol=1e-12)
 
 
+def test_ffn_bf16_activation_matches_torch():
+    """The bf16-operand activation: torch's SiLU in fp64, its fp32 -> bf16
+    conversions (round to nearest even), then an fp64 contraction, agree with
+    the oracle's act_bf16 path to fp64 rounding; and the rounding changes the
+    result (so the flag is not ignored)."""
+    rng = np.random.default_rng(12)
+    M, d, I = 9, 32, 40
+    X = gen.f32_to_bf16_bits(rng.normal(0, 2, (M, d)).astype(np.float32))
+    Wg, Wu, WdT = (gen.f32_to_bf16_bits(rng.normal(0, 0.3, (I, d)).astype(np.float32)) for _ in range(3))
+    chan = np.arange(0, I, 2)
+    x = _T(X)
+    g = x @ _T(Wg[chan]).T
+    u = x @ _T(Wu[chan]).T
+    a = (F.silu(g) * u).float().bfloat16().double()
+    want = (a @ _T(WdT[chan])).numpy()
+    got = ora.routed_ffn(X, Wg, Wu, WdT, chan, act_bf16=True)
+    assert np.max(np.abs(got - want)) < 1e-12 * max(1.0, np.max(np.abs(want)))
+    exact = ora.routed_ffn(X, Wg, Wu, WdT, chan)
+    assert np.max(np.abs(got - exact)) > 1e-6
+
+
 def test_ffn_pruned_equals_dense_with_removed_channels_zeroed():
     rng = np.random.default_rng(9)
     M, d, I = 9, 16, 32
@@ -397,6 +418,7 @@ def _all_pin_failures():
         test_block_full_keep_equals_dense_block()
         test_block_invariants()
         test_sigmoid_values()
+        test_ffn_bf16_activation_matches_torch()
     except AssertionError as e:
         f.append(str(e))
     return f
@@ -413,12 +435,14 @@ MUTATIONS = {
     "ties_to_higher_index": ("select_topk", lambda orig: (
         lambda lg, r0, r1, K: _reverse_ties(orig, lg, r0, r1, K))),
     "down_not_transposed": ("routed_ffn", lambda orig: (
-        lambda X, Wg, Wu, WdT, chan: _ffn_wrong_down(X, Wg, Wu, WdT, chan))),
+        lambda X, Wg, Wu, WdT, chan, **kw: _ffn_wrong_down(X, Wg, Wu, WdT, chan))),
     "silu_without_gate": ("routed_ffn", lambda orig: (
-        lambda X, Wg, Wu, WdT, chan: _ffn_no_silu(X, Wg, Wu, WdT, chan))),
+        lambda X, Wg, Wu, WdT, chan, **kw: _ffn_no_silu(X, Wg, Wu, WdT, chan))),
     "bias_sign": ("mlp_score", lambda orig: (lambda x, W1, w2, bias: orig(x, W1, w2, -bias))),
     "sigmoid_tanh_scale": ("sigmoid", lambda orig: (lambda x: 0.5 * (1 + np.tanh(np.asarray(x, np.float64))))),
     "sigmoid_offset": ("sigmoid", lambda orig: (lambda x: orig(np.asarray(x, np.float64) + 0.01))),
+    "act_bf16_truncated": ("round_to_bf16", lambda orig: (
+        lambda x: (np.asarray(x, np.float64).astype(np.float32).view(np.uint32) >> np.uint32(16)).astype(np.uint16))),
 }
 
 
