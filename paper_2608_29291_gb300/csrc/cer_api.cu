@@ -312,6 +312,21 @@ cudaError_t ensure_max_smem(const void* func, size_t bytes) {
   return e;
 }
 
+cudaError_t prefer_max_shared(const void* func) {
+  static std::mutex mu;
+  static std::set<std::pair<unsigned long long, const void*>> done;
+  const unsigned long long ctx = current_context_id();
+  std::lock_guard<std::mutex> lk(mu);
+  if (ctx != 0 && done.count({ctx, func})) return cudaSuccess;
+  cudaError_t e = cudaFuncSetAttribute(func, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                       static_cast<int>(cudaSharedmemCarveoutMaxShared));
+  if (e == cudaSuccess) {
+    const unsigned long long now = current_context_id();
+    if (now != 0) done.insert({now, func});
+  }
+  return e;
+}
+
 }  // namespace cer
 
 // ---------------------------------------------------------------- the ABI

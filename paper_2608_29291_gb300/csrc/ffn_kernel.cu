@@ -87,6 +87,7 @@ struct GateUpProblemT {
   // from rank 1's; every copy counts on the even CTA's barrier.  `part`
   // selects the activation copy, the weight copy or both (kPart*).
   __device__ static bool weights_first(const Params&) { return true; }
+  __device__ static bool acts_first(const Params&) { return false; }   // X comes from the row gather
   __device__ static void prod_kb(const Params& p, const ProdState& st, int, int kb, int lane, uint8_t* a,
                                  uint8_t* b, uint32_t leader_bar, int part) {
     if (lane == 0) {
@@ -226,6 +227,7 @@ struct DownProblem {
   // The K extent may come from a device flag the previous kernel writes (the
   // UCS gate); only without it may the weights go out before that kernel ends.
   __device__ static bool weights_first(const Params& p) { return p.use_small_k == nullptr; }
+  __device__ static bool acts_first(const Params&) { return false; }   // act comes from the gate/up GEMM
   __device__ static void prod_kb(const Params& p, const ProdState& st, int, int kb, int lane, uint8_t* a,
                                  uint8_t* b, uint64_t* bar, int part) {
     if (lane == 0) {

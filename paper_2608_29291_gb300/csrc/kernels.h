@@ -28,9 +28,17 @@ bool encode_bf16_col_blocks(CUtensorMap* map, const void* base, uint64_t rows, u
 // Launch `kernel` with programmatic dependent launch allowed (and a cluster
 // dimension when cluster_x > 1): it may start while the previous kernel on
 // the stream finishes; its griddep_wait() orders it after that kernel.
+// Every kernel of this library prefers the largest shared-memory carveout,
+// so the SMs keep one configuration and a kernel with large shared memory
+// (the GEMMs) can be resident beside a small one that runs before it (an SM
+// whose carveout must change has to drain first).  Set once per context.
+cudaError_t prefer_max_shared(const void* func);
+
 template <typename... KArgs, typename... Args>
 inline cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
                             int cluster_x, Args&&... args) {
+  cudaError_t e = prefer_max_shared(reinterpret_cast<const void*>(kernel));
+  if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = grid;
   cfg.blockDim = block;
@@ -143,6 +151,7 @@ struct TopkArgs {
   uint8_t* mask;         // nullable
   int* status;
   int chunk;             // tokens per CTA of a sequence's cluster (set by launch_topk)
+  int vec4;              // the partial rows may be read as float4 (set by launch_topk)
 };
 constexpr int kTopkMaxN = 49152;
 cudaError_t launch_topk(const TopkArgs& a, cudaStream_t stream);

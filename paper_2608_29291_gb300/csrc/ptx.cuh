@@ -174,6 +174,15 @@ __device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t b
       : "memory");
 }
 
+// Plain bulk copy of `bytes` (a multiple of 16, both addresses 16-byte
+// aligned) from this CTA's shared memory to global memory, tracked by the
+// thread's bulk async group (bulk_commit_group / bulk_wait_group*).
+__device__ __forceinline__ void bulk_store(void* dst, const void* src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(reinterpret_cast<uint64_t>(dst)),
+               "r"(smem_u32(src)), "r"(bytes)
+               : "memory");
+}
+
 // Order this thread's earlier generic-proxy accesses to global memory (such
 // as an acquire of a flag) before its later async-proxy (bulk copy) accesses.
 __device__ __forceinline__ void fence_proxy_async_global() {

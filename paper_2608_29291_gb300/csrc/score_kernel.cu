@@ -24,9 +24,13 @@ namespace cer {
 
 // bias_tab[b][j], w2_tab[b][j] for the concatenated hidden index j in
 // [0, Hc + He): core columns take b1 and w2; expansion columns take
-// U[m] emb(t_b) + b1e[m] and w2e[m] with m = m(t_b).  Grid (B, Ht/8): each
-// block builds emb(t_b) in shared memory, then each of its 8 warps owns one
-// column and reduces its U row across the lanes (coalesced reads).
+// U[m] emb(t_b) + b1e[m] and w2e[m] with m = m(t_b).  Grid (B, nb), nb about
+// the SM count over B: each block builds emb(t_b) in shared memory, then its
+// 8 warps take the sequence's columns in turn, one column per warp at a time,
+// reducing its U row across the lanes (coalesced reads).  About one block per
+// SM leaves the registers of every SM to the scorer's CTAs, which start as
+// soon as this kernel has: their copies and MMAs do not depend on it, only
+// their epilogues read the tables.
 //
 // emb_j = cos / sin(1000 t f_j).  FP64 transcendentals are very slow on this
 // part, so the argument is formed in turns -- x = (1000 t) * f_j / (2 pi), one
@@ -34,11 +38,35 @@ namespace cer {
 // (x - rint(x), |r| <= 1/2), and only then handed to the fp32 sincospif.  The
 // result differs from the fp64 sinusoid by about 2e-7 before it is rounded
 // to fp32.
-constexpr int kBiasColsPerBlock = 8;
+constexpr int kBiasWarps = 8;
 
-__global__ void __launch_bounds__(32 * kBiasColsPerBlock) time_bias_kernel(ScoreArgs a,
-                                                                           const __grid_constant__ EmbFreqTable ft,
-                                                                           float* bias_tab, float* w2_tab) {
+__device__ __forceinline__ void bias_column(const ScoreArgs& a, const float* emb, int m, int b, int j, int Ht,
+                                            int lane, float* bias_tab, float* w2_tab) {
+  float bias, w2;
+  if (j < a.Hc) {
+    bias = a.b1 ? a.b1[j] : 0.f;
+    w2 = a.w2[j];
+  } else {
+    const int jj = j - a.Hc;
+    float s = 0.f;
+    if (a.U != nullptr) {
+      const __nv_bfloat16* u = a.U + (static_cast<size_t>(m) * a.He + jj) * a.E;
+      for (int e = lane; e < a.E; e += 32) s = fmaf(__bfloat162float(u[e]), emb[e], s);
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
+    }
+    bias = (a.b1e ? a.b1e[static_cast<size_t>(m) * a.He + jj] : 0.f) + s;
+    w2 = a.w2e[static_cast<size_t>(m) * a.He + jj];
+  }
+  if (lane == 0) {
+    bias_tab[static_cast<size_t>(b) * Ht + j] = bias;
+    w2_tab[static_cast<size_t>(b) * Ht + j] = w2;
+  }
+}
+
+__global__ void __launch_bounds__(32 * kBiasWarps) time_bias_kernel(ScoreArgs a,
+                                                                    const __grid_constant__ EmbFreqTable ft,
+                                                                    float* bias_tab, float* w2_tab) {
   griddep_wait();
   griddep_launch_dependents();
   extern __shared__ float emb[];
@@ -65,28 +93,14 @@ __global__ void __launch_bounds__(32 * kBiasColsPerBlock) time_bias_kernel(Score
     }
   }
   __syncthreads();
-  const int j = blockIdx.y * kBiasColsPerBlock + warp;
-  if (j >= Ht) return;
-  float bias, w2;
-  if (j < a.Hc) {
-    bias = a.b1 ? a.b1[j] : 0.f;
-    w2 = a.w2[j];
-  } else {
-    const int jj = j - a.Hc;
-    float s = 0.f;
-    if (a.U != nullptr) {
-      const __nv_bfloat16* u = a.U + (static_cast<size_t>(m) * a.He + jj) * a.E;
-      for (int e = lane; e < a.E; e += 32) s = fmaf(__bfloat162float(u[e]), emb[e], s);
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
-    }
-    bias = (a.b1e ? a.b1e[static_cast<size_t>(m) * a.He + jj] : 0.f) + s;
-    w2 = a.w2e[static_cast<size_t>(m) * a.He + jj];
+  const int step = gridDim.y * kBiasWarps;
+  // two columns per round, their loads in flight together
+  int j = blockIdx.y * kBiasWarps + warp;
+  for (; j + step < Ht; j += 2 * step) {
+    bias_column(a, emb, m, b, j, Ht, lane, bias_tab, w2_tab);
+    bias_column(a, emb, m, b, j + step, Ht, lane, bias_tab, w2_tab);
   }
-  if (lane == 0) {
-    bias_tab[static_cast<size_t>(b) * Ht + j] = bias;
-    w2_tab[static_cast<size_t>(b) * Ht + j] = w2;
-  }
+  if (j < Ht) bias_column(a, emb, m, b, j, Ht, lane, bias_tab, w2_tab);
 }
 
 // ---------------------------------------------------------------- scorer GEMM
@@ -140,6 +154,7 @@ struct ScoreProblem {
     int* status;
     int B, N, d, S, He, Ht;
     int n_rt, n_core, n_chunks;
+    int acts_first;      // the previous kernel (the bias-table kernel) writes no h
   };
   struct ProdState {
     int b, rt, chunk, wrow;
@@ -170,6 +185,7 @@ struct ScoreProblem {
   // With several expansion segments the weight rows depend on t, which a
   // previous kernel may write; with one, the weights may go out first.
   __device__ static bool weights_first(const Params& p) { return p.S <= 1; }
+  __device__ static bool acts_first(const Params& p) { return p.acts_first != 0; }
   __device__ static uint32_t stage_bytes(const Params&, int, int, int part) {
     return ((part & kPartAct) ? kATileBytes : 0u) + ((part & kPartWeights) ? BN * 128u : 0u);
   }
@@ -251,6 +267,7 @@ struct ScorePairProblem {
     int* status;
     int rows, N, d, Ht;      // rows = B * N
     int n_rp, n_core, n_chunks;
+    int acts_first;          // the previous kernel (the bias-table kernel) writes no h
   };
   struct ProdState {
     int m0, wrow, core;
@@ -260,6 +277,7 @@ struct ScorePairProblem {
   __device__ static int num_tiles(const Params& p) { return p.n_rp * p.n_chunks; }
   __device__ static int num_kb(const Params& p) { return p.d / 64; }
   __device__ static bool weights_first(const Params&) { return true; }
+  __device__ static bool acts_first(const Params& p) { return p.acts_first != 0; }
   __device__ static uint32_t stage_bytes(const Params&, int, int, int part) {
     return 2 * (((part & kPartAct) ? kATileBytes : 0u) + ((part & kPartWeights) ? kBoxBytes : 0u));
   }
@@ -392,6 +410,7 @@ static cudaError_t launch_score_gemm(const ScoreArgs& a, const float* bias_tab, 
   p.n_rt = (a.N + 127) / 128;
   p.n_core = a.Hc / BN;
   p.n_chunks = Ht / BN;
+  p.acts_first = bias_tab != nullptr;   // generation: right behind the bias-table kernel
   return launch_gemm<P>(p, a.B * p.n_rt * p.n_chunks, a.d / 64, nullptr, n_sm, stream);
 }
 
@@ -428,6 +447,7 @@ static cudaError_t launch_score_pair(const ScoreArgs& a, const float* bias_tab, 
   p.n_rp = static_cast<int>((rows + 255) / 256);
   p.n_core = a.Hc / 256;
   p.n_chunks = Ht / 256;
+  p.acts_first = bias_tab != nullptr;   // generation: right behind the bias-table kernel
   return launch_gemm<P>(p, p.n_rp * p.n_chunks, a.d / 64, sk, n_sm, stream);
 }
 
@@ -459,8 +479,12 @@ cudaError_t launch_score(const ScoreArgs& a, const ScoreWorkspace& ws, const Str
   const int half = (a.gen && a.U) ? a.E / 2 : 0;
   for (int j = 0; j < half; ++j) ft.g[j] = std::pow(10000.0, -static_cast<double>(j) / half) / (2.0 * M_PI);
   for (int j = half; j < 512; ++j) ft.g[j] = 0.0;
-  const dim3 bias_grid(a.B, (Ht + kBiasColsPerBlock - 1) / kBiasColsPerBlock);
-  cudaError_t e = launch_k(time_bias_kernel, bias_grid, dim3(32 * kBiasColsPerBlock), emb_bytes, stream, 1, a, ft,
+  int nb = (n_sm + a.B - 1) / a.B;
+  const int max_nb = (Ht + kBiasWarps - 1) / kBiasWarps;
+  if (nb > max_nb) nb = max_nb;
+  if (nb < 1) nb = 1;
+  const dim3 bias_grid(a.B, nb);
+  cudaError_t e = launch_k(time_bias_kernel, bias_grid, dim3(32 * kBiasWarps), emb_bytes, stream, 1, a, ft,
                            ws.bias_tab, ws.w2_tab);
   if (e != cudaSuccess) return e;
   return launch_score_chunks(a, ws.bias_tab, ws.w2_tab, ws.partial, sk, n_sm, stream, n_partials);

@@ -2,8 +2,10 @@
 // Eq. 6 (Sec. 3.4), computed exactly on the fp32 logits (the sigmoid is
 // monotonic, App. B.2).
 //
-// A sequence is handled by a cluster of G <= 8 CTAs (G chosen so each CTA
-// holds at most ~1024 tokens; G = 1 for short sequences), CTA `rank` owning
+// A sequence is handled by a cluster of G <= 8 CTAs (G = 1 up to 4096
+// tokens, else enough CTAs for about 4096 tokens each: measured on GB300, the
+// cluster barriers and remote reads cost more than they save below that),
+// CTA `rank` owning
 // the tokens [rank * chunk, (rank + 1) * chunk).  Each CTA keeps the
 // order-preserving 32-bit keys of its tokens in shared memory (reducing the
 // scorer's partial sums, in chunk order, into the logits on the way).  An
@@ -35,7 +37,7 @@ constexpr int kTopkThreads = 512;
 constexpr int kTopkWarps = kTopkThreads / 32;
 constexpr int kTopkMaxCluster = 8;
 // Tokens per CTA the cluster size aims at.
-constexpr int kTopkChunkTarget = 1024;
+constexpr int kTopkChunkTarget = 4096;
 
 // Monotone map from fp32 to uint32: a > b (as floats) iff key(a) > key(b);
 // -0.0 is mapped like +0.0.
@@ -49,48 +51,81 @@ __device__ __forceinline__ uint32_t order_key(float v) {
 // contention of logits that share a few digit values; merged after each pass.
 constexpr int kSubHist = 8;
 
-// Tokens a thread reduces at once in the logits pass (their partial-sum loads
-// are in flight together).
-constexpr int kLoadUnroll = 4;
-
 // Logits of tokens [lo, hi) from the scorer's partial sums, summed in chunk
-// order, into the order keys: a thread takes U tokens at a time and reads
-// their partial rows eight at a time, so up to 8U loads are in flight.
-template <int U>
-__device__ __forceinline__ void reduce_logits(const TopkArgs& a, size_t base, int lo, int hi, uint32_t* keys,
-                                              int* s_nan) {
-  for (int i0 = lo + threadIdx.x; i0 < hi; i0 += U * blockDim.x) {
-    float v[U];
+// order, into the order keys; the routable keys are counted into pass 0's
+// histogram (their top byte) on the way.  Vector form: a thread takes 4
+// consecutive tokens, one float4 of each partial row, eight rows' loads in
+// flight at once; it needs lo, the sequence base and the row stride to be
+// multiples of 4 (checked by the caller).  The kernel runs once per step from
+// a cold instruction cache, so its loops are kept short rather than unrolled.
+__device__ __forceinline__ void key_out(const TopkArgs& a, size_t base, int lo, int i, float v, uint32_t* keys,
+                                        uint32_t* hist0, bool count, int* s_nan) {
+  if (a.logits_out) a.logits_out[base + i] = v;
+  if (a.probs_out) a.probs_out[base + i] = 1.0f / (1.0f + expf(-v));
+  const bool routable = i >= a.r0 && i < a.r1;
+  if (routable && v != v) *s_nan = 1;
+  const uint32_t k = order_key(v);
+  keys[i - lo] = k;
+  if (count && routable) atomicAdd(&hist0[k >> 24], 1u);
+}
+
+__device__ __forceinline__ float4 sum_partials4(const TopkArgs& a, const float4* src, size_t stride4, int q) {
+  float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 1
+  for (int c0 = 0; c0 < a.n_chunks; c0 += 8) {
+    float4 part[8];
 #pragma unroll
-    for (int u = 0; u < U; ++u) v[u] = 0.f;
-    for (int c0 = 0; c0 < a.n_chunks; c0 += 8) {
-      float part[U][8];
-      // Every load in bounds (token and chunk clamped), so all 8U go out
-      // back to back; the clamped ones are not used.
+    for (int c = 0; c < 8; ++c) part[c] = __ldg(src + static_cast<size_t>(min(c0 + c, a.n_chunks - 1)) * stride4 + q);
 #pragma unroll
-      for (int u = 0; u < U; ++u) {
-        const int i = min(i0 + u * static_cast<int>(blockDim.x), hi - 1);
-#pragma unroll
-        for (int c = 0; c < 8; ++c) {
-          const int cc = min(c0 + c, a.n_chunks - 1);
-          part[u][c] = __ldg(a.src + static_cast<size_t>(cc) * a.chunk_stride + base + i);
-        }
+    for (int c = 0; c < 8; ++c) {
+      if (c0 + c >= a.n_chunks) break;
+      if (c0 + c == 0) {
+        v = part[c];
+      } else {
+        v.x += part[c].x;
+        v.y += part[c].y;
+        v.z += part[c].z;
+        v.w += part[c].w;
       }
-#pragma unroll
-      for (int u = 0; u < U; ++u)
-#pragma unroll
-        for (int c = 0; c < 8; ++c)
-          if (c0 + c < a.n_chunks) v[u] = (c0 + c == 0) ? part[u][c] : v[u] + part[u][c];
     }
+  }
+  return v;
+}
+
+__device__ __forceinline__ void reduce_logits_vec4(const TopkArgs& a, size_t base, int lo, int hi, uint32_t* keys,
+                                                   uint32_t* hist0, bool count, int* s_nan) {
+  const int q_hi = (hi + 3) / 4;
+  const float4* src = reinterpret_cast<const float4*>(a.src + base);
+  const size_t stride4 = a.chunk_stride / 4;
+#pragma unroll 1
+  for (int q = lo / 4 + threadIdx.x; q < q_hi; q += 2 * blockDim.x) {
+    // two groups of 4 tokens: both groups' loads go out before either is summed
+    const int q2 = min(q + static_cast<int>(blockDim.x), q_hi - 1);
+    const float4 v0 = sum_partials4(a, src, stride4, q);
+    const float4 v1 = sum_partials4(a, src, stride4, q2);
 #pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int i = i0 + u * blockDim.x;
-      if (i >= hi) break;
-      if (a.logits_out) a.logits_out[base + i] = v[u];
-      if (a.probs_out) a.probs_out[base + i] = 1.0f / (1.0f + expf(-v[u]));
-      if (i >= a.r0 && i < a.r1 && v[u] != v[u]) *s_nan = 1;
-      keys[i - lo] = order_key(v[u]);
+    for (int g = 0; g < 2; ++g) {
+      const int qq = g == 0 ? q : q + blockDim.x;
+      if (qq >= q_hi) break;
+      const float4 v = g == 0 ? v0 : v1;
+      const int i = 4 * qq;
+      key_out(a, base, lo, i, v.x, keys, hist0, count, s_nan);
+      if (i + 1 < hi) key_out(a, base, lo, i + 1, v.y, keys, hist0, count, s_nan);
+      if (i + 2 < hi) key_out(a, base, lo, i + 2, v.z, keys, hist0, count, s_nan);
+      if (i + 3 < hi) key_out(a, base, lo, i + 3, v.w, keys, hist0, count, s_nan);
     }
+  }
+}
+
+// Scalar form for rows whose layout does not allow the vector loads.
+__device__ __forceinline__ void reduce_logits_scalar(const TopkArgs& a, size_t base, int lo, int hi, uint32_t* keys,
+                                                  uint32_t* hist0, bool count, int* s_nan) {
+#pragma unroll 1
+  for (int i = lo + threadIdx.x; i < hi; i += blockDim.x) {
+    float v = __ldg(a.src + base + i);
+#pragma unroll 1
+    for (int c = 1; c < a.n_chunks; ++c) v += __ldg(a.src + static_cast<size_t>(c) * a.chunk_stride + base + i);
+    key_out(a, base, lo, i, v, keys, hist0, count, s_nan);
   }
 }
 
@@ -126,19 +161,6 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(TopkArgs a) {
   const int lo = rank * a.chunk;
   const int hi = min(N, lo + a.chunk);         // hi <= lo: this CTA holds no token
   const size_t base = static_cast<size_t>(b) * N;
-  if (tid == 0) {
-    s_nan = 0;
-    s_ncand = 0;
-  }
-  __syncthreads();
-
-  // 1. logits (reduced from partial sums in chunk order) -> keys
-  if (hi - lo >= 2 * static_cast<int>(blockDim.x)) {
-    reduce_logits<kLoadUnroll>(a, base, lo, hi, keys, &s_nan);
-  } else {
-    reduce_logits<1>(a, base, lo, hi, keys, &s_nan);
-  }
-
   const int Nr = a.r1 - a.r0;
   const int K = a.K;
   const bool keep_all = (K == Nr);
@@ -146,21 +168,38 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(TopkArgs a) {
   const bool select = !keep_all && !keep_none;
   const int rlo = max(lo, a.r0), rhi = min(hi, a.r1);   // this CTA's routable tokens
   uint32_t thr = 0, need_eq = 0;
+  if (tid == 0) {
+    s_nan = 0;
+    s_ncand = 0;
+  }
+  for (int i = tid; i < kSubHist * 256; i += blockDim.x) (&sub[0][0])[i] = 0;
+  __syncthreads();
+
+  // 1. logits (reduced from partial sums in chunk order) -> keys, with pass
+  // 0's histogram (top byte) of the routable keys
+  uint32_t* my = sub[warp % kSubHist];
+  if (a.vec4) {
+    reduce_logits_vec4(a, base, lo, hi, keys, my, select, &s_nan);
+  } else {
+    reduce_logits_scalar(a, base, lo, hi, keys, my, select, &s_nan);
+  }
+  __syncthreads();
 
   // 2. radix select of the K-th largest routable key (every CTA of the
   // cluster takes the same branches: they all see the same histograms)
   if (select) {
     uint32_t prefix = 0, pmask = 0, remaining = static_cast<uint32_t>(K);
-    for (int i = tid; i < kSubHist * 256; i += blockDim.x) (&sub[0][0])[i] = 0;
-    __syncthreads();
     int par = 0;
+#pragma unroll 1
     for (int shift = 24; shift >= 0; shift -= 8, par ^= 1) {
-      uint32_t* my = sub[warp % kSubHist];
-      for (int i = rlo + tid; i < rhi; i += blockDim.x) {
-        const uint32_t k = keys[i - lo];
-        if ((k & pmask) == prefix) atomicAdd(&my[(k >> shift) & 255u], 1u);
+      if (shift < 24) {   // pass 0 was counted with the keys
+#pragma unroll 1
+        for (int i = rlo + tid; i < rhi; i += blockDim.x) {
+          const uint32_t k = keys[i - lo];
+          if ((k & pmask) == prefix) atomicAdd(&my[(k >> shift) & 255u], 1u);
+        }
+        __syncthreads();
       }
-      __syncthreads();
       for (int i = tid; i < 256; i += blockDim.x) {
         uint32_t c = 0;
 #pragma unroll
@@ -175,16 +214,24 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(TopkArgs a) {
       // barrier, which no CTA passes before its reads of this pass are done.
       cluster_sync();
       if (warp == 0) {
+        // The lane's 8 bins: its own CTA's counts, plus every other CTA's,
+        // read through distributed shared memory with all loads of a CTA
+        // issued before any is added (each one takes a round trip).
         uint32_t local[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) local[j] = hist[par][8 * lane + j];
+        const uint32_t addr = smem_u32(&hist[par][8 * lane]);
+        for (int r = 1; r < G; ++r) {
+          const uint32_t remote = mapa_shared(addr, static_cast<uint32_t>((rank + r) % G));
+          uint32_t v[8];
+#pragma unroll
+          for (int j = 0; j < 8; ++j) v[j] = ld_dsmem_u32(remote + 4u * j);
+#pragma unroll
+          for (int j = 0; j < 8; ++j) local[j] += v[j];
+        }
         uint32_t tot = 0;
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          const uint32_t addr = smem_u32(&hist[par][8 * lane + j]);
-          uint32_t v = 0;
-          for (int r = 0; r < G; ++r) v += ld_dsmem_u32(mapa_shared(addr, static_cast<uint32_t>(r)));
-          local[j] = v;
-          tot += v;
-        }
+        for (int j = 0; j < 8; ++j) tot += local[j];
         uint32_t incl = tot;  // sum over lanes >= lane
 #pragma unroll
         for (int off = 1; off < 32; off <<= 1) {
@@ -218,15 +265,19 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(TopkArgs a) {
         }
         cluster_sync();
         if (warp == 0) {
-          uint32_t k = 0, off = 0;
+          // lane r < G reads CTA r's candidate count; a prefix over the lanes
+          // gives each candidate's place; lane l then fetches candidate l.
+          const uint32_t nr = lane < G ? ld_dsmem_u32(mapa_shared(smem_u32(&s_ncand), static_cast<uint32_t>(lane))) : 0u;
+          const uint32_t before = warp_inclusive_scan(nr, lane) - nr;
+          const uint32_t off = __shfl_sync(0xffffffffu, before + nr, G - 1);   // all candidates
+          uint32_t k = 0;
           bool have = false;
           for (int r = 0; r < G; ++r) {
-            const uint32_t n = ld_dsmem_u32(mapa_shared(smem_u32(&s_ncand), static_cast<uint32_t>(r)));
-            if (static_cast<uint32_t>(lane) >= off && static_cast<uint32_t>(lane) < off + n) {
-              k = ld_dsmem_u32(mapa_shared(smem_u32(&s_cand[lane - off]), static_cast<uint32_t>(r)));
+            const uint32_t br = __shfl_sync(0xffffffffu, before, r), n = __shfl_sync(0xffffffffu, nr, r);
+            if (static_cast<uint32_t>(lane) >= br && static_cast<uint32_t>(lane) < br + n) {
+              k = ld_dsmem_u32(mapa_shared(smem_u32(&s_cand[lane - br]), static_cast<uint32_t>(r)));
               have = true;
             }
-            off += n;
           }
           uint32_t gt = 0, ge = 0;
           for (uint32_t j = 0; j < off; ++j) {
@@ -333,7 +384,7 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(TopkArgs a) {
 
 // Cluster size and tokens per CTA for sequences of N tokens.
 static void topk_split(int N, int* G, int* chunk) {
-  int g = (N + kTopkChunkTarget - 1) / kTopkChunkTarget;
+  int g = N <= kTopkChunkTarget ? 1 : (N + kTopkChunkTarget - 1) / kTopkChunkTarget;
   g = g < 1 ? 1 : g > kTopkMaxCluster ? kTopkMaxCluster : g;
   int c = (N + g - 1) / g;
   c = (c + 31) / 32 * 32;
@@ -346,6 +397,7 @@ cudaError_t launch_topk(const TopkArgs& args, cudaStream_t stream) {
   TopkArgs a = args;
   int G = 1;
   topk_split(a.N, &G, &a.chunk);
+  a.vec4 = (a.N % 4 == 0) && (a.chunk_stride % 4 == 0) && (reinterpret_cast<uintptr_t>(a.src) % 16 == 0);
   const size_t smem = static_cast<size_t>(a.chunk) * sizeof(uint32_t);
   // The limit is raised once per context to the largest chunk ever accepted.
   cudaError_t e = ensure_max_smem(reinterpret_cast<const void*>(topk_kernel), kTopkMaxN * sizeof(uint32_t));

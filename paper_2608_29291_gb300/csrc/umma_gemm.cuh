@@ -87,6 +87,7 @@
 //   weights_first(p): true when num_tiles, num_kb, prod_tile and the weight
 //   copies read nothing a previous kernel may write, so the weight producer
 //   need not wait for that kernel to finish,
+//   acts_first(p): the same for the activation copies,
 //   stage_bytes(p, tile, kb, part) (the bytes of the selected copies of one
 //   K block; with MMA_PAIR, of both CTAs),
 //   bdesc(saddr), prefetch(p) (prefetches the tensor maps' descriptors),
@@ -184,11 +185,16 @@ struct SplitPlan {
 
 constexpr int kMaxSplit = 4;
 
-inline SplitPlan stream_k_plan(int tiles, int nkb, int slots) {
+//   - balance_waves (the tensor-bound pair scorer, whose tiles are few and
+//     long): whenever the tiles fill at least one wave but not a whole number
+//     of them, the last full wave and the remainder are split, so every slot
+//     takes the same number of K blocks.
+inline SplitPlan stream_k_plan(int tiles, int nkb, int slots, bool balance_waves = false) {
   const SplitPlan whole{tiles < slots ? tiles : slots, tiles};
   if (slots <= 1 || tiles <= 0) return whole;
   const int q = tiles / slots;
   const int r = tiles % slots;
+  if (balance_waves && q > 0 && r > 0) return SplitPlan{slots, (q - 1) * slots};
   if (q == 0) {
     if (2 * tiles > slots) return whole;
     const int s = tiles * kMaxSplit < slots ? tiles * kMaxSplit : slots;
@@ -358,8 +364,16 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1)
   // that when a kernel starts, the kernels two or more launches back have
   // completed -- which is what makes weights written there safe to read
   // without the wait.
+  // The activation producer (and, when neither operand waits, the MMA
+  // issuer, which reads no global memory) likewise skip it when the previous
+  // kernel writes nothing the activation copies read (acts_first: the
+  // scorer behind the generation bias-table kernel); the epilogue always
+  // waits.
   const bool weights_first = P::weights_first(p);
-  if (warp != 2 || !weights_first) {
+  const bool acts_first = P::acts_first(p);
+  const bool skip_wait = (warp == 2 && weights_first) || (warp == 0 && acts_first) ||
+                         (warp == 1 && weights_first && acts_first);
+  if (!skip_wait) {
     griddep_wait();
     griddep_launch_dependents();
   }
@@ -634,7 +648,7 @@ inline unsigned long long next_stream_k_token() {
 // be resident at once; with a stream-K region the tiles may be split.
 template <class P>
 cudaError_t launch_gemm(const typename P::Params& p, int tiles, int nkb, const StreamKArea* area, int n_sm,
-                        cudaStream_t stream) {
+                        cudaStream_t stream, bool balance_waves = false) {
   if (tiles == 0) return cudaSuccess;
   const size_t smem = gemm_smem_bytes<P>();
   cudaError_t e = ensure_max_smem(reinterpret_cast<const void*>(umma_gemm_kernel<P>), smem);
@@ -669,7 +683,7 @@ cudaError_t launch_gemm(const typename P::Params& p, int tiles, int nkb, const S
   StreamK sk{};
   SplitPlan plan{tiles < slots ? tiles : slots, tiles};
   if (area != nullptr && area->partial != nullptr && area->flags != nullptr) {
-    const SplitPlan split = stream_k_plan(tiles, nkb, slots);
+    const SplitPlan split = stream_k_plan(tiles, nkb, slots, balance_waves);
     const size_t partial = static_cast<size_t>(split.slots) * P::CLUSTER * 128 * P::BN * sizeof(float);
     const size_t flags = static_cast<size_t>(split.slots) * P::CLUSTER * (P::EPI_WARPS / 4) * sizeof(unsigned long long);
     if (split.dp_tiles < tiles && partial <= kStreamKPartialBytes && flags <= kStreamKFlagBytes) {
