@@ -58,6 +58,7 @@ struct GateUpProblemT {
   static constexpr uint32_t kBStepBytes = 32;
   static constexpr uint32_t kBoxBytes = 128 * 128;          // 128 rows x 64 bf16
   static constexpr uint32_t kEpiSmemBytes = 2 * kBoxBytes;  // the act tile as two TMA boxes
+  static constexpr uint32_t kEpiZeroBytes = 0;
 
   struct Params {
     CUtensorMap tm_x;    // X [M, d], box 64 x 128
@@ -184,6 +185,7 @@ struct DownProblem {
   static constexpr uint32_t kBStepBytes = 2048;     // 16 K-rows = two 1024 B row groups
   static constexpr uint32_t kAtomBytes = 64 * 128;  // 64 K-rows x 64 columns
   static constexpr uint32_t kEpiSmemBytes = 0;
+  static constexpr uint32_t kEpiZeroBytes = 0;
   static_assert(CTA_N % 64 == 0, "whole 64-column B atoms per CTA");
 
   struct Params {

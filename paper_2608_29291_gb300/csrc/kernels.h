@@ -123,7 +123,7 @@ struct EmbFreqTable {
 struct ScoreWorkspace {
   float* bias_tab;  // [B][Hc + He]
   float* w2_tab;    // [B][Hc + He]
-  float* partial;   // [n_partials][B*N], n_partials <= 2 * (Hc + He) / 64
+  float* partial;   // [n_partials][B*N], n_partials = (Hc + He) / chunk width <= (Hc + He) / 64
 };
 
 // Largest hidden-chunk width the scorer may use for these widths (0: none).

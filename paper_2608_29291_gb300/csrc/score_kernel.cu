@@ -6,8 +6,9 @@
 // chunks.  A work tile is (sequence b, 128-token row tile, hidden chunk); its
 // epilogue adds the per-sequence bias column (b1, or U emb(t_b) + b1e for the
 // expansion), applies the exact-erf GELU in fp32 and folds the chunk into a
-// per-token partial score w2 . GELU(.); each half of the chunk's columns
-// (one per group of four epilogue warps) writes partial[2*chunk + half][b*N + n].
+// per-token partial score w2 . GELU(.), partial[chunk][b*N + n]: two groups of
+// four epilogue warps each fold half the chunk's columns and the second group
+// to finish a row adds the two halves.
 // The partial scores are summed in chunk order by the consumer (the reduce
 // kernel below, or the top-K kernel in the fused block), so the logits do not
 // depend on scheduling.
@@ -129,6 +130,30 @@ __device__ __forceinline__ float gelu_as(float x) {
   return x * phi;
 }
 
+// The two epilogue groups fold disjoint column halves of the same accumulator
+// rows (warps w and w + 4 read the same TMEM lanes); whichever finishes a row
+// second adds the halves, half 0's sum on the left (fp32 addition of two
+// terms does not depend on their order either way).  Per accumulator buffer
+// there is one sum slot per half and row and one arrival counter per row.
+// A buffer's slots come round again two tiles later, after both groups have
+// released that buffer; the counters only grow (an odd prior count marks the
+// second arrival), so nothing waits and nothing is reset.  Returns whether
+// this thread holds the row's chunk score in *out.
+constexpr uint32_t kHalfSumBytes = 2 * 2 * 128 * 4;
+constexpr uint32_t kHalfCountBytes = 2 * 128 * 4;
+__device__ __forceinline__ bool combine_halves(const EpiCtx& ctx, int row, int half, float s, float* out) {
+  volatile float* sum = reinterpret_cast<volatile float*>(ctx.smem) + ctx.acc * 256;   // [half][row]
+  uint32_t* cnt = reinterpret_cast<uint32_t*>(ctx.smem + kHalfSumBytes) + ctx.acc * 128;
+  sum[half * 128 + row] = s;
+  __threadfence_block();
+  const uint32_t prior = atomicAdd(&cnt[row], 1u);
+  if ((prior & 1u) == 0u) return false;
+  __threadfence_block();
+  const float other = sum[(half ^ 1) * 128 + row];
+  *out = half == 0 ? s + other : other + s;
+  return true;
+}
+
 template <int BN_>
 struct ScoreProblem {
   static constexpr int BN = BN_;
@@ -139,7 +164,8 @@ struct ScoreProblem {
   static constexpr int B_MN_MAJOR = 0;
   static constexpr int EPI_WARPS = 8;
   static constexpr uint32_t kBStepBytes = 32;
-  static constexpr uint32_t kEpiSmemBytes = 0;
+  static constexpr uint32_t kEpiSmemBytes = kHalfSumBytes + kHalfCountBytes;
+  static constexpr uint32_t kEpiZeroBytes = kEpiSmemBytes;
 
   struct Params {
     CUtensorMap tm_h;    // h as [B*N, d], box 64 x 128
@@ -205,7 +231,7 @@ struct ScoreProblem {
   }
 
   __device__ static void epilogue_done(const Params&, int, int) {}
-  __device__ static bool epilogue(const Params& p, int tile, int row, int half, uint32_t taddr, EpiCtx&) {
+  __device__ static bool epilogue(const Params& p, int tile, int row, int half, uint32_t taddr, EpiCtx& ctx) {
     int b, rt, chunk;
     decode(p, tile, b, rt, chunk);
     const float* bias = p.bias_tab ? p.bias_tab + static_cast<size_t>(b) * p.Ht + chunk * BN
@@ -228,7 +254,9 @@ struct ScoreProblem {
       }
     }
     const int n = rt * 128 + row;
-    if (n < p.N) p.partial[static_cast<size_t>(2 * chunk + half) * p.B * p.N + static_cast<size_t>(b) * p.N + n] = s;
+    float score;
+    if (combine_halves(ctx, row, half, s, &score) && n < p.N)
+      p.partial[static_cast<size_t>(chunk) * p.B * p.N + static_cast<size_t>(b) * p.N + n] = score;
     return true;
   }
 };
@@ -252,7 +280,8 @@ struct ScorePairProblem {
   static constexpr int B_MN_MAJOR = 0;
   static constexpr int EPI_WARPS = 8;
   static constexpr uint32_t kBStepBytes = 32;
-  static constexpr uint32_t kEpiSmemBytes = 0;
+  static constexpr uint32_t kEpiSmemBytes = kHalfSumBytes + kHalfCountBytes;
+  static constexpr uint32_t kEpiZeroBytes = kEpiSmemBytes;
   static constexpr uint32_t kBoxBytes = 128 * 128;   // 128 weight rows x 64 bf16
 
   struct Params {
@@ -330,7 +359,8 @@ struct ScorePairProblem {
         s = fmaf(ww.w, gelu_as(v[4 * q + 3] + bb.w), s);
       }
     }
-    if (valid) p.partial[static_cast<size_t>(2 * chunk + half) * p.rows + grow] = s;
+    float score;
+    if (combine_halves(ctx, row, half, s, &score) && valid) p.partial[static_cast<size_t>(chunk) * p.rows + grow] = score;
     return true;
   }
 };
@@ -361,7 +391,7 @@ int score_chunk_width(int Hc, int He, int gen) {
 
 int score_max_partials(int Hc, int He, int gen) {
   if (score_chunk_width(Hc, He, gen) == 0) return 0;
-  return 2 * (Hc + (gen ? He : 0)) / 64;
+  return (Hc + (gen ? He : 0)) / 64;
 }
 
 // Chunk width for a launch: the widest whose tiles fill at least ~90% of a
@@ -457,11 +487,11 @@ static cudaError_t launch_score_chunks(const ScoreArgs& a, const float* bias_tab
                                        float* partial, const StreamKArea* sk, int n_sm, cudaStream_t stream,
                                        int* n_partials) {
   if (use_pair_scorer(a)) {
-    *n_partials = 2 * (a.Hc + (a.gen ? a.He : 0)) / 256;
+    *n_partials = (a.Hc + (a.gen ? a.He : 0)) / 256;
     return launch_score_pair(a, bias_tab, w2_tab, partial, sk, n_sm, stream);
   }
   const int bn = pick_chunk_width(a, n_sm);
-  *n_partials = bn ? 2 * (a.Hc + (a.gen ? a.He : 0)) / bn : 0;
+  *n_partials = bn ? (a.Hc + (a.gen ? a.He : 0)) / bn : 0;
   switch (bn) {
     case 256: return launch_score_gemm<256>(a, bias_tab, w2_tab, partial, n_sm, stream);
     case 128: return launch_score_gemm<128>(a, bias_tab, w2_tab, partial, n_sm, stream);

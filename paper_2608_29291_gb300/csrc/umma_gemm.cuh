@@ -92,12 +92,16 @@
 //   K block; with MMA_PAIR, of both CTAs),
 //   bdesc(saddr), prefetch(p) (prefetches the tensor maps' descriptors),
 //   kEpiSmemBytes (shared memory reserved for the epilogue, may be 0),
+//   kEpiZeroBytes (how much of it, from its start, is zeroed before any
+//   thread starts its role),
 //   epilogue(p, tile, row, half, taddr, ctx) -> false to abort (ctx.rank is
 //   the CTA's rank in its cluster): columns
 //   [half*BN/H, (half+1)*BN/H) of accumulator row `row` (H = EPI_WARPS/4
 //   groups of four warps), taddr addressing
-//   column 0 of that row's lanes, ctx the reserved shared memory and a
-//   bounded barrier over the 128 threads of the half;
+//   column 0 of that row's lanes, ctx the reserved shared memory, a
+//   bounded barrier over the 128 threads of the half and the accumulator
+//   buffer (0 or 1) the tile is in -- that buffer's next tile is delivered
+//   only after every epilogue thread has returned from this one;
 //   epilogue_done(p, row, half): once, after the last tile.
 #pragma once
 
@@ -272,6 +276,7 @@ struct EpiCtx {
   uint32_t phase;
   volatile int* abort_flag;
   int* status;
+  int acc = 0;   // the tile's TMEM accumulator buffer
   __device__ __forceinline__ bool sync() {
     mbar_arrive(half_bar);
     const bool ok = mbar_wait(half_bar, phase, abort_flag, status);
@@ -338,6 +343,9 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1)
     *abort_flag = 0;
     fence_mbar_init();
   }
+  static_assert(P::kEpiZeroBytes <= P::kEpiSmemBytes && P::kEpiZeroBytes % 4 == 0, "zeroed epilogue smem");
+  for (uint32_t i = threadIdx.x; i < P::kEpiZeroBytes / 4; i += blockDim.x)
+    reinterpret_cast<uint32_t*>(epi_smem)[i] = 0u;
   if (warp == 1) {
     if (PAIR) {
       tmem_alloc_pair(tmem_slot, TMEM_COLS);   // together with warp 1 of the peer CTA
@@ -596,6 +604,7 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1)
             if (ok && row == 0) st_relaxed_u64(flag, 0ull);
           }
         }
+        ctx.acc = acc;
         if (ok) ok = P::epilogue(p, tile, row, half, taddr, ctx);
       }
       tc_fence_before();

@@ -46,10 +46,10 @@ def _r256(x):
 
 
 def test_workspace_sizes(lib):
-    # scorer: bias + w2 tables [B][Ht] and at most 2*Ht/64 partial-score rows of B*N
-    assert lib.cer_score_workspace_size(4, 1024, 256, 0, 0) == 2 * 4096 + 8 * 4 * 1024 * 4
-    assert lib.cer_score_workspace_size(2, 4096, 512, 512, 1) == 2 * 8192 + 32 * 2 * 4096 * 4
-    assert lib.cer_score_workspace_size(1, 256, 64, 64, 1) == 2 * 512 + 4 * 256 * 4
+    # scorer: bias + w2 tables [B][Ht] and at most Ht/64 partial-score rows of B*N
+    assert lib.cer_score_workspace_size(4, 1024, 256, 0, 0) == 2 * 4096 + 4 * 4 * 1024 * 4
+    assert lib.cer_score_workspace_size(2, 4096, 512, 512, 1) == 2 * 8192 + 16 * 2 * 4096 * 4
+    assert lib.cer_score_workspace_size(1, 256, 64, 64, 1) == 2 * 512 + 2 * 256 * 4
     assert lib.cer_score_workspace_size(1, 10, 100, 0, 0) == 0          # hidden not a multiple of 64
     # FFN: act [M, C] bf16, plus three [C, d] slices when a channel list is packed per call
     sk = (24 << 20) + 8192     # stream-K partial accumulators and flags of the GEMMs

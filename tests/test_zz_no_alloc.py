@@ -51,8 +51,8 @@ def test_static_scratch_scorer_matches_workspace_scorer_twice():
 def test_static_scratch_refuses_sizes_beyond_its_capacity():
     lib = cer.load()
     fake = ctypes.c_void_p(1 << 20)
-    core = cer.CerScorerC(fake.value, None, fake.value, None, 1024, 0, 1)
-    # B*N = 65536 tokens x 32 partial rows x 4 bytes = 8 MiB of partial scores > 4 MiB
+    core = cer.CerScorerC(fake.value, None, fake.value, None, 2048, 0, 1)
+    # B*N = 65536 tokens x 32 partial rows (hidden 2048 / 64) x 4 bytes = 8 MiB of partial scores > 4 MiB
     st = lib.cer_score_static(fake, 4, 16384, 1536, ctypes.pointer(core), None, None, 0, fake, None, None)
     assert st == 9, lib.cer_get_error()
     assert b"static scratch holds 4194304 bytes" in lib.cer_get_error()
