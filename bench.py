@@ -463,6 +463,8 @@ def stage_report(w: gen.Workload, stage_ms, peaks) -> dict:
         bound = "tensor" if t_tc > t_hbm else "hbm"
         r = {"us": round(t * 1e6, 2), "bound": bound, "frac": round(max(t_hbm, t_tc) / t, 4) if t > 0 else None,
              "gbs": round(nbytes / t / 1e9, 1) if t > 0 else None}
+        if bound == "hbm" and t > 0:
+            r["frac_vs_8tbs"] = round(nbytes / NOMINAL_HBM_BPS / t, 4)   # the nominal HBM3e figure
         if flops:
             r["tflops"] = round(flops / t / 1e12, 1) if t > 0 else None
         out[name] = r
@@ -472,6 +474,26 @@ def stage_report(w: gen.Workload, stage_ms, peaks) -> dict:
     out["ffn"] = {"us": round(t_ffn * 1e6, 2), "bound": "tensor" if ffn_f / pk > ffn_b / bw else "hbm",
                   "frac": round(max(ffn_f / pk, ffn_b / bw) / t_ffn, 4), "tflops": round(ffn_f / t_ffn / 1e12, 1)}
     return out
+
+
+NOMINAL_HBM_BPS = 8.0e12   # GB300 HBM3e, nominal (the stages' "frac" uses the measured copy bandwidth)
+
+
+def stage_floor_us(torch, cer, stream, reps=60):
+    """The floor every serialised stage carries: two events on the stream with
+    one near-empty library kernel between them (a bounded wait on an mbarrier
+    phase that the kernel completes itself), median over `reps`."""
+    ts = []
+    for i in range(reps):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda._sleep(20000)   # keeps the host ahead, so no launch latency is timed
+        a.record(stream)
+        cer.cer_selftest_bounded_wait(1, arrive=True, limit_us=1000, stream=stream)
+        b.record(stream)
+        ts.append((a, b))
+    torch.cuda.synchronize()
+    cer.cer_sync_status(stream)
+    return float(np.median([a.elapsed_time(b) * 1e3 for a, b in ts[reps // 6:]]))
 
 
 SWEEP_N = (1024, 2048, 4096, 8192, 16384)
@@ -566,6 +588,7 @@ def run_gpu(args, info):
     slow_ms = runtime.max_over_ranks(dist, mean_ms, device=dev)
     tokens = w.B * w.N * info.world
     value = tokens / (slow_ms * 1e-3)
+    floor_us = round(stage_floor_us(torch, cer, stream), 2)
 
     # ---- end to end through the public API: pinned host h in, h out.  Every
     # step uploads its own h (and t) from pinned host memory, runs the block,
@@ -734,6 +757,10 @@ def run_gpu(args, info):
         "stage_peaks": f"hbm_gbs and bf16_tflops (burst) of {peak_kind}",
         "gpu_launches": kernels_per_step(w.task) * args.steps,
         "stage_pass": f"per-stage times from a separate pass of {n_stage} steps with events between kernels",
+        "stage_floor_us": {"value": floor_us,
+                           "what": "median time between two events with one near-empty library kernel between "
+                                   "them: the event and launch cost each serialised stage carries on top of its "
+                                   "kernels (the overlapped step does not pay it)"},
         "clocks": clocks.summary(),
     }
     print(json.dumps(line), flush=True)
