@@ -344,8 +344,10 @@ __global__ void __launch_bounds__(gemm_threads<P>(), 1)
     fence_mbar_init();
   }
   static_assert(P::kEpiZeroBytes <= P::kEpiSmemBytes && P::kEpiZeroBytes % 4 == 0, "zeroed epilogue smem");
-  for (uint32_t i = threadIdx.x; i < P::kEpiZeroBytes / 4; i += blockDim.x)
-    reinterpret_cast<uint32_t*>(epi_smem)[i] = 0u;
+  if constexpr (P::kEpiZeroBytes > 0) {
+    for (uint32_t i = threadIdx.x; i < P::kEpiZeroBytes / 4; i += blockDim.x)
+      reinterpret_cast<uint32_t*>(epi_smem)[i] = 0u;
+  }
   if (warp == 1) {
     if (PAIR) {
       tmem_alloc_pair(tmem_slot, TMEM_COLS);   // together with warp 1 of the peer CTA
