@@ -302,7 +302,10 @@ struct ScorePairProblem {
     int m0, wrow, core;
   };
 
-  // Cluster tile t: row pair t % n_rp (rows 256 (t % n_rp) + 128 rank ..), chunk t / n_rp.
+  // Cluster tile t: row pair t / n_chunks (rows 256 (t / n_chunks) + 128 rank ..), chunk t % n_chunks.
+  // The chunks of a row pair are consecutive tiles, so they run side by side
+  // and read the pair's rows of h from L2 while they are there (chunk-major
+  // order measured 56.5 against 54.2 us at long_7b).
   __device__ static int num_tiles(const Params& p) { return p.n_rp * p.n_chunks; }
   __device__ static int num_kb(const Params& p) { return p.d / 64; }
   __device__ static bool weights_first(const Params&) { return true; }
@@ -311,8 +314,8 @@ struct ScorePairProblem {
     return 2 * (((part & kPartAct) ? kATileBytes : 0u) + ((part & kPartWeights) ? kBoxBytes : 0u));
   }
   __device__ static void prod_tile(const Params& p, int tile, int rank, ProdState& st) {
-    const int chunk = tile / p.n_rp;
-    st.m0 = (2 * (tile % p.n_rp) + rank) * 128;   // rows past B*N load as zeros
+    const int chunk = tile % p.n_chunks;
+    st.m0 = (2 * (tile / p.n_chunks) + rank) * 128;   // rows past B*N load as zeros
     st.core = chunk < p.n_core;
     st.wrow = (st.core ? chunk : chunk - p.n_core) * BN + rank * 128;
   }
@@ -333,8 +336,8 @@ struct ScorePairProblem {
 
   __device__ static void epilogue_done(const Params&, int, int) {}
   __device__ static bool epilogue(const Params& p, int tile, int row, int half, uint32_t taddr, EpiCtx& ctx) {
-    const int chunk = tile / p.n_rp;
-    const int grow = (2 * (tile % p.n_rp) + ctx.rank) * 128 + row;
+    const int chunk = tile % p.n_chunks;
+    const int grow = (2 * (tile / p.n_chunks) + ctx.rank) * 128 + row;
     // Rows past B*N (the ragged last tile) still take part in every tensor
     // memory load -- tcgen05.ld is warp-collective (.sync.aligned) -- and
     // only skip the store; their bias and w2 come from the last sequence.
