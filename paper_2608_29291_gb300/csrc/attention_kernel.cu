@@ -46,7 +46,8 @@ constexpr int kRopeThreads = 256;   // 8 warps, one packed row per warp at a tim
 // a = pos * theta_j is formed in turns, x = pos * g_j with g_j = theta_j /
 // (2 pi) from the host's fp64 table, reduced exactly in fp64 (x - rint(x))
 // and handed to fp32 sincospif: accurate to ~2e-7 for any position, where an
-// fp32 product pos * theta_j would lose the angle.
+// fp32 product pos * theta_j would lose the angle.  (A two-part fp32 form of
+// the reduction measured slower than these eight fp64 products per row.)
 __global__ void __launch_bounds__(kRopeThreads)
     rope_kernel(__nv_bfloat16* qkv, long long rows, int Hq, int Hkv, const int32_t* __restrict__ pos,
                 const __grid_constant__ RopeFreqTable ft, int* status) {
@@ -62,6 +63,10 @@ __global__ void __launch_bounds__(kRopeThreads)
     __nv_bfloat16* r = qkv + row * width;
     // Heads lane/8, lane/8 + 4, ... in batches of four: a batch's loads are
     // issued before the angles (and the previous batch's stores) are needed.
+    // The angles depend on the row and the lane's pairs only: they are formed
+    // once, after the first batch's loads (fp64 is slow on this part).
+    float c[8], s[8];
+    bool have_angles = false;
     for (int h0 = lane >> 3; h0 < heads; h0 += 16) {
       uint4 lo[4], hi[4];
 #pragma unroll
@@ -73,11 +78,13 @@ __global__ void __launch_bounds__(kRopeThreads)
         }
       }
       if (p < 0) break;
-      float c[8], s[8];
+      if (!have_angles) {
 #pragma unroll
-      for (int e = 0; e < 8; ++e) {
-        const double x = static_cast<double>(p) * ft.g[j0 + e];
-        sincospif(2.0f * static_cast<float>(x - rint(x)), &s[e], &c[e]);
+        for (int e = 0; e < 8; ++e) {
+          const double x = static_cast<double>(p) * ft.g[j0 + e];
+          sincospif(2.0f * static_cast<float>(x - rint(x)), &s[e], &c[e]);
+        }
+        have_angles = true;
       }
 #pragma unroll
       for (int i = 0; i < 4; ++i) {

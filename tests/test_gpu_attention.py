@@ -77,6 +77,30 @@ def test_rope_matches_oracle(B, L, Hq, Hkv, N):
     assert np.array_equal(bits_host(qkv)[:, n_rot:], bits[:, n_rot:])      # value heads untouched
 
 
+def test_rope_at_large_positions():
+    """Positions up to 2^31 - 1, where an fp32 product of position and
+    frequency would have lost the angle entirely."""
+    Hq, Hkv = 4, 2
+    pos = np.array([[0, 1, 4095, (1 << 24) - 3, (1 << 24) - 1, 1 << 24, (1 << 24) + 5, 123456789, (1 << 30) + 7,
+                     (1 << 31) - 1]], dtype=np.int32)
+    B, L = pos.shape
+    bits = _qkv(77, B, L, Hq, Hkv)
+    qkv = bf16_dev(bits)
+    cer.cer_rope_packed(qkv, B, L, Hq, Hkv, i32_dev(pos.reshape(-1)), 1e6)
+    cer.cer_sync_status()
+    got = ora.bf16_to_f64(bits_host(qkv))
+    x = ora.bf16_to_f64(bits)
+    q, k, v = _split(x, Hq, Hkv)
+    p = pos.reshape(-1)
+    want = np.concatenate([ora.rope(q, p, 1e6).reshape(B * L, -1), ora.rope(k, p, 1e6).reshape(B * L, -1)], axis=1)
+    n_rot = (Hq + Hkv) * DH
+    xr = x[:, :n_rot].reshape(B * L, Hq + Hkv, 2, DH // 2)
+    norm = np.sqrt(xr[:, :, 0] ** 2 + xr[:, :, 1] ** 2)
+    bound = ulp_bf16(want) + 1e-6 * np.concatenate([norm, norm], axis=2).reshape(B * L, n_rot)
+    err = np.abs(got[:, :n_rot] - want)
+    assert np.all(err <= bound), float(np.max(err / bound))
+
+
 def test_rope_negative_position_reported():
     bits = _qkv(5, 1, 4, 2, 1)
     qkv = bf16_dev(bits)
