@@ -89,7 +89,8 @@ __global__ void __launch_bounds__(kDropThreads) drop_stats_kernel(const uint8_t*
 // four K steps of loads in flight per lane): 56 warps, so B = 2 sequences of
 // 4096 tokens (54 rows per SM) take one round of rows; at 40 registers six
 // blocks fitted and a seventh ran as a second round (ncu: 31.4 us cold for
-// 117 MB, 49 % of DRAM).  The gap measured 48.5 -> 45.0 us with the change.
+// 117 MB, 49 % of DRAM; the whole gap at that shape 48.5 us, against 45.0 us
+// with seven).
 __global__ void __launch_bounds__(kStatThreads, 7) row_cosine_kernel(const uint4* __restrict__ h_in,
                                                                    const uint4* __restrict__ h_out, int d8,
                                                                    long rows, float* __restrict__ cosv) {
